@@ -36,8 +36,10 @@ design notes):
 
 ``mirror=True`` rounds to bfloat16 (round to nearest, ties to even) at the
 points where the bf16 storage path stores a value: LN(v) (R1), k and u (R2),
-LN(h) + E_dep (R3), q (R4), r before the fusion (R6), the SiLU activations
-(R7) and h_hat (R8).  ``mirror=False`` is exact float64 throughout.
+LN(h) + E_dep (R3), r before the fusion (R6), the SiLU activations (R7) and
+h_hat (R8).  The query q is not rounded: the bf16 path carries it as a pair
+of bf16 values (about 16 significant bits), so its scores follow the exact
+q.  ``mirror=False`` is exact float64 throughout.
 
 Parity pins: tests/test_oracle_pins.py (bf16 rounding against torch, LN/RMSNorm
 against torch.nn.functional, subset enumeration, closed forms, dense
@@ -151,7 +153,7 @@ def query(p, h, depth, *, mirror=False, ln_eps=1e-5):
     """q_n = W_Q (LN(h_n) + E_dep[l_n])."""
     x = _maybe(layer_norm(h, p["ln_h_gamma"], p["ln_h_beta"], ln_eps)
                + p["E_dep"][np.asarray(depth)], mirror)
-    return _maybe(x @ p["W_Q"].T, mirror)
+    return x @ p["W_Q"].T
 
 
 def scores(q_n, K_b, d, row_scale_n=1.0):

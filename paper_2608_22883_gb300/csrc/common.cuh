@@ -1,0 +1,173 @@
+// Shared device helpers and internal launch interfaces of libfovea.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fovea.h"
+
+namespace fovea {
+
+// Sticky device error bits (workspace / memory error word).
+enum : int { kErrDepth = 1, kErrTimeout = 2 };
+
+// ---------------------------------------------------------------------------
+// Scalar conversions
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <class T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+  return __float2bfloat16_rn(x);
+}
+
+__device__ __forceinline__ float sigmoidf_(float z) { return 1.0f / (1.0f + expf(-z)); }
+
+// ---------------------------------------------------------------------------
+// Reductions (fixed order, so results are run-to-run deterministic)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Block-wide sum / max; `scratch` holds >= 32 floats.  Every thread returns
+// the result.  Contains __syncthreads().
+__device__ __forceinline__ float block_sum(float v, float* scratch) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) scratch[warp] = v;
+  __syncthreads();
+  float t = lane < nw ? scratch[lane] : 0.0f;
+  return warp_sum(t);
+}
+__device__ __forceinline__ float block_max(float v, float* scratch) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_max(v);
+  __syncthreads();
+  if (lane == 0) scratch[warp] = v;
+  __syncthreads();
+  float t = lane < nw ? scratch[lane] : -INFINITY;
+  return warp_max(t);
+}
+
+// ---------------------------------------------------------------------------
+// Per-call tables passed by value as kernel parameters
+// ---------------------------------------------------------------------------
+
+// One independent sub-problem of a GEMM C = A . B^T: output rows are B rows
+// (draft states / tokens), output columns are A rows (features / keys).
+struct GemmGroup {
+  int a_row0;        // first A row of this group
+  int m;             // A rows (output columns) in this group
+  int b_row0;        // first B row of this group
+  int n;             // B rows (output rows) in this group
+  long long c_off;   // output element offset (grouped epilogues)
+};
+
+enum EpiKind : int {
+  kEpiStore = 0,      // out{0,1}[row * ldc + col] = T(acc), columns split at epi_split
+  kEpiScores = 1,     // out0 (fp32)[c_off + n * m + col] = acc * scale * row_scale[row]
+  kEpiBiasSilu = 2,   // out0[row * ldc + col] = T(silu(acc + bias{0,1}[col]))
+  kEpiBiasF32 = 3,    // out0 (fp32)[row * ldc + col] = acc + bias0[col]
+  kEpiStoreHiLo = 4,  // out0 = T(acc), out1 = T(acc - out0): acc carried as two stored values
+  kEpiStoreKeys = 5,  // kEpiStore, and columns < epi_split whose acc lies near a bf16
+                      // rounding midpoint are listed for an exact recomputation
+};
+
+struct KeyFix {       // one listed key element: memory row, feature
+  int row, col;
+};
+
+struct GemmArgs {
+  int k_total;        // contraction length (multiple of 64)
+  int a_split;        // A rows >= a_split come from A1 (row - a_split)
+  int b_split;        // contraction index >= b_split comes from B1 (k - b_split)
+  int dual_b;         // tensor-core scores: B0 and B1 are the hi / lo parts of one
+                      // operand, both multiplied by the same A tile
+  // raw operands (SIMT path; the tensor-core path uses tensor maps)
+  const void* A0; const void* A1; long long lda0, lda1;
+  const void* B0; const void* B1; long long ldb0, ldb1;
+  // epilogue
+  int epi_split;
+  void* out0; void* out1; long long ldc;
+  const void* bias0; const void* bias1;
+  const float* row_scale; float scale;
+  KeyFix* fix_list; int* fix_count; int fix_cap;   // kEpiStoreKeys
+  int* err;
+  int ngroups;
+  GemmGroup groups[FOVEA_MAX_SEQ];
+};
+
+// Per-sequence view of one retrieve_fuse call.
+struct SeqTable {
+  int B;
+  int row_start[FOVEA_MAX_SEQ + 1];
+  int key_off[FOVEA_MAX_SEQ];
+  int m[FOVEA_MAX_SEQ];
+  long long score_off[FOVEA_MAX_SEQ];
+};
+
+__device__ __forceinline__ int seq_of_row(const SeqTable& t, int row) {
+  int lo = 0, hi = t.B - 1;
+  while (lo < hi) {                    // last b with row_start[b] <= row
+    int mid = (lo + hi + 1) >> 1;
+    if (t.row_start[mid] <= row) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launch interfaces (defined in the kernel translation units)
+// ---------------------------------------------------------------------------
+
+cudaError_t launch_ln_rows(int dtype, const void* x, const int32_t* src_row, int rows, int d,
+                           const void* gamma, const void* beta, float eps, const void* E,
+                           const int32_t* depth, int max_depth, int* err, void* out,
+                           cudaStream_t s);
+cudaError_t launch_count_valid(const uint8_t* mask, int B, int M_max, int32_t* counts,
+                               cudaStream_t s);
+cudaError_t launch_compact(const uint8_t* mask, int B, int M_max, const int32_t* key_off,
+                           int32_t* orig_index, int32_t* src_row, cudaStream_t s);
+cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
+                          float rho, int k_min, int k_max, int max_m, int32_t* counts,
+                          int32_t* indices, int32_t* sel_pos, float* sel_w, int32_t* sel_cnt,
+                          cudaStream_t s);
+cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, const int32_t* sel_pos,
+                           const float* sel_w, int N, int k_max, int d, float* r_out, void* r_lo,
+                           cudaStream_t s);
+// Exact rounding of listed key elements: k = sum_l x[row, l] W[col, l]
+// evaluated in double-float, rounded once to bf16.  list == nullptr refines
+// every element of the [rows, d] key matrix.
+cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
+                               const int* count, int cap, int rows, void* K, cudaStream_t s);
+cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,
+                            const void* w_g2, const void* b_g2, const void* rms_gamma, float eps,
+                            int N, void* h_out, float* gate_out, cudaStream_t s);
+
+// GEMM C = A . B^T with a chosen epilogue.  `tc` selects the tcgen05 path
+// (bf16 only); otherwise the SIMT path (fp32 and bf16).
+// max_m / max_n bound the per-group extents (grid size).
+cudaError_t launch_gemm_simt(int dtype, int epi, const GemmArgs& a, int max_m, int max_n,
+                             cudaStream_t s);
+
+struct TmaOperand {     // a row-major [rows, cols] bf16 matrix with a row stride
+  const void* base;
+  long long rows, cols, ld;   // ld in elements
+};
+cudaError_t launch_gemm_tc(int epi, const GemmArgs& a, const TmaOperand& A0, const TmaOperand& A1,
+                           const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
+                           cudaStream_t s);
+
+}  // namespace fovea

@@ -368,8 +368,11 @@ def test_mirror_rounds_at_the_storage_points():
     for k in mem.keys + mem.values:
         np.testing.assert_array_equal(k, oracle.round_bf16(k))
     out = oracle.retrieve_fuse(p, mem, h, depth, offs, None, 0.9, 1, 8, mirror=True)
-    for key in ("q", "a_f", "a_g", "h_out"):
+    for key in ("a_f", "a_g", "h_out"):
         np.testing.assert_array_equal(out[key], oracle.round_bf16(out[key]))
+    # q = W_Q x_h is kept exact; x_h = LN(h) + E_dep is rounded
+    x = oracle.round_bf16(oracle.layer_norm(h, p["ln_h_gamma"], p["ln_h_beta"], 1e-5) + p["E_dep"][depth])
+    np.testing.assert_allclose(out["q"], x @ p["W_Q"].T, rtol=1e-12, atol=1e-12)
     pure = oracle.retrieve_fuse(p, oracle.build_memory(p, v, mask), h, depth, offs, None, 0.9, 1, 8)
     rel = np.abs(out["h_out"] - pure["h_out"]).max() / np.abs(pure["h_out"]).max()
     assert rel < 5e-2

@@ -1,0 +1,233 @@
+"""GPU parity: the C-ABI path against the CPU oracle on the same stored inputs.
+
+Small cases span several 128-row tiles, ragged tails, masks, empty and single
+entry memories, the selection clamps (k_max = 1, k_max > |V|, the paper's
+rho = 0.8 / K_min = 32 / K_max = 256, fixed top-16, dense), per-row
+temperatures, clustered keys and the fp32 path.  The five named workloads run
+at full size (the long-memory one on sampled rows and steps).
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from parity import compare, params_for, rel_err_rows, run_gpu, run_oracle, store
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def fovea():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2608_22883_gb300 import fovea as f
+    f.lib()          # raises if the library was not built: no fallback
+    return f
+
+
+SMALL = {
+    "bf16-ragged": dict(d=256, m_sizes=[200, 37, 129], rows=[37, 5, 20], rho=0.9, k_max=16),
+    "bf16-scattered-mask-d320": dict(d=320, m_sizes=[150, 90], rows=[13, 40], M_max=220,
+                                     scattered_mask=True, rho=0.8, k_max=32),
+    "bf16-empty-and-single": dict(d=256, m_sizes=[0, 1, 70], rows=[3, 4, 9], M_max=80, k_max=8),
+    "bf16-kmax-1": dict(d=256, m_sizes=[300], rows=[33], k_max=1),
+    "bf16-kmax-beyond-valid": dict(d=256, m_sizes=[45, 3], rows=[10, 6], k_max=256, rho=0.99),
+    "bf16-paper-defaults": dict(d=384, m_sizes=[600], rows=[40], rho=0.8, k_min=32, k_max=256),
+    "bf16-fixed-top16": dict(d=256, m_sizes=[400, 250], rows=[20, 20], k_min=16, k_max=16),
+    "bf16-dense": dict(d=256, m_sizes=[180], rows=[21], k_min=180, k_max=180),
+    "bf16-temperature": dict(d=512, m_sizes=[256, 1024, 700], rows=[32, 32, 17],
+                             temperature=(0.1, 10.0), rho=0.8, k_max=128),
+    "bf16-clustered": dict(d=256, m_sizes=[2048], rows=[128], clusters=16, cluster_sigma=0.2,
+                           k_max=256),
+    "bf16-many-rows": dict(d=256, m_sizes=[130, 500], rows=[300, 4], k_max=64),
+    "bf16-hidden-128": dict(d=256, m_sizes=[100], rows=[9], k_max=16, H=128),
+    "fp32-ragged": dict(d=256, m_sizes=[64, 130], rows=[4, 11], dtype="fp32", k_max=16),
+    "fp32-temperature": dict(d=192, m_sizes=[300, 20], rows=[17, 3], dtype="fp32", k_max=64,
+                             temperature=(0.1, 10.0), rho=0.8),
+}
+
+
+def small_workload(name):
+    kw = dict(SMALL[name])
+    return workloads.generate_custom(name, kw.pop("d"), kw.pop("m_sizes"), kw.pop("rows"), **kw)
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_small_parity(fovea, name):
+    w = small_workload(name)
+    s = store(w)
+    gpu = run_gpu(s, fovea)
+    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
+    rep = compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"))
+    print(f"{name}: boundary rows {rep['exempt']}, readout err {rep['readout_err']:.2e}, "
+          f"h_out err {rep['h_out_err']:.2e}")
+
+
+@pytest.mark.parametrize("name", ["bf16-ragged", "bf16-scattered-mask-d320", "fp32-ragged",
+                                  "bf16-empty-and-single"])
+def test_memory_build_matches_oracle(fovea, name):
+    w = small_workload(name)
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
+    K, U, idx, offs = mem.views()
+    orc = oracle.build_memory({n: s.f64[n] for n in workloads.PARAM_NAMES}, s.f64["v"],
+                              s.f64.get("mask"), mirror=(w.dtype == "bf16"))
+    assert mem.valid_counts == [len(i) for i in orc.index]
+    idx = idx.cpu().numpy()
+    tol = 2e-2 if w.dtype == "bf16" else 1e-4
+    for b in range(w.B):
+        lo, hi = offs[b], offs[b + 1]
+        np.testing.assert_array_equal(idx[lo:hi], orc.index[b])
+        if hi == lo:
+            continue
+        for got, ref in ((K, orc.keys[b]), (U, orc.values[b])):
+            g = got[lo:hi].double().cpu().numpy()
+            assert rel_err_rows(g, ref).max() <= tol
+            if w.dtype == "bf16":
+                assert np.mean(g == ref) > 0.99     # same bf16 value almost everywhere
+    mem.destroy()
+
+
+def test_zero_gate_returns_rmsnorm_of_h(fovea):
+    w = small_workload("bf16-ragged")
+    w.params["w_g2"] = np.zeros_like(w.params["w_g2"])
+    w.params["b_g2"] = np.array([-1000.0], dtype=np.float32)
+    s = store(w)
+    gpu = run_gpu(s, fovea)
+    assert np.all(gpu["gate"] == 0.0)
+    h = s.f64["h"]
+    want = oracle.round_bf16(oracle.rms_norm(h, s.f64["rms_gamma"], 1e-6))
+    assert rel_err_rows(gpu["h_out"].astype(np.float64), want).max() <= 2e-2
+
+
+def test_planted_rows_select_one_entry(fovea):
+    spec = workloads.Spec(0, "planted-d512", d=512, B=1, rows_per_seq=24, rho=0.9, k_max=32,
+                          k_min=1, dtype="bf16", seed=31, m_fixed=300, peaked_rows=6)
+    w = workloads.generate(spec)
+    s = store(w)
+    gpu = run_gpu(s, fovea)
+    for row, entry in w.planted.items():
+        assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
+    orc, mem = run_oracle(s, mirror=True)
+    compare(gpu, orc, s, mem=mem)
+
+
+def test_repeat_calls_are_deterministic(fovea):
+    w = small_workload("bf16-temperature")
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
+    ws = fovea.new_workspace(params, mem, w.row_offsets, w.k_max)
+    outs = []
+    for _ in range(3):
+        o = fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets,
+                       s.dev.get("row_scale"), w.rho, w.k_min, w.k_max, workspace=ws)
+        torch.cuda.synchronize()
+        outs.append({k: v.clone() for k, v in o.items() if k != "workspace" and v is not None})
+    for o in outs[1:]:
+        for k in o:
+            assert torch.equal(o[k], outs[0][k]), k
+    fovea.sync_errors(ws)
+
+
+def test_invalid_depth_sets_error_word(fovea):
+    w = small_workload("bf16-ragged")
+    w.depth = w.depth.copy()
+    w.depth[3] = 9
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
+    o = fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets, None, w.rho, 1, 16)
+    with pytest.raises(fovea.FoveaError, match="INVALID_ARG"):
+        fovea.sync_errors(o["workspace"])
+    fovea.sync_errors(o["workspace"])      # the word was cleared
+
+
+def test_bad_row_offsets_and_workspace(fovea):
+    w = small_workload("bf16-ragged")
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
+    ws = fovea.new_workspace(params, mem, w.row_offsets, 16)
+    h_out = torch.empty_like(s.dev["h"])
+    for offs in ([1, 37, 42, 62], [0, 37, 20, 62]):
+        with pytest.raises(fovea.FoveaError, match="INVALID_ARG"):
+            fovea.retrieve_fuse(params, mem, s.dev["h"], s.dev["depth"], offs, None, 0.9, 1, 16,
+                                h_out, ws)
+    with pytest.raises(fovea.FoveaError, match="INVALID_ARG"):
+        fovea.retrieve_fuse(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets, None, 0.9, 1,
+                            16, h_out, ws[:1024])
+    with pytest.raises(fovea.FoveaError, match="UNSUPPORTED"):
+        fovea.retrieve_fuse(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets, None, 0.9, 1,
+                            4096, h_out, ws)
+    # zero draft states: nothing to do
+    fovea.retrieve_fuse(params, mem, s.dev["h"], s.dev["depth"], [0, 0, 0, 0], None, 0.9, 1, 16,
+                        h_out, ws)
+    fovea.sync_errors(ws)
+
+
+# ---------------------------------------------------------------------------
+# The five named workloads at full size
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("idx", [1, 2, 3, 4])
+def test_named_workload_parity(fovea, idx):
+    w = workloads.generate(workloads.WORKLOADS[idx])
+    s = store(w)
+    gpu = run_gpu(s, fovea)
+    mirror = w.dtype == "bf16"
+    orc, mem = run_oracle(s, mirror=mirror)
+    rep = compare(gpu, orc, s, mem=mem, mirror=mirror)
+    print(f"workload {idx}: {rep}")
+    if idx == 2:
+        for row, entry in w.planted.items():
+            assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
+        assert (gpu["counts"] == w.k_max).sum() > 16        # flat rows reach the cap
+    if idx == 3:
+        assert gpu["counts"].min() == 1 and gpu["counts"].max() == w.k_max
+
+
+def test_long_memory_sampled_steps(fovea):
+    """Long-memory workload: one memory of 4 x 8192 clustered entries queried
+    over 100 draft steps.  The GPU runs every step; the oracle checks sampled
+    rows of two sequences at steps 0, 1, 49 and 99."""
+    spec = workloads.WORKLOADS[5]
+    w0 = workloads.generate(spec, step=0)
+    s0 = store(w0)
+    params = params_for(s0, fovea)
+    mem = fovea.build_memory(params, s0.dev["v"], s0.dev.get("mask"))
+    ws = fovea.new_workspace(params, mem, w0.row_offsets, w0.k_max)
+    seqs = [0, 3]
+    p64 = {n: s0.f64[n] for n in workloads.PARAM_NAMES}
+    omem = oracle.build_memory(p64, s0.f64["v"][seqs], None, mirror=True)
+    R = spec.rows_per_seq
+    rng = np.random.default_rng(5)
+    checked = {}
+    for t in range(spec.steps):
+        h = workloads.hidden_states(spec.seed, w0.N, spec.d, step=t)
+        ht = torch.from_numpy(h).to(torch.bfloat16).cuda()
+        out = fovea.step(params, mem, ht, s0.dev["depth"], w0.row_offsets, None, w0.rho,
+                         w0.k_min, w0.k_max, workspace=ws)
+        if t not in (0, 1, 49, 99):
+            continue
+        torch.cuda.synchronize()
+        gpu = {k: (v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy())
+               for k, v in out.items() if v is not None and k != "workspace"}
+        rows = sorted(int(b * R + j) for b in seqs for j in rng.choice(R, size=12, replace=False))
+        # oracle over the two sequences only: a 2-sequence batch of the sampled rows
+        sub_offsets = np.array([0, 12, 24])
+        hw = dataclasses.replace(w0, h=h[rows], depth=w0.depth[rows], row_offsets=sub_offsets,
+                                 v=w0.v[seqs], mask=None)
+        sub = store(hw, device=None)
+        orc = oracle.retrieve_fuse(p64, omem, sub.f64["h"], sub.f64["depth"], sub_offsets, None,
+                                   w0.rho, w0.k_min, w0.k_max, mirror=True)
+        g_sub = {k: v[rows] for k, v in gpu.items()}
+        rep = compare(g_sub, orc, sub, mem=omem, mirror=True)
+        checked[t] = rep
+    fovea.sync_errors(ws)
+    assert sorted(checked) == [0, 1, 49, 99]
+    print(checked)
