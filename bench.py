@@ -1,0 +1,462 @@
+#!/usr/bin/env python3
+"""Benchmark of the FOVEA retrieve+fuse step on GB300.
+
+One step = one fovea_retrieve_fuse call over a batch of draft states against a
+visual memory built once beforehand (query LN + projection, scores over every
+valid entry, cumulative-mass selection, readout, gated correction + RMSNorm).
+Metric: draft states per second through retrieve+fuse (higher is better),
+with the roofline fraction of the dominant kernel and of the whole step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2]
+  python bench.py --impl reference ...   # the CPU oracle as the reference arm
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs an independent
+replica of the workload (the path has no exchange step); value = the draft
+states of all ranks / the slowest rank's time.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import workloads  # noqa: E402
+
+METRIC = "draft states/sec through retrieve+fuse at 1 GB300; % of HBM/tensor roofline"
+UNIT = "draft_states/s"
+L2_FLUSH_BYTES = 512 << 20
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {k: float(p[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained")}, "measured"
+    except Exception:
+        return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic bytes / flops (what the method itself must move and compute)
+# ---------------------------------------------------------------------------
+
+def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray):
+    """Per-step algorithmic bytes and flops: W_Q, the fusion weights, every
+    valid key of every sequence, the unique selected value rows, row I/O
+    (h in, h_hat out, counts and indices); scores and hidden activations are
+    intermediates and are not counted."""
+    d, H, N = w.d, w.params["b_f1"].shape[0], w.N
+    es = 2 if w.dtype == "bf16" else 4
+    weights = d * d + 2 * H * 2 * d + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
+    weights += 2 * d + 2 * d      # LN_h gamma/beta + the E_dep rows touched (bound: 2 rows)
+    keys = sum(w.m_sizes) * d
+    uniq = 0
+    for b in range(w.B):
+        lo, hi = int(w.row_offsets[b]), int(w.row_offsets[b + 1])
+        sel = set()
+        for n in range(lo, hi):
+            sel.update(int(x) for x in indices[n, :int(counts[n])])
+        uniq += len(sel)
+    values = uniq * d
+    rows_io = 2 * N * d
+    nbytes = es * (weights + keys + values + rows_io) + N * 4 + N * w.k_max * 4
+    flops = 2 * N * d * d                                       # query
+    rows = [int(w.row_offsets[b + 1] - w.row_offsets[b]) for b in range(w.B)]
+    flops += sum(2 * rows[b] * int(w.m_sizes[b]) * d for b in range(w.B))
+    flops += 2 * int(counts.sum()) * d                          # readout
+    flops += 2 * N * (2 * d * 2 * H + H * d + H)                # fusion
+    return float(nbytes), float(flops), int(uniq)
+
+
+def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int) -> float:
+    """HBM bytes one launch of a kernel must move (reads + writes)."""
+    d, H, N = w.d, w.params["b_f1"].shape[0], w.N
+    es = 2 if w.dtype == "bf16" else 4
+    if name == "query_proj":
+        return es * (d * d + N * d + 2 * N * d)
+    if name == "fuse_hidden":
+        return es * (2 * H * 2 * d + 2 * N * d + N * 2 * H + 2 * H)
+    if name == "fuse_out":
+        return es * (d * H + N * H + d) + 4 * N * d
+    if name == "score":
+        keys = sum(w.m_sizes) * d * es
+        scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
+        return keys + 2 * N * d * es + scores
+    if name == "readout":
+        return uniq_values * d * es + N * d * (4 + es)
+    if name == "select":
+        scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
+        return scores + 3 * N * w.k_max * 4
+    if name == "ln_query":
+        return es * (2 * N * d + 4 * d)
+    if name == "finalize":
+        return es * (2 * N * d + N * H + 2 * d) + 4 * N * d
+    return 0.0
+
+
+# ---------------------------------------------------------------------------
+# Clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.dev}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, val in zip(names, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": float(max(mx)) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# Reference arm: the CPU oracle
+# ---------------------------------------------------------------------------
+
+def oracle_inputs(w: workloads.Workload):
+    """The stored (bf16 / fp32) inputs as float64, exactly as the GPU sees them."""
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+
+    def f64(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dt).to(torch.float64).numpy()
+    p = {k: f64(v) for k, v in w.params.items()}
+    return p, f64(w.v), f64(w.h)
+
+
+def time_oracle(w: workloads.Workload, min_seconds: float, max_rows: int = None,
+                rows_per_call: int = None):
+    """Run the oracle's retrieve+fuse on rows of the workload until
+    min_seconds elapsed; returns (rows/s, rows, seconds, build seconds)."""
+    import oracle
+    p, v, h = oracle_inputs(w)
+    mirror = w.dtype == "bf16"
+    t0 = time.perf_counter()
+    mem = oracle.build_memory(p, v, w.mask, mirror=mirror, ln_eps=float(np.float32(1e-5)))
+    build_s = time.perf_counter() - t0
+    rows_per_call = rows_per_call or w.N
+    done, t_start, i = 0, time.perf_counter(), 0
+    while True:
+        sel = [(i * rows_per_call + j) % w.N for j in range(rows_per_call)]
+        oracle.retrieve_fuse(p, mem, h, w.depth, w.row_offsets, w.row_scale, w.rho, w.k_min,
+                             w.k_max, mirror=mirror, rows=sel, ln_eps=float(np.float32(1e-5)),
+                             rms_eps=float(np.float32(1e-6)))
+        done += rows_per_call
+        i += 1
+        el = time.perf_counter() - t_start
+        if el >= min_seconds or (max_rows is not None and done >= max_rows):
+            return done / el, done, el, build_s
+
+
+def cores_used() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, w):
+    import oracle
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    p, v, h = oracle_inputs(w)
+    mirror = w.dtype == "bf16"
+    mem = oracle.build_memory(p, v, w.mask, mirror=mirror, ln_eps=float(np.float32(1e-5)))
+    eps = dict(ln_eps=float(np.float32(1e-5)), rms_eps=float(np.float32(1e-6)))
+
+    def one(i):
+        n = i % w.N
+        oracle.retrieve_fuse(p, mem, h, w.depth, w.row_offsets, w.row_scale, w.rho, w.k_min,
+                             w.k_max, mirror=mirror, rows=[n], **eps)
+    for i in range(args.warmup):
+        one(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        one(args.warmup + i)
+    el = time.perf_counter() - t0
+    value = args.steps / el
+    sample = f"one draft state per step (cycling the {w.N} rows), memory built once (excluded)"
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": 1000 * el / args.steps, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference",
+           "config": {"workload": w.name, "d_model": w.d, "memory_entries": w.m_sizes,
+                      "draft_states": w.N, "rho": w.rho, "k_max": w.k_max},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                            "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# The GPU arm
+# ---------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="fovea", choices=["fovea", "reference"])
+    ap.add_argument("--workload", type=int, default=2)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+
+    spec = workloads.WORKLOADS[args.workload]
+    w = workloads.generate(spec)
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    from paper_2608_22883_gb300 import fovea
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    dev = torch.device("cuda", local)
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    weights = {k: torch.from_numpy(np.ascontiguousarray(v)).to(dt).to(dev) for k, v in w.params.items()}
+    params = fovea.Params(weights, d_model=w.d, mlp_hidden=w.params["b_f1"].shape[0],
+                          max_depth=w.params["E_dep"].shape[0] - 1,
+                          dtype=fovea.BF16 if w.dtype == "bf16" else fovea.FP32)
+    v = torch.from_numpy(w.v).to(dt).to(dev)
+    mask = torch.from_numpy(w.mask).to(dev) if w.mask is not None else None
+    h_host = torch.from_numpy(w.h).to(dt).pin_memory()
+    depth_host = torch.from_numpy(w.depth).pin_memory()
+    h = h_host.to(dev)
+    depth = depth_host.to(dev)
+    row_scale = torch.from_numpy(w.row_scale).to(dev) if w.row_scale is not None else None
+
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    mem = fovea.build_memory(params, v, mask)
+    torch.cuda.synchronize()
+    build_ms = 1000 * (time.perf_counter() - t0)
+
+    N, d, K = w.N, w.d, w.k_max
+    ws = fovea.new_workspace(params, mem, w.row_offsets, K)
+    h_out = torch.empty_like(h)
+    counts = torch.empty(N, dtype=torch.int32, device=dev)
+    indices = torch.empty((N, K), dtype=torch.int32, device=dev)
+    offs_c = fovea._offsets(w.row_offsets)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(hh=h, dd=depth):
+        fovea.retrieve_fuse(params, mem, hh, dd, w.row_offsets, row_scale, w.rho, w.k_min, K,
+                            h_out, ws, counts=counts, indices=indices, offsets_c=offs_c)
+
+    for i in range(args.warmup):
+        flush.fill_(i & 0xFF)
+        step()
+    torch.cuda.synchronize()
+    fovea.sync_errors(ws)
+
+    # ---- timed region: K steps, L2 flushed before each (outside the events) ----
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    fovea.timing_enable(True)
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_((i + 7) & 0xFF)
+        ev0[i].record(stream)
+        step()
+        ev1[i].record(stream)
+    torch.cuda.synchronize()
+    wall_s = time.perf_counter() - t_wall
+    if dist is not None:
+        dist.barrier()
+    clk = clocks.stop()
+    per_kernel = fovea.timing_read()
+    fovea.timing_enable(False)
+    step_ms = [a.elapsed_time(b) for a, b in zip(ev0, ev1)]
+    ms = float(np.mean(step_ms))
+    fovea.sync_errors(ws)
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * N / (ms / 1000.0)
+
+    # ---- untimed-kernel step (for the step's own duration without event hooks) ----
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(min(args.steps, 500))]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(len(ev_a))]
+    for i in range(len(ev_a)):
+        flush.fill_(i & 0xFF)
+        ev_a[i].record(stream)
+        step()
+        ev_b[i].record(stream)
+    torch.cuda.synchronize()
+    ms_nohooks = float(np.mean([a.elapsed_time(b) for a, b in zip(ev_a, ev_b)]))
+
+    # ---- end to end through the C ABI with host buffers ----
+    h_out_host = torch.empty(h_out.shape, dtype=h_out.dtype).pin_memory()
+    counts_host = torch.empty(N, dtype=torch.int32).pin_memory()
+    idx_host = torch.empty((N, K), dtype=torch.int32).pin_memory()
+    n_e2e = min(args.steps, 500)
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
+    h_dev2 = torch.empty_like(h)
+    depth_dev2 = torch.empty_like(depth)
+    for i in range(n_e2e):
+        flush.fill_(i & 0xFF)
+        e0[i].record(stream)
+        h_dev2.copy_(h_host, non_blocking=True)
+        depth_dev2.copy_(depth_host, non_blocking=True)
+        step(h_dev2, depth_dev2)
+        h_out_host.copy_(h_out, non_blocking=True)
+        counts_host.copy_(counts, non_blocking=True)
+        idx_host.copy_(indices, non_blocking=True)
+        e1[i].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = float(np.mean([a.elapsed_time(b) for a, b in zip(e0, e1)]))
+    h2d = h_host.numel() * h_host.element_size() + depth_host.numel() * 4
+    d2h = h_out_host.numel() * h_out_host.element_size() + N * 4 + N * K * 4
+
+    # ---- roofline ----
+    c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
+    nbytes, flops, uniq = step_cost(w, c_np, i_np)
+    peaks, peak_src = load_peaks()
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    t_roof = max(t_hbm, t_tc)
+    kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
+    dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
+    dom_bytes = kernel_bytes(dom, w, uniq)
+    achieved = dom_bytes / (kern[dom]["ms_avg"] / 1000.0) / 1e9
+    launches = sum(k["launches"] for k in kern.values())
+    total_kernel_ms = sum(k["ms_avg"] * k["launches"] for k in kern.values())
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        try:
+            with open(tpath) as f:
+                tr = json.load(f)
+            ent = tr.get(w.name, {}).get(dom)
+            if ent and ent.get("kernel_sha") == _kernel_sha():
+                traffic = ent["bytes_per_launch"]
+        except Exception:
+            traffic = None
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": w.name, "d_model": w.d, "memory_entries": w.m_sizes,
+                   "draft_states": N, "sequences": w.B, "rho": w.rho, "k_min": w.k_min,
+                   "k_max": K, "mlp_hidden": int(w.params["b_f1"].shape[0]),
+                   "l2": "flushed before every step (512 MB write outside the per-step events)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                     "traffic": traffic, "algorithmic_bytes": dom_bytes,
+                     "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                     else "fallback 6.8 TB/s"},
+        "step_roofline": {"bytes": nbytes, "flops": flops, "unique_value_rows": uniq,
+                          "t_roof_us": 1e6 * t_roof, "bound": "hbm" if t_hbm >= t_tc else "tensor",
+                          "frac": t_roof / (ms / 1000.0),
+                          "frac_without_event_hooks": t_roof / (ms_nohooks / 1000.0),
+                          "peaks": f"{peak_src}: {peaks['hbm_gbs']} GB/s, {peaks['bf16_tflops']} TF/s"},
+        "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"]} for k, v in kern.items()},
+        "ms_per_step_without_event_hooks": ms_nohooks,
+        "kernel_ms_per_step": total_kernel_ms / args.steps,
+        "gpu_launches": launches,
+        "memory_build_ms": build_ms,
+        "clocks": clk,
+        "e2e": {"value": world * N / (e2e_ms / 1000.0), "unit": UNIT, "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
+        "wall_s_timed_region": wall_s,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, rows, secs, build_s = time_oracle(w, args.cpu_seconds)
+        out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                               "sample": f"{rows} draft states ({rows // w.N} oracle steps of the "
+                                         f"{w.N}-row batch) in {secs:.1f} s; memory build "
+                                         f"({build_s:.1f} s) excluded"}
+    if rank == 0:
+        print(json.dumps(out))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def _kernel_sha() -> str:
+    import hashlib
+    hsh = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_22883_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            hsh.update(fh.read())
+    return hsh.hexdigest()[:16]
+
+
+if __name__ == "__main__":
+    sys.exit(main())
