@@ -202,6 +202,38 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                                            void* workspace, size_t workspace_bytes,
                                            void* stream);
 
+/*
+ * fovea_retrieve_fuse without a workspace argument, for callers that cannot
+ * allocate device memory where they run the draft step: code recorded into a
+ * CUDA graph or running inside a runtime with a fixed, pre-planned memory
+ * budget (where cudaMalloc is illegal or unavailable), and latency-critical
+ * loops that must not take the implicit device synchronisation of
+ * cudaMalloc / cudaFree.  The paper has no counterpart: this is an interface
+ * convenience of this library.
+ *
+ * Arguments and outputs are those of fovea_retrieve_fuse.  The scratch is a
+ * file-scope device array of FOVEA_NOALLOC_WORKSPACE_BYTES that every GPU
+ * loading the library holds until the process exits; the call allocates
+ * nothing (no cudaMalloc, cudaFree or allocating library routine).
+ * - A call whose scratch need (fovea_workspace_size) exceeds the array returns
+ *   FOVEA_ERR_UNSUPPORTED and enqueues nothing.
+ * - The first call on a device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.
+ * - Every call on a device shares the one array: calls that overlap on the GPU
+ *   (other streams, other host threads) race and corrupt each other.  Each
+ *   call clears the array's error word first; device-side conditions (a bad
+ *   depth) are not reported back by this entry point, so validate depths.
+ */
+#define FOVEA_NOALLOC_WORKSPACE_BYTES (32u << 20)
+FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(const fovea_params* p, const fovea_memory* mem,
+                                                   const void* h, const int32_t* depth,
+                                                   const int32_t* row_offsets,
+                                                   const float* row_scale, float rho, int k_min,
+                                                   int k_max, void* h_out, int32_t* counts,
+                                                   int32_t* indices, float* readout, float* gate,
+                                                   void* stream);
+
 /* Synchronise `stream`, read and clear the workspace's sticky error word.
  * Returns FOVEA_OK, FOVEA_ERR_INVALID_ARG (a depth outside [0, D] was seen)
  * or FOVEA_ERR_TIMEOUT (a bounded device wait gave up), or FOVEA_ERR_CUDA. */

@@ -26,6 +26,14 @@ static fovea_status fail(fovea_status st, const char* fmt, ...) {
   g_last_error = buf;
   return st;
 }
+namespace fovea {
+// Records the message fovea_last_error() returns (for other translation units).
+fovea_status report_error(fovea_status st, const char* msg) {
+  g_last_error = msg;
+  return st;
+}
+}  // namespace fovea
+
 static fovea_status cuda_fail(cudaError_t e, const char* where) {
   return fail(FOVEA_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
 }
@@ -271,7 +279,7 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
     void* src_row = nullptr;
     void* fix = nullptr;                     // bf16: count word + listed key elements
     const bool bf = p->dtype == FOVEA_BF16;
-    const long long fix_cap = bf ? (long long)total * d / 16 + 4096 : 0;
+    const long long fix_cap = bf ? (long long)total * d / 8 + 4096 : 0;
     if ((st = alloc_dev(&m->keys, (size_t)total * d * es, "keys")) != FOVEA_OK ||
         (st = alloc_dev(&m->values, (size_t)total * d * es, "values")) != FOVEA_OK ||
         (st = alloc_dev(reinterpret_cast<void**>(&m->orig_index), total * sizeof(int32_t),

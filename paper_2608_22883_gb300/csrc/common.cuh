@@ -105,6 +105,8 @@ struct GemmArgs {
   const void* bias0; const void* bias1;
   const float* row_scale; float scale;
   KeyFix* fix_list; int* fix_count; int fix_cap;   // kEpiStoreKeys
+  int splits;         // tensor-core path: CTAs of a cluster sharing one output tile (split K)
+  int stages;         // tensor-core path: depth of the shared-memory ring
   int* err;
   int ngroups;
   GemmGroup groups[FOVEA_MAX_SEQ];
@@ -131,6 +133,9 @@ __device__ __forceinline__ int seq_of_row(const SeqTable& t, int row) {
 // ---------------------------------------------------------------------------
 // Host-side launch interfaces (defined in the kernel translation units)
 // ---------------------------------------------------------------------------
+
+// Sets the message fovea_last_error() returns on this thread (api.cu).
+fovea_status report_error(fovea_status st, const char* msg);
 
 cudaError_t launch_ln_rows(int dtype, const void* x, const int32_t* src_row, int rows, int d,
                            const void* gamma, const void* beta, float eps, const void* E,

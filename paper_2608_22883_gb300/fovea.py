@@ -35,7 +35,9 @@ EXPORTS = (
     "fovea_build_memory", "fovea_memory_destroy", "fovea_memory_info", "fovea_memory_tensors",
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
+    "fovea_retrieve_fuse_noalloc",
 )
+NOALLOC_WORKSPACE_BYTES = 32 << 20
 
 
 class FoveaError(RuntimeError):
@@ -76,6 +78,10 @@ def lib() -> ctypes.CDLL:
         L.fovea_retrieve_fuse.argtypes = [ctypes.POINTER(CParams), vp, vp, vp, i32p, vp,
                                           ctypes.c_float, ctypes.c_int, ctypes.c_int,
                                           vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+        L.fovea_retrieve_fuse_noalloc.argtypes = [ctypes.POINTER(CParams), vp, vp, vp, i32p, vp,
+                                                  ctypes.c_float, ctypes.c_int, ctypes.c_int,
+                                                  vp, vp, vp, vp, vp, vp]
+        L.fovea_retrieve_fuse_noalloc.restype = ctypes.c_int
         L.fovea_sync_errors.argtypes = [vp, vp]
         L.fovea_last_error.restype = ctypes.c_char_p
         L.fovea_last_error.argtypes = []
@@ -258,6 +264,22 @@ def step(params: Params, memory: Memory, h: torch.Tensor, depth: torch.Tensor, r
                   readout=out["readout"], gate=out["gate"], stream=stream)
     out["workspace"] = workspace
     return out
+
+
+def retrieve_fuse_noalloc(params: Params, memory: Memory, h: torch.Tensor, depth: torch.Tensor,
+                          row_offsets, row_scale: Optional[torch.Tensor], rho: float, k_min: int,
+                          k_max: int, h_out: torch.Tensor, *,
+                          counts: Optional[torch.Tensor] = None,
+                          indices: Optional[torch.Tensor] = None,
+                          readout: Optional[torch.Tensor] = None,
+                          gate: Optional[torch.Tensor] = None, stream=None) -> None:
+    """fovea_retrieve_fuse_noalloc: the draft step with the library's static
+    scratch instead of a workspace (for callers that cannot allocate)."""
+    _check(lib().fovea_retrieve_fuse_noalloc(params.ref, memory.handle, _ptr(h), _ptr(depth),
+                                             _offsets(row_offsets), _ptr(row_scale), float(rho),
+                                             int(k_min), int(k_max), _ptr(h_out), _ptr(counts),
+                                             _ptr(indices), _ptr(readout), _ptr(gate),
+                                             _stream(stream)))
 
 
 def sync_errors(workspace: torch.Tensor, stream=None) -> None:
