@@ -160,7 +160,10 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
                                             const int32_t* row_offsets, int k_max,
                                             size_t* bytes);
 
-/* Zero the workspace's error word (enqueued on `stream`). */
+/* Zero the workspace's header: the error word and the counters the split-K
+ * GEMMs use (enqueued on `stream`).  Kernels leave the counters at zero, so
+ * one initialisation serves every later call; re-initialise after a call that
+ * reported FOVEA_ERR_TIMEOUT. */
 FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void* stream);
 
 /*

@@ -4,6 +4,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <algorithm>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -392,11 +393,39 @@ FOVEA_API fovea_status fovea_memory_tensors(const fovea_memory* mem, const void*
 // Workspace layout (all regions 256-byte aligned)
 // ---------------------------------------------------------------------------
 namespace {
+// Workspace header: the sticky error word (first 256 bytes) and the split-K
+// tile counters (pairs of ints).  Zero when the workspace is initialised; the
+// kernels leave the counters at zero after every launch.
+constexpr size_t kWsHeaderBytes = 16384;
+constexpr long long kTileSyncTiles = (kWsHeaderBytes - 256) / 8;
+
 struct WsLayout {
-  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, total;
+  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, partials, total;
+  long long partial_floats;
 };
 
-WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems) {
+// fp32 scratch for the split-K partial tiles of the step's tensor-core GEMMs
+// (they run one after another, so one region serves all of them).
+long long step_partial_floats(int dtype, int d, int H, int N, int ngroups, int max_m, int max_r) {
+  if (dtype != FOVEA_BF16 || N == 0) return 0;
+  GemmArgs* a = new GemmArgs;
+  auto plan = [&](int epi, int k_total, int a_split, int groups, int mm, int mn) {
+    memset(a, 0, sizeof(GemmArgs));
+    a->k_total = k_total;
+    a->a_split = a_split;
+    a->ngroups = groups;
+    return plan_gemm_tc(epi, *a, mm, mn).partial_floats;
+  };
+  long long need = plan(kEpiStoreHiLo, d, 0x7fffffff, 1, d, N);
+  if (ngroups > 0) need = std::max(need, plan(kEpiScores, d, 0x7fffffff, ngroups, max_m, max_r));
+  need = std::max(need, plan(kEpiBiasSilu, 2 * d, H, 1, 2 * H, N));
+  need = std::max(need, plan(kEpiBiasF32, H, 0x7fffffff, 1, d, N));
+  delete a;
+  return need;
+}
+
+WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems,
+                   long long partial_floats) {
   WsLayout L;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -405,7 +434,7 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
     return o;
   };
   const size_t es = esize(dtype);
-  L.err = take(256);
+  L.err = take(kWsHeaderBytes);          // error word, then split-K tile counters
   L.xh = take((size_t)N * d * es);
   L.q = take((size_t)N * d * es * (dtype == FOVEA_BF16 ? 2 : 1));   // bf16: q_hi | q_lo
   L.scores = take((size_t)score_elems * 4);
@@ -415,28 +444,34 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
   L.r_lo = take((size_t)N * d * es);
   L.act = take((size_t)N * 2 * H * es);
   L.c = take((size_t)N * d * 4);
+  L.partials = take((size_t)partial_floats * 4);
+  L.partial_floats = partial_floats;
   L.total = off;
   return L;
 }
 
 fovea_status check_rows(const fovea_memory* mem, const int32_t* row_offsets, int* N_out,
-                        long long* score_elems, int* max_m, int* max_r) {
+                        long long* score_elems, int* max_m, int* max_r, int* ngroups) {
   if (mem == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "memory is NULL");
   if (row_offsets == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "row_offsets is NULL");
   if (row_offsets[0] != 0) return fail(FOVEA_ERR_INVALID_ARG, "row_offsets[0] = %d, expected 0", row_offsets[0]);
   long long se = 0;
-  int mm = 0, mr = 0;
+  int mm = 0, mr = 0, ng = 0;
   for (int b = 0; b < mem->B; ++b) {
     const int r = row_offsets[b + 1] - row_offsets[b];
     if (r < 0) return fail(FOVEA_ERR_INVALID_ARG, "row_offsets decrease at sequence %d", b);
     se += (long long)r * mem->counts[b];
     if (r > 0 && mem->counts[b] > mm) mm = mem->counts[b];
-    if (r > mr) mr = r;
+    if (r > 0 && mem->counts[b] > 0) {
+      ++ng;
+      if (r > mr) mr = r;
+    }
   }
   *N_out = row_offsets[mem->B];
   *score_elems = se;
   *max_m = mm;
   *max_r = mr;
+  *ngroups = ng;
   return FOVEA_OK;
 }
 }  // namespace
@@ -454,18 +489,20 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
     return fail(FOVEA_ERR_INVALID_ARG, "mlp_hidden %d must be a positive multiple of 128",
                 p->mlp_hidden);
   if (k_max < 1) return fail(FOVEA_ERR_INVALID_ARG, "k_max = %d < 1", k_max);
-  int N, mm, mr;
+  int N, mm, mr, ng;
   long long se;
-  if ((st = check_rows(mem, row_offsets, &N, &se, &mm, &mr)) != FOVEA_OK) return st;
-  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se).total;
+  if ((st = check_rows(mem, row_offsets, &N, &se, &mm, &mr, &ng)) != FOVEA_OK) return st;
+  const long long pf = step_partial_floats(p->dtype, p->d_model, p->mlp_hidden, N, ng, mm, mr);
+  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se, pf).total;
   return FOVEA_OK;
 }
 
 FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void* stream) {
   g_last_error.clear();
   if (workspace == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "workspace is NULL");
-  if (bytes < 256) return fail(FOVEA_ERR_INVALID_ARG, "workspace of %zu bytes is too small", bytes);
-  FOVEA_CUDA(cudaMemsetAsync(workspace, 0, 256, static_cast<cudaStream_t>(stream)),
+  if (bytes < kWsHeaderBytes)
+    return fail(FOVEA_ERR_INVALID_ARG, "workspace of %zu bytes is too small", bytes);
+  FOVEA_CUDA(cudaMemsetAsync(workspace, 0, kWsHeaderBytes, static_cast<cudaStream_t>(stream)),
              "cudaMemsetAsync");
   return FOVEA_OK;
 }
@@ -507,9 +544,10 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if (mem->d != p->d_model || mem->dtype != p->dtype)
     return fail(FOVEA_ERR_INVALID_ARG, "memory was built with d=%d dtype=%d, params have d=%d dtype=%d",
                 mem->d, mem->dtype, p->d_model, p->dtype);
-  int N, max_m, max_r;
+  int N, max_m, max_r, ngroups;
   long long score_elems;
-  if ((st = check_rows(mem, row_offsets, &N, &score_elems, &max_m, &max_r)) != FOVEA_OK) return st;
+  if ((st = check_rows(mem, row_offsets, &N, &score_elems, &max_m, &max_r, &ngroups)) != FOVEA_OK)
+    return st;
   if (N == 0) return FOVEA_OK;
   NEED_PTR(h, "h");
   NEED_PTR(h_out, "h_out");
@@ -520,7 +558,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   const int d = p->d_model, H = p->mlp_hidden, dt = p->dtype;
-  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems);
+  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems,
+                               step_partial_floats(dt, d, H, N, ngroups, max_m, max_r));
   if (workspace_bytes < L.total)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);
 
@@ -536,6 +575,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   void* r_lo = ws + L.r_lo;
   void* act = ws + L.act;
   float* cbuf = reinterpret_cast<float*>(ws + L.c);
+  float* partials = reinterpret_cast<float*>(ws + L.partials);
+  int* tile_sync = reinterpret_cast<int*>(ws + L.err + 256);
 
   // Per-sequence table (kernel parameter).
   static thread_local SeqTable tab;
@@ -570,6 +611,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.A0 = p->W_Q; a.lda0 = d;
   a.B0 = xh; a.ldb0 = d;
   a.out0 = q; a.out1 = q_lo; a.ldc = d; a.err = err;
+  a.partials = partials; a.partials_floats = L.partial_floats;
+  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
   { KernelTimer t("query_proj", s);
@@ -588,6 +631,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.row_scale = row_scale;
     a.scale = (float)(1.0 / sqrt((double)d));
     a.err = err;
+  a.partials = partials; a.partials_floats = L.partial_floats;
+  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
     int g = 0;
     for (int b = 0; b < mem->B; ++b) {
       const int r = row_offsets[b + 1] - row_offsets[b];
@@ -625,6 +670,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.out0 = act; a.ldc = 2 * H;
   a.bias0 = p->b_f1; a.bias1 = p->b_g1;
   a.err = err;
+  a.partials = partials; a.partials_floats = L.partial_floats;
+  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, 2 * H, 0, N, 0};
   { KernelTimer t("fuse_hidden", s);
@@ -641,6 +688,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.out0 = cbuf; a.ldc = d;
   a.bias0 = p->b_f2;
   a.err = err;
+  a.partials = partials; a.partials_floats = L.partial_floats;
+  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
   { KernelTimer t("fuse_out", s);

@@ -107,6 +107,10 @@ struct GemmArgs {
   KeyFix* fix_list; int* fix_count; int fix_cap;   // kEpiStoreKeys
   int splits;         // tensor-core path: CTAs of a cluster sharing one output tile (split K)
   int stages;         // tensor-core path: depth of the shared-memory ring
+  float* partials;    // tensor-core split K: fp32 partial tiles (scratch)
+  long long partials_floats;
+  int* tile_sync;     // tensor-core split K: per tile {arrivals, departures}, zero between launches
+  long long tile_sync_tiles;
   int* err;
   int ngroups;
   GemmGroup groups[FOVEA_MAX_SEQ];
@@ -171,6 +175,14 @@ struct TmaOperand {     // a row-major [rows, cols] bf16 matrix with a row strid
   const void* base;
   long long rows, cols, ld;   // ld in elements
 };
+// Tile plan of a tensor-core GEMM: feature tile width, split-K factor and
+// the fp32 scratch (partial tiles) that split needs.
+struct GemmPlan {
+  int bn, splits, stages;
+  long long partial_floats;
+  long long tiles;       // output tiles of a split-K launch (counter pairs it needs)
+};
+GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n);
 cudaError_t launch_gemm_tc(int epi, const GemmArgs& a, const TmaOperand& A0, const TmaOperand& A1,
                            const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
                            cudaStream_t s);

@@ -5,39 +5,58 @@
 // significant bits) and each key tile meets both parts, so the scores are not
 // limited by a bf16 rounding of q.
 //
-// A (weights or keys) supplies the UMMA M = 128 rows; B (draft states or
-// tokens) supplies UMMA N = BN columns, so a 64-row draft batch is one N = 64
-// MMA instead of a mostly-empty M tile ("swap AB").  Both operands are
-// K-major bf16, staged by TMA into 128-byte-swizzled shared-memory tiles of
-// 64 contraction elements; fp32 accumulators live in tensor memory and are
-// read back with tcgen05.ld for the epilogue.
+// Operand roles.  In the GemmArgs vocabulary A holds the output columns
+// (weights, keys: the "feature" operand) and B the output rows (draft states,
+// tokens: the "row" operand).  On the tensor core the row operand is the MMA
+// A operand (M = 128 rows; a 64-row batch is zero-filled by TMA) and the
+// feature operand is the MMA B operand (N = BN <= 256 features).  A tcgen05
+// MMA costs about the same time for any N up to 256, so a wide feature tile
+// consumes twice the weight bytes per MMA of a 128-feature tile: the
+// weight-streaming GEMMs are limited by that consumption rate per SM.
+// Both operands are K-major bf16, staged by TMA into 128-byte-swizzled
+// shared-memory tiles of 64 contraction elements; fp32 accumulators live in
+// tensor memory (lane = row, column = feature) and are read back with
+// tcgen05.ld: each epilogue thread owns one row and its BN features.
 //
-// Roles (128 threads): warp 0 lane 0 issues TMA loads into a STAGES-deep ring,
-// warp 1 owns the tensor-memory allocation and its lane 0 issues the MMAs
-// (one elected thread), and all four warps run the epilogue: warp w reads
-// accumulator lanes 32w..32w+31.  Every mbarrier wait is bounded (~2 s); a
-// wait that gives up sets kErrTimeout in the error word and the CTA unwinds.
+// Roles (128 threads): warp 0 lane 0 issues TMA loads into a ring of shared
+// memory stages, warp 1 owns the tensor-memory allocation and its lane 0
+// issues the MMAs (one elected thread), and all four warps run the epilogue:
+// warp w reads accumulator lanes (rows) 32w..32w+31.  Every mbarrier wait is
+// bounded (~2 s); a wait that gives up sets kErrTimeout in the error word and
+// the CTA unwinds.
+//
+// Split K: when the output tiles cannot fill the GPU (a 64-row batch against
+// a weight matrix), S CTAs share one output tile, each contracting a slice of
+// K and writing its fp32 partial tile (column-major, so the 32 rows a warp
+// holds land in one 128-byte line) to global scratch.  The grid is a
+// cooperative launch, so all its CTAs are resident together: the S CTAs of a
+// tile meet on a per-tile arrival counter (a bounded spin), then CTA r sums
+// the S partials of columns [r BN/S, (r+1) BN/S) in rank order (so the result
+// does not depend on timing) and runs the epilogue for them.  The last CTA to
+// leave resets the tile's counters for the next launch.
 #include "gemm_epilogue.cuh"
 
 namespace fovea {
 namespace tc {
 
-constexpr int BM = 128;          // UMMA M
+constexpr int BM = 128;          // UMMA M: rows per tile
 constexpr int BK = 64;           // contraction elements per stage (128 bytes bf16)
 constexpr int UMMA_K = 16;       // contraction elements per tcgen05.mma (kind::f16)
 constexpr int kThreads = 128;
-constexpr int kSmemBudget = 200 * 1024;
+constexpr int kSmemBudget = 200 * 1024;   // shared-memory stages, one CTA per SM
+constexpr int kSmemBudgetPair = 100 * 1024;  // two CTAs per SM
+constexpr int kSmemExtra = 1024 /*alignment*/ + 256 /*barriers*/;
+constexpr int kMaxStages = 8;
 
-// DUAL: the B stage holds two tiles (hi and lo parts of one operand), and
-// every A tile is multiplied by both into the same accumulator.
+// BN features per tile; DUAL: the row stage holds two tiles (hi and lo parts
+// of the row operand), and each feature tile is multiplied by both into the
+// same accumulator.
 template <int BN, bool DUAL = false>
 struct Cfg {
-  static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_TILE = BN * BK * 2;
-  static constexpr int B_BYTES = B_TILE * (DUAL ? 2 : 1);
-  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (kSmemBudget / STAGE_BYTES) < 8 ? (kSmemBudget / STAGE_BYTES) : 8;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 /*alignment*/ + 256 /*barriers*/;
+  static constexpr int R_TILE = BM * BK * 2;                 // one row tile
+  static constexpr int R_BYTES = R_TILE * (DUAL ? 2 : 1);
+  static constexpr int F_BYTES = BN * BK * 2;                // one feature tile
+  static constexpr int STAGE_BYTES = R_BYTES + F_BYTES;
   static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
   // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9
   // = 1), B bf16 (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at
@@ -91,6 +110,12 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
     if (abort_flag != nullptr && *abort_flag) return false;
     if (globaltimer_ns() - t0 > limit_ns) return false;
   }
+}
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
@@ -175,10 +200,11 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 }
 
 // Key epilogue: store bf16(acc); for key columns, list the element when acc
-// lies within 2^-14 * max(|acc|, scale) of a bf16 rounding midpoint.  The
-// tensor-core fp32 accumulation error measured on d = 4096 keys is about
-// 5e-6 of that scale (one tenth of the window), so an element outside the
-// window rounds as the exact value would.
+// lies within 2^-14 * max(|acc|, scale) of a bf16 rounding midpoint, scale
+// being the RMS of the token's values in this tile (the magnitude of the
+// partial sums).  The tensor-core fp32 accumulation error measured on
+// d = 4096 keys is about 5e-6 of that scale (one tenth of the window), so an
+// element outside the window rounds as the exact value would.
 __device__ __forceinline__ void store_key(const GemmArgs& a, const GemmGroup& g, int m, int n,
                                           float acc, float scale) {
   const long long row = (long long)g.b_row0 + n;
@@ -202,48 +228,52 @@ __device__ __forceinline__ void store_key(const GemmArgs& a, const GemmGroup& g,
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
-                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmF0, const __grid_constant__ CUtensorMap tmF1,
+                   const __grid_constant__ CUtensorMap tmR0, const __grid_constant__ CUtensorMap tmR1,
                    const __grid_constant__ GemmArgs args) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = Cfg<BN, DUAL>;
+  const int S = args.splits;
+  const uint32_t rank = (uint32_t)((int)blockIdx.x % S);
   const GemmGroup& g = args.groups[blockIdx.z];
-  // Output columns [0, a_split) come from A0 and [a_split, m) from A1; each
-  // part is tiled on its own so no tile straddles the two operands.
-  // (A group smaller than the grid leaves its extra CTAs idle.)
+  // Output columns (features) [0, a_split) come from F0 and [a_split, m) from
+  // F1; each part is tiled on its own so no tile straddles the two operands.
+  // A group smaller than the grid leaves its extra tiles idle.  The S CTAs of a
+  // tile share these decisions, so a tile's CTAs exit together.
   const int split = args.a_split;
   const bool has_second = split < g.m;
-  const int tiles0 = has_second ? (split + BM - 1) / BM : (g.m + BM - 1) / BM;
-  const int bx = (int)blockIdx.x;
-  if (!has_second && bx >= tiles0) return;    // uniform for the CTA, before any setup
-  const bool a_second = has_second && bx >= tiles0;
-  const int m0 = a_second ? split + (bx - tiles0) * BM : bx * BM;
-  const int m_end = a_second ? g.m : min(g.m, split);
-  const int n0 = blockIdx.y * BN;
+  const int tiles0 = has_second ? (split + BN - 1) / BN : (g.m + BN - 1) / BN;
+  const int tx = (int)blockIdx.x / S;
+  if (!has_second && tx >= tiles0) return;
+  const bool f_second = has_second && tx >= tiles0;
+  const int m0 = f_second ? split + (tx - tiles0) * BN : tx * BN;
+  const int m_end = f_second ? g.m : min(g.m, split);
+  const int n0 = blockIdx.y * BM;
   if (m0 >= m_end || n0 >= g.n) return;
 
+  const int stages = args.stages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
-  uint64_t* empty = full + C::STAGES;
-  uint64_t* accum = empty + C::STAGES;
+  uint8_t* sR = smem;                                  // [stages][R_BYTES]
+  uint8_t* sF = smem + stages * C::R_BYTES;            // [stages][F_BYTES]
+  uint64_t* full = reinterpret_cast<uint64_t*>(sF + stages * C::F_BYTES);
+  uint64_t* empty = full + stages;
+  uint64_t* accum = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C::STAGES; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int st = 0; st < stages; ++st) {
+      mbar_init(&full[st], 1);
+      mbar_init(&empty[st], 1);
     }
     mbar_init(accum, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    prefetch_tmap(&tmA0);
-    prefetch_tmap(&tmB0);
+    prefetch_tmap(&tmF0);
+    prefetch_tmap(&tmR0);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -254,108 +284,198 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int kb_total = args.k_total / BK;
-  const int b_split_kb = args.b_split / BK;
+  const int r_split_kb = args.b_split / BK;
+  const int kb_lo = (int)((long long)rank * kb_total / S);
+  const int kb_hi = (int)((long long)(rank + 1) * kb_total / S);
+  const int nkb = kb_hi - kb_lo;
 
   if (warp == 0 && lane == 0) {
     // ---- TMA producer ----
-    const CUtensorMap* mapA = a_second ? &tmA1 : &tmA0;
-    const int ay = a_second ? m0 - split : g.a_row0 + m0;
-    const int by = g.b_row0 + n0;
+    const CUtensorMap* mapF = f_second ? &tmF1 : &tmF0;
+    const int fy = f_second ? m0 - split : g.a_row0 + m0;
+    const int ry = g.b_row0 + n0;
     int issued = 0;
-    for (int kb = 0; kb < kb_total; ++kb) {
-      const int s = kb % C::STAGES;
-      const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
-      if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag)) {
+    for (int i = 0; i < nkb; ++i) {
+      const int kb = kb_lo + i;
+      const int st = i % stages;
+      const uint32_t ph = (uint32_t)(i / stages) & 1u;
+      if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
         *abort_flag = 1;
         break;
       }
-      mbar_expect_tx(&full[s], C::STAGE_BYTES);
-      tma_load_2d(sA + s * C::A_BYTES, mapA, &full[s], kb * BK, ay);
+      mbar_expect_tx(&full[st], C::STAGE_BYTES);
+      tma_load_2d(sF + st * C::F_BYTES, mapF, &full[st], kb * BK, fy);
       if constexpr (DUAL) {
-        tma_load_2d(sB + s * C::B_BYTES, &tmB0, &full[s], kb * BK, by);
-        tma_load_2d(sB + s * C::B_BYTES + C::B_TILE, &tmB1, &full[s], kb * BK, by);
+        tma_load_2d(sR + st * C::R_BYTES, &tmR0, &full[st], kb * BK, ry);
+        tma_load_2d(sR + st * C::R_BYTES + C::R_TILE, &tmR1, &full[st], kb * BK, ry);
       } else {
-        const bool b_second = kb >= b_split_kb;
-        tma_load_2d(sB + s * C::B_BYTES, b_second ? &tmB1 : &tmB0, &full[s],
-                    (b_second ? kb - b_split_kb : kb) * BK, by);
+        const bool r_second = kb >= r_split_kb;
+        tma_load_2d(sR + st * C::R_BYTES, r_second ? &tmR1 : &tmR0, &full[st],
+                    (r_second ? kb - r_split_kb : kb) * BK, ry);
       }
       ++issued;
     }
     if (*abort_flag) {
       // let copies already in flight land before the CTA gives up its shared memory
-      for (int kb = issued > C::STAGES ? issued - C::STAGES : 0; kb < issued; ++kb)
-        mbar_wait(&full[kb % C::STAGES], (uint32_t)(kb / C::STAGES) & 1u, nullptr, 20000000ull);
+      for (int i = issued > stages ? issued - stages : 0; i < issued; ++i)
+        mbar_wait(&full[i % stages], (uint32_t)(i / stages) & 1u, nullptr, 20000000ull);
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1 && lane == 0 && nkb > 0) {
     // ---- MMA issuer (single elected thread) ----
-    for (int kb = 0; kb < kb_total; ++kb) {
-      const int s = kb % C::STAGES;
-      const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
-      if (!mbar_wait(&full[s], ph, abort_flag)) {
+    for (int i = 0; i < nkb; ++i) {
+      const int st = i % stages;
+      const uint32_t ph = (uint32_t)(i / stages) & 1u;
+      if (!mbar_wait(&full[st], ph, abort_flag)) {
         *abort_flag = 1;
         break;
       }
       tc_fence_after();
-      const uint64_t adesc = sw128_desc(smem_u32(sA + s * C::A_BYTES));
-      const uint64_t bdesc = sw128_desc(smem_u32(sB + s * C::B_BYTES));
+      const uint64_t adesc = sw128_desc(smem_u32(sR + st * C::R_BYTES));
+      const uint64_t bdesc = sw128_desc(smem_u32(sF + st * C::F_BYTES));
 #pragma unroll
       for (int k = 0; k < BK / UMMA_K; ++k) {
         // advance the start address by k * 32 bytes inside the swizzle atom
         umma_bf16(tmem_base, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
-                  (kb > 0 || k > 0) ? 1u : 0u);
+                  (i > 0 || k > 0) ? 1u : 0u);
         if constexpr (DUAL) {
-          const uint64_t bdesc_lo = sw128_desc(smem_u32(sB + s * C::B_BYTES + C::B_TILE));
-          umma_bf16(tmem_base, adesc + (uint64_t)(2 * k), bdesc_lo + (uint64_t)(2 * k), C::IDESC,
+          const uint64_t adesc_lo = sw128_desc(smem_u32(sR + st * C::R_BYTES + C::R_TILE));
+          umma_bf16(tmem_base, adesc_lo + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
                     1u);
         }
       }
-      umma_commit(&empty[s]);       // frees this stage once its MMAs have read it
+      umma_commit(&empty[st]);      // frees this stage once its MMAs have read it
     }
     umma_commit(accum);             // all issued MMAs complete -> accumulator ready
   }
 
-  // ---- epilogue: all warps ----
+  // ---- epilogue: all warps; thread = one row of the tile ----
   __syncwarp();
-  const bool waited = mbar_wait(accum, 0, abort_flag);
-  // warp-uniform decision: tcgen05.ld below is a .sync.aligned instruction
-  const bool ok = __all_sync(0xffffffffu, waited && *abort_flag == 0);
-  if (!ok) {
-    if (lane == 0) atomicOr(args.err, kErrTimeout);
-  } else {
-    tc_fence_after();
-    const int m = m0 + warp * 32 + lane;
-    const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16);
-    float key_scale = 0.0f;
-    if constexpr (EPI == kEpiStoreKeys) {
-      // RMS of this feature over the tile's tokens: the magnitude of the
-      // partial sums, which sets the size of the accumulation error
-      float ss = 0.0f;
-      int cnt = 0;
+  bool ok = true;
+  if (nkb > 0) {
+    const bool waited = mbar_wait(accum, 0, abort_flag);
+    // warp-uniform decision: tcgen05.ld below is a .sync.aligned instruction
+    ok = __all_sync(0xffffffffu, waited && *abort_flag == 0);
+  }
+  if (!ok && lane == 0) atomicOr(args.err, kErrTimeout);
+  tc_fence_after();
+  const int row_in_tile = warp * 32 + lane;
+  const int n = n0 + row_in_tile;
+  const bool row_ok = n < g.n;
+  const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16);
+  const int n_cols = min(BN, m_end - m0);
+
+  if (S == 1) {
+    if (ok) {
+      float key_scale = 0.0f;
+      if constexpr (EPI == kEpiStoreKeys) {
+        float ss = 0.0f;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          float v[32];
+          tmem_ld32(taddr + (uint32_t)c0, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (c0 + j < n_cols) ss = fmaf(v[j], v[j], ss);
+        }
+        key_scale = sqrtf(ss / (float)max(n_cols, 1));
+      }
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
-        if (n0 + c0 >= g.n) break;
+        if (c0 >= n_cols) break;                    // uniform across the warp
         float v[32];
         tmem_ld32(taddr + (uint32_t)c0, v);
+        if (row_ok) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-          if (n0 + c0 + j < g.n) { ss = fmaf(v[j], v[j], ss); ++cnt; }
-      }
-      key_scale = sqrtf(ss / (float)max(cnt, 1));
-    }
-#pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 32) {
-      if (n0 + c0 >= g.n) break;                    // uniform across the warp
-      float v[32];
-      tmem_ld32(taddr + (uint32_t)c0, v);
-      if (m < m_end) {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int n = n0 + c0 + j;
-          if (n < g.n) {
-            if constexpr (EPI == kEpiStoreKeys) store_key(args, g, m, n, v[j], key_scale);
-            else gemm_epilogue<__nv_bfloat16, EPI>(args, g, m, n, v[j]);
+          for (int j = 0; j < 32; ++j) {
+            if (c0 + j < n_cols) {
+              if constexpr (EPI == kEpiStoreKeys) store_key(args, g, m0 + c0 + j, n, v[j], key_scale);
+              else gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + c0 + j, n, v[j]);
+            }
           }
         }
+      }
+    }
+  } else {
+    // ---- split K: partial tiles through global scratch ----
+    const long long tile_id =
+        ((long long)blockIdx.z * gridDim.y + blockIdx.y) * (gridDim.x / S) + tx;
+    float* base = args.partials + tile_id * S * (long long)(BM * BN);   // [S][BN][BM]
+    float* mine = base + (long long)rank * BN * BM;
+    const bool have_acc = ok && nkb > 0;          // warp-uniform
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      float v[32];
+      if (have_acc) {
+        tmem_ld32(taddr + (uint32_t)c0, v);       // the whole warp, converged
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+      }
+      if (row_ok) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) mine[(c0 + j) * BM + row_in_tile] = v[j];
+      }
+    }
+    // arrive, then wait (bounded) until the tile's S partials are written
+    __threadfence();
+    __syncthreads();
+    int* arrive = args.tile_sync + 2 * tile_id;
+    __shared__ int s_go;
+    if (threadIdx.x == 0) {
+      atomicAdd(arrive, 1);
+      int go = 1;
+      if (ld_acquire_gpu(arrive) < S) {
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire_gpu(arrive) < S) {
+          if (globaltimer_ns() - t0 > 2000000000ull) {
+            go = 0;
+            atomicOr(args.err, kErrTimeout);
+            break;
+          }
+        }
+      }
+      s_go = go;
+    }
+    __syncthreads();
+    // CTA `rank` owns columns [rank cpo, (rank+1) cpo); work items are
+    // (column, 4 rows); each item issues its S independent loads first, then
+    // sums them in rank order.
+    const int cpo = BN / S;
+    const int rows_real = min(BM, g.n - n0);
+    const int rgroups = (rows_real + 3) / 4;
+    if (ok && s_go) {
+      for (int it = threadIdx.x; it < cpo * rgroups; it += kThreads) {
+        const int cl = it / rgroups;
+        const int r4 = (it - cl * rgroups) * 4;
+        const int col = (int)rank * cpo + cl;
+        if (col >= n_cols) continue;
+        float4 part[16];
+#pragma unroll
+        for (int src = 0; src < 16; ++src)
+          if (src < S)
+            part[src] = __ldcg(reinterpret_cast<const float4*>(
+                base + ((long long)src * BN + col) * BM + r4));
+        float4 acc = part[0];
+#pragma unroll
+        for (int src = 1; src < 16; ++src)
+          if (src < S) {
+            acc.x += part[src].x;
+            acc.y += part[src].y;
+            acc.z += part[src].z;
+            acc.w += part[src].w;
+          }
+        const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (r4 + j < rows_real) gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + col, n0 + r4 + j, vals[j]);
+      }
+    }
+    // leave; the last CTA of the tile resets its counters for the next launch
+    __syncthreads();
+    if (threadIdx.x == 0 && s_go) {
+      if (atomicAdd(arrive + 1, 1) == S - 1) {
+        atomicExch(arrive, 0);
+        atomicExch(arrive + 1, 0);
       }
     }
   }
@@ -403,58 +523,174 @@ static bool make_map(CUtensorMap* m, const TmaOperand& op, int box_rows) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+static int num_sms() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+  }
+  return sms;
+}
+
 template <int BN, int EPI>
-static cudaError_t launch_tc_inst(const GemmArgs& a, const CUtensorMap* maps, int max_m, int max_n,
-                                  cudaStream_t s) {
-  using C = tc::Cfg<BN, EPI == kEpiScores>;
+static auto tc_kernel() {
+  auto kern = tc::tc_gemm_kernel<BN, EPI>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tc::tc_gemm_kernel<BN, EPI>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-    if (e != cudaSuccess) return e;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc::kSmemBudget + tc::kSmemExtra);
     configured = true;
   }
-  const int tiles_m = a.a_split >= max_m
-                          ? (max_m + tc::BM - 1) / tc::BM
-                          : (a.a_split + tc::BM - 1) / tc::BM + (max_m - a.a_split + tc::BM - 1) / tc::BM;
-  dim3 grid(tiles_m, (max_n + BN - 1) / BN, a.ngroups);
-  tc::tc_gemm_kernel<BN, EPI><<<grid, tc::kThreads, C::SMEM, s>>>(maps[0], maps[1], maps[2], maps[3],
-                                                                  a);
-  return cudaGetLastError();
+  return kern;
+}
+
+template <int BN, bool DUAL>
+static int stages_for(int nkb, int budget) {
+  using C = tc::Cfg<BN, DUAL>;
+  int st = budget / C::STAGE_BYTES;
+  st = st > tc::kMaxStages ? tc::kMaxStages : st;
+  st = st > nkb ? nkb : st;
+  return st < 1 ? 1 : st;
+}
+
+// CTAs of this kernel that can be resident on the GPU at once.
+template <int BN, int EPI>
+static int resident_ctas(int smem) {
+  static int cache[64];      // by smem / 4 KB
+  const int mi = (smem >> 12) & 63;
+  if (cache[mi] != 0) return cache[mi];
+  auto kern = tc_kernel<BN, EPI>();
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, tc::kThreads, smem) !=
+          cudaSuccess || per_sm <= 0) {
+    cudaGetLastError();
+    per_sm = 1;
+  }
+  cache[mi] = per_sm * num_sms();
+  return cache[mi];
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tiles_x, int max_n,
+                                  int splits, int stages, cudaStream_t s) {
+  using C = tc::Cfg<BN, EPI == kEpiScores>;
+  auto kern = tc_kernel<BN, EPI>();
+  a.splits = splits;
+  a.stages = stages;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles_x * splits, (max_n + tc::BM - 1) / tc::BM, a.ngroups);
+  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = stages * C::STAGE_BYTES + tc::kSmemExtra;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  cfg.attrs = attr;
+  cfg.numAttrs = 0;
+  if (splits > 1) {
+    // the CTAs of a tile wait for one another: the whole grid must be resident
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.numAttrs = 1;
+  }
+  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], a);
 }
 
 template <int EPI>
-static cudaError_t launch_tc_epi(const GemmArgs& a, const CUtensorMap* maps, int bn, int max_m,
-                                 int max_n, cudaStream_t s) {
-  switch (bn) {
-    case 32: return launch_tc_inst<32, EPI>(a, maps, max_m, max_n, s);
-    case 64: return launch_tc_inst<64, EPI>(a, maps, max_m, max_n, s);
-    case 128: return launch_tc_inst<128, EPI>(a, maps, max_m, max_n, s);
-    default: return launch_tc_inst<256, EPI>(a, maps, max_m, max_n, s);
+static cudaError_t launch_tc_epi(GemmArgs& a, const CUtensorMap* maps, const GemmPlan& p,
+                                 int tiles_x, int max_n, cudaStream_t s) {
+  switch (p.bn) {
+    case 64: return launch_tc_inst<64, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
+    case 128: return launch_tc_inst<128, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
+    default: return launch_tc_inst<256, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
   }
 }
 
-cudaError_t launch_gemm_tc(int epi, const GemmArgs& a, const TmaOperand& A0, const TmaOperand& A1,
+static int feature_tiles(const GemmArgs& a, int max_m, int bn) {
+  return a.a_split >= max_m ? (max_m + bn - 1) / bn
+                            : (a.a_split + bn - 1) / bn + (max_m - a.a_split + bn - 1) / bn;
+}
+
+template <int BN, int EPI>
+static void plan_for(const GemmArgs& a, int max_m, long long row_tiles, GemmPlan& best,
+                     long long& best_score) {
+  constexpr bool DUAL = EPI == kEpiScores;
+  const int kb_total = a.k_total / tc::BK;
+  const long long tiles = (long long)feature_tiles(a, max_m, BN) * row_tiles;
+  const long long useful = BN < max_m ? BN : max_m;      // real features per tile (bound)
+  const int sms = num_sms();
+  for (int splits = 1; splits <= 16; splits *= 2) {
+    if (splits > 1 && (EPI == kEpiStoreKeys || splits > kb_total || splits > BN)) break;
+    const int nkb = (kb_total + splits - 1) / splits;
+    const long long ctas = tiles * splits;
+    // one CTA per SM while the grid fits on the SMs, else the pair budget
+    int stages = stages_for<BN, DUAL>(nkb, ctas <= sms ? tc::kSmemBudget : tc::kSmemBudgetPair);
+    if (stages < 2 && nkb >= 2) stages = stages_for<BN, DUAL>(nkb, tc::kSmemBudget);
+    const int smem = stages * tc::Cfg<BN, DUAL>::STAGE_BYTES + tc::kSmemExtra;
+    const long long cap = resident_ctas<BN, EPI>(smem);
+    if (splits > 1 && ctas > cap) break;               // a cooperative grid must be resident
+    // weight bytes consumable per MMA time over the CTAs that run at once; a
+    // tie goes to more CTAs (more bytes in flight)
+    const long long run = ctas < sms ? ctas : sms;
+    const long long score = (run * useful) * 4096 + run;
+    if (score > best_score) {
+      best_score = score;
+      best = GemmPlan{BN, splits, stages, 0, 0};
+    }
+  }
+}
+
+template <int EPI>
+static GemmPlan plan_epi(const GemmArgs& a, int max_m, int max_n) {
+  const long long row_tiles = (long long)(max_n + tc::BM - 1) / tc::BM * a.ngroups;
+  GemmPlan best{256, 1, 2, 0, 0};
+  long long best_score = -1;
+  plan_for<256, EPI>(a, max_m, row_tiles, best, best_score);
+  plan_for<128, EPI>(a, max_m, row_tiles, best, best_score);
+  plan_for<64, EPI>(a, max_m, row_tiles, best, best_score);
+  if (best.splits > 1) {
+    best.tiles = (long long)feature_tiles(a, max_m, best.bn) * row_tiles;
+    best.partial_floats = best.tiles * best.splits * tc::BM * best.bn;
+  }
+  return best;
+}
+
+GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
+  switch (epi) {
+    case kEpiStore: return plan_epi<kEpiStore>(a, max_m, max_n);
+    case kEpiScores: return plan_epi<kEpiScores>(a, max_m, max_n);
+    case kEpiBiasSilu: return plan_epi<kEpiBiasSilu>(a, max_m, max_n);
+    case kEpiStoreHiLo: return plan_epi<kEpiStoreHiLo>(a, max_m, max_n);
+    case kEpiStoreKeys: return plan_epi<kEpiStoreKeys>(a, max_m, max_n);
+    default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
+  }
+}
+
+cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, const TmaOperand& A1,
                            const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
                            cudaStream_t s) {
-  if (max_m <= 0 || max_n <= 0 || a.ngroups <= 0) return cudaSuccess;
-  const int bn = max_n <= 32 ? 32 : max_n <= 64 ? 64 : max_n <= 128 ? 128 : 256;
+  if (max_m <= 0 || max_n <= 0 || args.ngroups <= 0) return cudaSuccess;
+  static thread_local GemmArgs a;
+  a = args;
+  const GemmPlan plan = plan_gemm_tc(epi, a, max_m, max_n);
+  if (plan.splits > 1 && (a.partials == nullptr || a.partials_floats < plan.partial_floats ||
+                          a.tile_sync == nullptr || a.tile_sync_tiles < plan.tiles))
+    return cudaErrorInvalidValue;             // the caller sized the scratch with plan_gemm_tc
   CUtensorMap maps[4];
   const TmaOperand& a1 = A1.base ? A1 : A0;
   const TmaOperand& b1 = B1.base ? B1 : B0;
-  if (!make_map(&maps[0], A0, tc::BM) || !make_map(&maps[1], a1, tc::BM) ||
-      !make_map(&maps[2], B0, bn) || !make_map(&maps[3], b1, bn))
+  if (!make_map(&maps[0], A0, plan.bn) || !make_map(&maps[1], a1, plan.bn) ||
+      !make_map(&maps[2], B0, tc::BM) || !make_map(&maps[3], b1, tc::BM))
     return cudaErrorInvalidValue;
-  cudaError_t e;
+  const int tiles_x = feature_tiles(a, max_m, plan.bn);
   switch (epi) {
-    case kEpiStore: e = launch_tc_epi<kEpiStore>(a, maps, bn, max_m, max_n, s); break;
-    case kEpiScores: e = launch_tc_epi<kEpiScores>(a, maps, bn, max_m, max_n, s); break;
-    case kEpiBiasSilu: e = launch_tc_epi<kEpiBiasSilu>(a, maps, bn, max_m, max_n, s); break;
-    case kEpiStoreHiLo: e = launch_tc_epi<kEpiStoreHiLo>(a, maps, bn, max_m, max_n, s); break;
-    case kEpiStoreKeys: e = launch_tc_epi<kEpiStoreKeys>(a, maps, bn, max_m, max_n, s); break;
-    default: e = launch_tc_epi<kEpiBiasF32>(a, maps, bn, max_m, max_n, s); break;
+    case kEpiStore: return launch_tc_epi<kEpiStore>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiScores: return launch_tc_epi<kEpiScores>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiBiasSilu: return launch_tc_epi<kEpiBiasSilu>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiStoreHiLo: return launch_tc_epi<kEpiStoreHiLo>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiStoreKeys: return launch_tc_epi<kEpiStoreKeys>(a, maps, plan, tiles_x, max_n, s);
+    default: return launch_tc_epi<kEpiBiasF32>(a, maps, plan, tiles_x, max_n, s);
   }
-  return e;
 }
 
 }  // namespace fovea

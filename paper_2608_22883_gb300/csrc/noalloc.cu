@@ -63,8 +63,9 @@ extern "C" FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(
   }
   void* ws = nullptr;
   if ((st = workspace_address(&ws)) != FOVEA_OK) return st;
-  // The array keeps the previous call's contents: the error word must start at zero.
-  cudaError_t e = cudaMemsetAsync(ws, 0, 256, static_cast<cudaStream_t>(stream));
+  // The array keeps the previous call's contents: the header (error word and
+  // split-K counters) must start at zero.
+  cudaError_t e = cudaMemsetAsync(ws, 0, 16384, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {
     char msg[256];
     snprintf(msg, sizeof(msg), "cudaMemsetAsync: %s", cudaGetErrorString(e));
