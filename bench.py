@@ -302,42 +302,75 @@ def main():
     counts = torch.empty(N, dtype=torch.int32, device=dev)
     indices = torch.empty((N, K), dtype=torch.int32, device=dev)
     offs_c = fovea._offsets(w.row_offsets)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.int32, device=dev)
+    h_in = torch.empty_like(h)          # the step reads its inputs from here
+    depth_in = torch.empty_like(depth)
+    h_in.copy_(h)
+    depth_in.copy_(depth)
+
+    def step():
+        fovea.retrieve_fuse(params, mem, h_in, depth_in, w.row_offsets, row_scale, w.rho, w.k_min,
+                            K, h_out, ws, counts=counts, indices=indices, offsets_c=offs_c)
+
+    def flush(i):
+        # evict everything: write 512 MB, then read 256 MB so the lines L2 holds
+        # when the step starts are clean (no write-back charged to the step)
+        flush_w.fill_(i & 0xFF)
+        flush_r.sum()
+
+    # The step is replayed from a CUDA graph (one launch per step), the form a
+    # decoding loop uses; the graph holds exactly the kernels of one call.
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        for _ in range(3):
+            step()
+    torch.cuda.current_stream().wait_stream(cap)
+    torch.cuda.synchronize()
+    g_plain = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_plain, stream=cap):
+        step()
+    fovea.timing_enable(True)            # per-kernel event nodes in the timed graph
+    g_timed = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_timed, stream=cap):
+        step()
+    torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
 
-    def step(hh=h, dd=depth):
-        fovea.retrieve_fuse(params, mem, hh, dd, w.row_offsets, row_scale, w.rho, w.k_min, K,
-                            h_out, ws, counts=counts, indices=indices, offsets_c=offs_c)
-
     for i in range(args.warmup):
-        flush.fill_(i & 0xFF)
-        step()
+        flush(i)
+        g_timed.replay()
     torch.cuda.synchronize()
     fovea.sync_errors(ws)
 
     # ---- timed region: K steps, L2 flushed before each (outside the events) ----
-    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(local)
     clocks.start()
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
-    fovea.timing_enable(True)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    step_ms = []
+    per_kernel = {}
     t_wall = time.perf_counter()
     for i in range(args.steps):
-        flush.fill_((i + 7) & 0xFF)
-        ev0[i].record(stream)
-        step()
-        ev1[i].record(stream)
+        flush(i + 7)
+        e0.record(stream)
+        g_timed.replay()
+        e1.record(stream)
+        e1.synchronize()
+        step_ms.append(e0.elapsed_time(e1))
+        for name, (tot, n) in fovea.timing_read().items():
+            a = per_kernel.setdefault(name, [0.0, 0])
+            a[0] += tot
+            a[1] += n
     torch.cuda.synchronize()
     wall_s = time.perf_counter() - t_wall
     if dist is not None:
         dist.barrier()
     clk = clocks.stop()
-    per_kernel = fovea.timing_read()
-    fovea.timing_enable(False)
-    step_ms = [a.elapsed_time(b) for a, b in zip(ev0, ev1)]
     ms = float(np.mean(step_ms))
     fovea.sync_errors(ws)
     if dist is not None:
@@ -346,40 +379,39 @@ def main():
         ms = float(t.item())
     value = world * N / (ms / 1000.0)
 
-    # ---- untimed-kernel step (for the step's own duration without event hooks) ----
-    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(min(args.steps, 500))]
-    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(len(ev_a))]
-    for i in range(len(ev_a)):
-        flush.fill_(i & 0xFF)
-        ev_a[i].record(stream)
-        step()
-        ev_b[i].record(stream)
-    torch.cuda.synchronize()
-    ms_nohooks = float(np.mean([a.elapsed_time(b) for a, b in zip(ev_a, ev_b)]))
+    # ---- the same step from a graph without the per-kernel event nodes ----
+    n_plain = min(args.steps, 500)
+    plain_ms = []
+    for i in range(n_plain):
+        flush(i)
+        e0.record(stream)
+        g_plain.replay()
+        e1.record(stream)
+        e1.synchronize()
+        plain_ms.append(e0.elapsed_time(e1))
+    ms_nohooks = float(np.mean(plain_ms))
 
-    # ---- end to end through the C ABI with host buffers ----
+    # ---- end to end: host buffers in, graph step, results back to host ----
     h_out_host = torch.empty(h_out.shape, dtype=h_out.dtype).pin_memory()
     counts_host = torch.empty(N, dtype=torch.int32).pin_memory()
     idx_host = torch.empty((N, K), dtype=torch.int32).pin_memory()
-    n_e2e = min(args.steps, 500)
-    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
-    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(n_e2e)]
-    h_dev2 = torch.empty_like(h)
-    depth_dev2 = torch.empty_like(depth)
-    for i in range(n_e2e):
-        flush.fill_(i & 0xFF)
-        e0[i].record(stream)
-        h_dev2.copy_(h_host, non_blocking=True)
-        depth_dev2.copy_(depth_host, non_blocking=True)
-        step(h_dev2, depth_dev2)
+    e2e_ms_l = []
+    for i in range(n_plain):
+        flush(i)
+        e0.record(stream)
+        h_in.copy_(h_host, non_blocking=True)
+        depth_in.copy_(depth_host, non_blocking=True)
+        g_plain.replay()
         h_out_host.copy_(h_out, non_blocking=True)
         counts_host.copy_(counts, non_blocking=True)
         idx_host.copy_(indices, non_blocking=True)
-        e1[i].record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = float(np.mean([a.elapsed_time(b) for a, b in zip(e0, e1)]))
+        e1.record(stream)
+        e1.synchronize()
+        e2e_ms_l.append(e0.elapsed_time(e1))
+    e2e_ms = float(np.mean(e2e_ms_l))
     h2d = h_host.numel() * h_host.element_size() + depth_host.numel() * 4
     d2h = h_out_host.numel() * h_out_host.element_size() + N * 4 + N * K * 4
+    assert torch.equal(h_out_host, h_out.cpu())
 
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
@@ -413,7 +445,8 @@ def main():
         "config": {"workload": w.name, "d_model": w.d, "memory_entries": w.m_sizes,
                    "draft_states": N, "sequences": w.B, "rho": w.rho, "k_min": w.k_min,
                    "k_max": K, "mlp_hidden": int(w.params["b_f1"].shape[0]),
-                   "l2": "flushed before every step (512 MB write outside the per-step events)",
+                   "l2": "flushed before every step outside the per-step events (512 MB write, then a 256 MB read so the evicted lines are clean)",
+                   "launch": "one CUDA graph replay per step (the kernels of one fovea_retrieve_fuse call)",
                    "parallelism": f"replicas x{world}"},
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved,
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],

@@ -249,7 +249,11 @@ FOVEA_API const char* fovea_last_error(void);
  * library (off by default; for measurement only).  fovea_timing_enable(1)
  * clears the records and starts recording; fovea_timing_read synchronises the
  * recorded events and fills up to `capacity` entries of kernel name, total
- * milliseconds and launch count; it returns the number of distinct kernels. */
+ * milliseconds and launch count; it returns the number of distinct kernels.
+ * Launches recorded while the stream is captured into a CUDA graph become
+ * external event nodes of the graph: after each replay, fovea_timing_read
+ * returns that replay's durations.  Keep timing enabled (do not call
+ * fovea_timing_enable again) while such a graph is still replayed. */
 FOVEA_API fovea_status fovea_timing_enable(int enable);
 FOVEA_API int fovea_timing_read(const char** names, double* total_ms, int* launches,
                                 int capacity);

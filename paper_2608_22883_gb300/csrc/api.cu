@@ -74,15 +74,20 @@ bool capturing(cudaStream_t s) {
   return st != cudaStreamCaptureStatusNone;
 }
 
-struct KernelTimer {   // records start/stop events around one launch when enabled
+// Records start/stop events around one launch when timing is enabled.  While
+// the stream is being captured into a CUDA graph the records become external
+// event nodes of the graph, re-recorded by every replay.
+struct KernelTimer {
   const char* name;
   cudaStream_t s;
-  bool on;
-  KernelTimer(const char* n, cudaStream_t st) : name(n), s(st), on(false) {
+  bool on, graph;
+  KernelTimer(const char* n, cudaStream_t st) : name(n), s(st), on(false), graph(false) {
     std::lock_guard<std::mutex> lk(g_tmu);
-    if (!g_timing || capturing(s)) return;
+    if (!g_timing) return;
+    graph = capturing(s);
     TimingRec r{name, take_event(), take_event()};
-    cudaEventRecord(r.start, s);
+    if (graph) cudaEventRecordWithFlags(r.start, s, cudaEventRecordExternal);
+    else cudaEventRecord(r.start, s);
     g_recs.push_back(r);
     on = true;
   }
@@ -91,7 +96,8 @@ struct KernelTimer {   // records start/stop events around one launch when enabl
     std::lock_guard<std::mutex> lk(g_tmu);
     for (auto it = g_recs.rbegin(); it != g_recs.rend(); ++it)
       if (it->name == name) {
-        cudaEventRecord(it->stop, s);
+        if (graph) cudaEventRecordWithFlags(it->stop, s, cudaEventRecordExternal);
+        else cudaEventRecord(it->stop, s);
         break;
       }
   }

@@ -27,6 +27,16 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 
 __device__ __forceinline__ float sigmoidf_(float z) { return 1.0f / (1.0f + expf(-z)); }
 
+// Programmatic dependent launch: kernels of the step are launched so that a
+// kernel may start while its predecessor finishes.  pdl_wait() blocks until
+// the predecessor grid has completed and its writes are visible; a kernel
+// calls it before it reads anything the predecessor wrote and before it
+// writes anything.  pdl_trigger() lets the successor begin its own prologue.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------
 // Reductions (fixed order, so results are run-to-run deterministic)
 // ---------------------------------------------------------------------------
@@ -137,6 +147,23 @@ __device__ __forceinline__ int seq_of_row(const SeqTable& t, int row) {
 // ---------------------------------------------------------------------------
 // Host-side launch interfaces (defined in the kernel translation units)
 // ---------------------------------------------------------------------------
+
+// Launches `kern` on `s` with the programmatic-dependent-launch attribute.
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
 
 // Sets the message fovea_last_error() returns on this thread (api.cu).
 fovea_status report_error(fovea_status st, const char* msg);

@@ -34,6 +34,11 @@
 // the S partials of columns [r BN/S, (r+1) BN/S) in rank order (so the result
 // does not depend on timing) and runs the epilogue for them.  The last CTA to
 // leave resets the tile's counters for the next launch.
+//
+// Launch overlap: kernels are launched with programmatic dependent launch.
+// The producer issues the feature-operand (weight / key) loads of the first
+// stages before griddepcontrol.wait; those operands never depend on the
+// previous kernel, so the weight stream starts while the predecessor drains.
 #include "gemm_epilogue.cuh"
 
 namespace fovea {
@@ -294,17 +299,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     const CUtensorMap* mapF = f_second ? &tmF1 : &tmF0;
     const int fy = f_second ? m0 - split : g.a_row0 + m0;
     const int ry = g.b_row0 + n0;
+    // weights / keys of the first stages: independent of the previous kernel
+    const int pre = nkb < stages ? nkb : stages;
+    for (int i = 0; i < pre; ++i) {
+      mbar_expect_tx(&full[i], C::STAGE_BYTES);
+      tma_load_2d(sF + i * C::F_BYTES, mapF, &full[i], (kb_lo + i) * BK, fy);
+    }
+    pdl_wait();
+    pdl_trigger();
     int issued = 0;
     for (int i = 0; i < nkb; ++i) {
       const int kb = kb_lo + i;
       const int st = i % stages;
       const uint32_t ph = (uint32_t)(i / stages) & 1u;
-      if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
-        *abort_flag = 1;
-        break;
+      if (i >= pre) {
+        if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
+          *abort_flag = 1;
+          break;
+        }
+        mbar_expect_tx(&full[st], C::STAGE_BYTES);
+        tma_load_2d(sF + st * C::F_BYTES, mapF, &full[st], kb * BK, fy);
       }
-      mbar_expect_tx(&full[st], C::STAGE_BYTES);
-      tma_load_2d(sF + st * C::F_BYTES, mapF, &full[st], kb * BK, fy);
       if constexpr (DUAL) {
         tma_load_2d(sR + st * C::R_BYTES, &tmR0, &full[st], kb * BK, ry);
         tma_load_2d(sR + st * C::R_BYTES + C::R_TILE, &tmR1, &full[st], kb * BK, ry);
@@ -349,6 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ---- epilogue: all warps; thread = one row of the tile ----
+  pdl_wait();
   __syncwarp();
   bool ok = true;
   if (nkb > 0) {
@@ -467,7 +483,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          if (r4 + j < rows_real) gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + col, n0 + r4 + j, vals[j]);
+          if (r4 + j < rows_real)
+            gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + col, n0 + r4 + j, vals[j]);
       }
     }
     // leave; the last CTA of the tile resets its counters for the next launch
@@ -584,14 +601,16 @@ static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tile
   cfg.blockDim = dim3(tc::kThreads, 1, 1);
   cfg.dynamicSmemBytes = stages * C::STAGE_BYTES + tc::kSmemExtra;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 0;
+  cfg.numAttrs = 1;
   if (splits > 1) {
     // the CTAs of a tile wait for one another: the whole grid must be resident
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.numAttrs = 1;
+    attr[1].id = cudaLaunchAttributeCooperative;
+    attr[1].val.cooperative = 1;
+    cfg.numAttrs = 2;
   }
   return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], a);
 }

@@ -8,33 +8,43 @@ namespace fovea {
 
 // ---------------------------------------------------------------------------
 // LN over rows of d elements (memory equation: LN(v_i); query equation:
-// LN(h_n) + E_dep[l_n]).  One CTA per row; the row stays in registers.
-// Mean, variance, 1/sqrt and the affine map are evaluated in double-float so
-// the single rounding to the stored type is taken on an almost exact value
-// (the same value a float64 evaluation rounds).  Optional gather of source
-// rows, optional depth embedding (depth checked against [0, D]; an invalid
-// depth sets kErrDepth and uses depth 0).
+// LN(h_n) + E_dep[l_n]).  One CTA per row.  A single pass accumulates sum(x)
+// and sum(x^2) in double-float (the square of a stored value is formed
+// exactly with an FMA), one block reduction gives mean and variance
+// (var = E[x^2] - mean^2, free of cancellation at double-float precision),
+// and the affine map is evaluated in double-float, so the single rounding to
+// the stored type is taken on an almost exact value (the value a float64
+// evaluation rounds).  16-byte vector loads; the row, gamma, beta and the
+// depth embedding are all requested before any arithmetic.  Optional gather
+// of source rows; an invalid depth sets kErrDepth and uses depth 0.
 // ---------------------------------------------------------------------------
-constexpr int kLnThreads = 256;
-constexpr int kLnMaxPerThread = FOVEA_MAX_D / kLnThreads;
+constexpr int kLnThreads = 512;
 
-__device__ __forceinline__ dfloat block_sum_df(dfloat v, dfloat* scratch) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+template <class T> struct LnVec;     // elements per 16-byte vector, vectors per thread
+template <> struct LnVec<__nv_bfloat16> {
+  static constexpr int N = 8, MAX = FOVEA_MAX_D / 8 / kLnThreads;
+};
+template <> struct LnVec<float> {
+  static constexpr int N = 4, MAX = FOVEA_MAX_D / 4 / kLnThreads;
+};
+
+template <class T>
+__device__ __forceinline__ void ln_load(const T* p, float (&v)[LnVec<T>::N]);
+template <>
+__device__ __forceinline__ void ln_load<__nv_bfloat16>(const __nv_bfloat16* p, float (&v)[8]) {
+  const uint4 raw = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const dfloat t = {__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)};
-    v = df_add(v, t);
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(h2[i]);
+    v[2 * i] = f.x;
+    v[2 * i + 1] = f.y;
   }
-  __syncthreads();
-  if (lane == 0) scratch[warp] = v;
-  __syncthreads();
-  dfloat t = lane < nw ? scratch[lane] : dfloat{0.0f, 0.0f};
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const dfloat u = {__shfl_xor_sync(0xffffffffu, t.hi, o), __shfl_xor_sync(0xffffffffu, t.lo, o)};
-    t = df_add(t, u);
-  }
-  return t;
+}
+template <>
+__device__ __forceinline__ void ln_load<float>(const float* p, float (&v)[4]) {
+  const float4 raw = *reinterpret_cast<const float4*>(p);
+  v[0] = raw.x; v[1] = raw.y; v[2] = raw.z; v[3] = raw.w;
 }
 
 template <class T> __device__ __forceinline__ T df_store(dfloat y);
@@ -43,54 +53,106 @@ template <> __device__ __forceinline__ __nv_bfloat16 df_store<__nv_bfloat16>(dfl
   return df_to_bf16(y);
 }
 
+__device__ __forceinline__ dfloat warp_sum_df(dfloat v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const dfloat t = {__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)};
+    v = df_add(v, t);
+  }
+  return v;
+}
+
 template <class T>
 __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
     const T* __restrict__ x, const int32_t* __restrict__ src_row, int d,
     const T* __restrict__ gamma, const T* __restrict__ beta, float eps,
     const T* __restrict__ E, const int32_t* __restrict__ depth, int max_depth, int* err,
     T* __restrict__ out) {
-  __shared__ dfloat scratch[32];
+  constexpr int V = LnVec<T>::N;
+  constexpr int kLnMaxVec = LnVec<T>::MAX;
+  __shared__ dfloat red[2][kLnThreads / 32];
   const int row = blockIdx.x;
-  const long long src = src_row ? (long long)src_row[row] : (long long)row;
-  const T* xr = x + src * d;
-  float vals[kLnMaxPerThread];
-  dfloat s = {0.0f, 0.0f};
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nvec = d / V;
+  float xv[kLnMaxVec][V], gv[kLnMaxVec][V], bv[kLnMaxVec][V], ev[kLnMaxVec][V];
 #pragma unroll
-  for (int j = 0; j < kLnMaxPerThread; ++j) {
-    const int i = threadIdx.x + j * kLnThreads;
-    vals[j] = i < d ? to_f32(xr[i]) : 0.0f;
-    s = df_add_f(s, vals[j]);
-  }
-  const dfloat mean = df_div_f(block_sum_df(s, scratch), (float)d);
-  const dfloat neg_mean = {-mean.hi, -mean.lo};
-  dfloat ss = {0.0f, 0.0f};
-#pragma unroll
-  for (int j = 0; j < kLnMaxPerThread; ++j) {
-    const int i = threadIdx.x + j * kLnThreads;
-    if (i < d) {
-      const dfloat c = df_add_f(neg_mean, vals[j]);
-      ss = df_add(ss, df_mul(c, c));
+  for (int j = 0; j < kLnMaxVec; ++j) {      // weights: independent of the predecessor
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      ln_load<T>(gamma + vi * V, gv[j]);
+      ln_load<T>(beta + vi * V, bv[j]);
     }
   }
-  const dfloat var = df_div_f(block_sum_df(ss, scratch), (float)d);
-  const dfloat rstd = df_rsqrt(df_add_f(var, eps));
+  pdl_wait();
+  pdl_trigger();
+  const long long src = src_row ? (long long)src_row[row] : (long long)row;
   int dep = 0;
   if (E != nullptr) {
     dep = depth[row];
     if (dep < 0 || dep > max_depth) {
-      if (threadIdx.x == 0) atomicOr(err, kErrDepth);
+      if (tid == 0) atomicOr(err, kErrDepth);
       dep = 0;
     }
   }
+  const T* xr = x + src * d;
+  const T* er = E != nullptr ? E + (long long)dep * d : nullptr;
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      ln_load<T>(xr + vi * V, xv[j]);
+      if (er != nullptr) ln_load<T>(er + vi * V, ev[j]);
+    }
+  }
+  dfloat s1 = {0.0f, 0.0f}, s2 = {0.0f, 0.0f};
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    if (tid + j * kLnThreads < nvec) {
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        s1 = df_add_f(s1, xv[j][i]);
+        s2 = df_add(s2, df_two_prod(xv[j][i], xv[j][i]));
+      }
+    }
+  }
+  s1 = warp_sum_df(s1);
+  s2 = warp_sum_df(s2);
+  if (lane == 0) {
+    red[0][warp] = s1;
+    red[1][warp] = s2;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    constexpr int NW = kLnThreads / 32;
+    dfloat a = lane < NW ? red[0][lane] : dfloat{0.0f, 0.0f};
+    dfloat b = lane < NW ? red[1][lane] : dfloat{0.0f, 0.0f};
+    a = warp_sum_df(a);
+    b = warp_sum_df(b);
+    if (lane == 0) {
+      const dfloat mean = df_div_f(a, (float)d);
+      const dfloat ex2 = df_div_f(b, (float)d);
+      const dfloat var = df_add(ex2, df_mul(dfloat{-mean.hi, -mean.lo}, mean));
+      red[0][0] = mean;
+      red[1][0] = df_rsqrt(df_add_f(var, eps));
+    }
+  }
+  __syncthreads();
+  const dfloat neg_mean = {-red[0][0].hi, -red[0][0].lo};
+  const dfloat rstd = red[1][0];
   T* o = out + (long long)row * d;
 #pragma unroll
-  for (int j = 0; j < kLnMaxPerThread; ++j) {
-    const int i = threadIdx.x + j * kLnThreads;
-    if (i < d) {
-      dfloat y = df_mul(df_add_f(neg_mean, vals[j]), rstd);
-      y = df_add_f(df_mul_f(y, to_f32(gamma[i])), to_f32(beta[i]));
-      if (E != nullptr) y = df_add_f(y, to_f32(E[(long long)dep * d + i]));
-      o[i] = df_store<T>(y);
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      T res[V];
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        dfloat y = df_mul(df_add_f(neg_mean, xv[j][i]), rstd);
+        y = df_add_f(df_mul_f(y, gv[j][i]), bv[j][i]);
+        if (er != nullptr) y = df_add_f(y, ev[j][i]);
+        res[i] = df_store<T>(y);
+      }
+      *reinterpret_cast<uint4*>(o + vi * V) = *reinterpret_cast<const uint4*>(res);
     }
   }
 }
@@ -102,16 +164,13 @@ cudaError_t launch_ln_rows(int dtype, const void* x, const int32_t* src_row, int
   if (rows == 0) return cudaSuccess;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
-    ln_rows_kernel<T><<<rows, kLnThreads, 0, s>>>((const T*)x, src_row, d, (const T*)gamma,
-                                                  (const T*)beta, eps, (const T*)E, depth,
-                                                  max_depth, err, (T*)out);
-  } else {
-    ln_rows_kernel<float><<<rows, kLnThreads, 0, s>>>((const float*)x, src_row, d,
-                                                      (const float*)gamma, (const float*)beta,
-                                                      eps, (const float*)E, depth, max_depth,
-                                                      err, (float*)out);
+    return launch_pdl(ln_rows_kernel<T>, dim3(rows), dim3(kLnThreads), 0, s, (const T*)x, src_row,
+                      d, (const T*)gamma, (const T*)beta, eps, (const T*)E, depth, max_depth, err,
+                      (T*)out);
   }
-  return cudaGetLastError();
+  return launch_pdl(ln_rows_kernel<float>, dim3(rows), dim3(kLnThreads), 0, s, (const float*)x,
+                    src_row, d, (const float*)gamma, (const float*)beta, eps, (const float*)E,
+                    depth, max_depth, err, (float*)out);
 }
 
 // ---------------------------------------------------------------------------
@@ -219,6 +278,8 @@ __global__ void __launch_bounds__(kReadoutThreads) readout_kernel(
   constexpr int V = Vec16<T>::N;
   const int n = blockIdx.x;
   const int col = (blockIdx.y * kReadoutThreads + threadIdx.x) * V;
+  pdl_wait();
+  pdl_trigger();
   if (col >= d) return;
   const int K = sel_cnt[n];
   const int32_t* pos = sel_pos + (long long)n * k_max;
@@ -264,14 +325,12 @@ cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, con
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
     dim3 grid(N, (d / 8 + kReadoutThreads - 1) / kReadoutThreads);
-    readout_kernel<T><<<grid, kReadoutThreads, 0, s>>>((const T*)U, sel_cnt, sel_pos, sel_w, k_max,
-                                                       d, r_out, (T*)r_lo);
-  } else {
-    dim3 grid(N, (d / 4 + kReadoutThreads - 1) / kReadoutThreads);
-    readout_kernel<float><<<grid, kReadoutThreads, 0, s>>>((const float*)U, sel_cnt, sel_pos,
-                                                           sel_w, k_max, d, r_out, (float*)r_lo);
+    return launch_pdl(readout_kernel<T>, grid, dim3(kReadoutThreads), 0, s, (const T*)U, sel_cnt,
+                      sel_pos, sel_w, k_max, d, r_out, (T*)r_lo);
   }
-  return cudaGetLastError();
+  dim3 grid(N, (d / 4 + kReadoutThreads - 1) / kReadoutThreads);
+  return launch_pdl(readout_kernel<float>, grid, dim3(kReadoutThreads), 0, s, (const float*)U,
+                    sel_cnt, sel_pos, sel_w, k_max, d, r_out, (float*)r_lo);
 }
 
 // ---------------------------------------------------------------------------
@@ -331,41 +390,75 @@ cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFi
 // ---------------------------------------------------------------------------
 // Gate, gated residual and RMSNorm (Eq. hidden_correction):
 // g = sigma(a_g . w_g2 + b_g2), y = h + g c, h_hat = y / sqrt(mean(y^2) + eps) * gamma.
-// One CTA per row; `act` is [N, 2H] with a_f in columns 0..H-1 and a_g in H..2H-1.
+// One CTA per row; `act` is [N, 2H] with a_f in columns 0..H-1 and a_g in
+// H..2H-1.  Every operand of the row is requested before the first reduction.
 // ---------------------------------------------------------------------------
-constexpr int kFinThreads = 256;
+constexpr int kFinThreads = 512;
 
 template <class T>
 __global__ void __launch_bounds__(kFinThreads) finalize_kernel(
     const T* __restrict__ h, const float* __restrict__ c, const T* __restrict__ act, int H, int d,
     const T* __restrict__ w_g2, const T* __restrict__ b_g2, const T* __restrict__ rms_gamma,
     float eps, T* __restrict__ h_out, float* __restrict__ gate_out) {
+  constexpr int V = LnVec<T>::N;
+  constexpr int MV = LnVec<T>::MAX;
   __shared__ float scratch[32];
-  const int n = blockIdx.x;
+  const int n = blockIdx.x, tid = threadIdx.x;
+  const int nvec = d / V;
+  const T* hr = h + (long long)n * d;
+  const float* cr = c + (long long)n * d;
+  float hv[MV][V], cv[MV][V], gv[MV][V];
+#pragma unroll
+  for (int j = 0; j < MV; ++j) {
+    const int vi = tid + j * kFinThreads;
+    if (vi < nvec) {
+      ln_load<T>(hr + vi * V, hv[j]);
+      ln_load<T>(rms_gamma + vi * V, gv[j]);
+    }
+  }
+  pdl_wait();
+  pdl_trigger();
+#pragma unroll
+  for (int j = 0; j < MV; ++j) {
+    const int vi = tid + j * kFinThreads;
+    if (vi < nvec) {
+#pragma unroll
+      for (int i = 0; i < V; i += 4) {
+        const float4 c4 = *reinterpret_cast<const float4*>(cr + vi * V + i);
+        cv[j][i] = c4.x; cv[j][i + 1] = c4.y; cv[j][i + 2] = c4.z; cv[j][i + 3] = c4.w;
+      }
+    }
+  }
   const T* a_g = act + (long long)n * 2 * H + H;
   float part = 0.0f;
-  for (int j = threadIdx.x; j < H; j += kFinThreads) part = fmaf(to_f32(a_g[j]), to_f32(w_g2[j]), part);
+  for (int k = tid; k < H; k += kFinThreads) part = fmaf(to_f32(a_g[k]), to_f32(w_g2[k]), part);
   const float z = block_sum(part, scratch) + to_f32(b_g2[0]);
   const float g = sigmoidf_(z);
-  float y[kLnMaxPerThread];
   float ss = 0.0f;
 #pragma unroll
-  for (int j = 0; j < kLnMaxPerThread; ++j) {
-    const int i = threadIdx.x + j * kFinThreads;
-    y[j] = 0.0f;
-    if (i < d) {
-      y[j] = fmaf(g, c[(long long)n * d + i], to_f32(h[(long long)n * d + i]));
-      ss = fmaf(y[j], y[j], ss);
+  for (int j = 0; j < MV; ++j) {
+    if (tid + j * kFinThreads < nvec) {
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        hv[j][i] = fmaf(g, cv[j][i], hv[j][i]);          // y = h + g c
+        ss = fmaf(hv[j][i], hv[j][i], ss);
+      }
     }
   }
   const float tot = block_sum(ss, scratch);
   const float inv = 1.0f / sqrtf(tot / (float)d + eps);
+  T* o = h_out + (long long)n * d;
 #pragma unroll
-  for (int j = 0; j < kLnMaxPerThread; ++j) {
-    const int i = threadIdx.x + j * kFinThreads;
-    if (i < d) h_out[(long long)n * d + i] = from_f32<T>(y[j] * inv * to_f32(rms_gamma[i]));
+  for (int j = 0; j < MV; ++j) {
+    const int vi = tid + j * kFinThreads;
+    if (vi < nvec) {
+      T res[V];
+#pragma unroll
+      for (int i = 0; i < V; ++i) res[i] = from_f32<T>(hv[j][i] * inv * gv[j][i]);
+      *reinterpret_cast<uint4*>(o + vi * V) = *reinterpret_cast<const uint4*>(res);
+    }
   }
-  if (gate_out != nullptr && threadIdx.x == 0) gate_out[n] = g;
+  if (gate_out != nullptr && tid == 0) gate_out[n] = g;
 }
 
 cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,
@@ -374,16 +467,13 @@ cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void
   if (N == 0) return cudaSuccess;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
-    finalize_kernel<T><<<N, kFinThreads, 0, s>>>((const T*)h, c, (const T*)act, H, d,
-                                                 (const T*)w_g2, (const T*)b_g2,
-                                                 (const T*)rms_gamma, eps, (T*)h_out, gate_out);
-  } else {
-    finalize_kernel<float><<<N, kFinThreads, 0, s>>>((const float*)h, c, (const float*)act, H, d,
-                                                     (const float*)w_g2, (const float*)b_g2,
-                                                     (const float*)rms_gamma, eps, (float*)h_out,
-                                                     gate_out);
+    return launch_pdl(finalize_kernel<T>, dim3(N), dim3(kFinThreads), 0, s, (const T*)h, c,
+                      (const T*)act, H, d, (const T*)w_g2, (const T*)b_g2, (const T*)rms_gamma,
+                      eps, (T*)h_out, gate_out);
   }
-  return cudaGetLastError();
+  return launch_pdl(finalize_kernel<float>, dim3(N), dim3(kFinThreads), 0, s, (const float*)h, c,
+                    (const float*)act, H, d, (const float*)w_g2, (const float*)b_g2,
+                    (const float*)rms_gamma, eps, (float*)h_out, gate_out);
 }
 
 }  // namespace fovea

@@ -48,6 +48,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 
   const int n = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_wait();
+  pdl_trigger();
   const int b = seq_of_row(tab, n);
   const int M = tab.m[b];
   const int k_max = a.k_max;
@@ -262,8 +264,7 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
     configured = true;
   }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt};
-  select_kernel<<<N, kSelThreads, smem, s>>>(a, tab);
-  return cudaGetLastError();
+  return launch_pdl(select_kernel, dim3(N), dim3(kSelThreads), smem, s, a, tab);
 }
 
 }  // namespace fovea
