@@ -240,11 +240,15 @@ cudaError_t launch_compact(const uint8_t* mask, int B, int M_max, const int32_t*
 
 // ---------------------------------------------------------------------------
 // Readout r_n = sum_{t < K} alpha_t u_{pi(t)} (the alpha / r_n equation).
-// Grid (N, column chunks); each thread owns one 16-byte vector of columns
-// and walks the selected entries in pi order (fp32 accumulation, fixed
-// order).  The weights were renormalised over I_n by the select kernel.
+// Grid (N rows, column chunks of 64 x vector width); 8 warps per CTA split the
+// selected entries (warp w takes t = w, w + 8, ...), each lane owns one
+// 16-byte vector of columns and keeps several gathers in flight; the warps'
+// partial sums are combined in warp order (fixed order, fp32).  The weights
+// were renormalised over I_n by the select kernel.
 // ---------------------------------------------------------------------------
-constexpr int kReadoutThreads = 128;
+constexpr int kReadoutWarps = 8;
+constexpr int kReadoutThreads = 32 * kReadoutWarps;
+constexpr int kReadoutUnroll = 4;
 
 template <class T>
 struct Vec16;
@@ -276,46 +280,56 @@ __global__ void __launch_bounds__(kReadoutThreads) readout_kernel(
     const int32_t* __restrict__ sel_pos, const float* __restrict__ sel_w, int k_max, int d,
     float* __restrict__ r_out, T* __restrict__ r_lo) {
   constexpr int V = Vec16<T>::N;
+  __shared__ float part[kReadoutWarps][32 * V];
   const int n = blockIdx.x;
-  const int col = (blockIdx.y * kReadoutThreads + threadIdx.x) * V;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int col = (blockIdx.y * 32 + lane) * V;
   pdl_wait();
   pdl_trigger();
-  if (col >= d) return;
   const int K = sel_cnt[n];
   const int32_t* pos = sel_pos + (long long)n * k_max;
   const float* w = sel_w + (long long)n * k_max;
   float acc[V];
 #pragma unroll
   for (int i = 0; i < V; ++i) acc[i] = 0.0f;
-  int t = 0;
-  for (; t + 4 <= K; t += 4) {
-    float u0[V], u1[V], u2[V], u3[V];
-    load_vec<T>(U + (long long)pos[t] * d + col, u0);
-    load_vec<T>(U + (long long)pos[t + 1] * d + col, u1);
-    load_vec<T>(U + (long long)pos[t + 2] * d + col, u2);
-    load_vec<T>(U + (long long)pos[t + 3] * d + col, u3);
-    const float w0 = w[t], w1 = w[t + 1], w2 = w[t + 2], w3 = w[t + 3];
+  if (col < d) {
+    int t = warp;
+    for (; t + (kReadoutUnroll - 1) * kReadoutWarps < K; t += kReadoutUnroll * kReadoutWarps) {
+      float u[kReadoutUnroll][V];
+      float wt[kReadoutUnroll];
 #pragma unroll
-    for (int i = 0; i < V; ++i) {
-      acc[i] = fmaf(w0, u0[i], acc[i]);
-      acc[i] = fmaf(w1, u1[i], acc[i]);
-      acc[i] = fmaf(w2, u2[i], acc[i]);
-      acc[i] = fmaf(w3, u3[i], acc[i]);
+      for (int j = 0; j < kReadoutUnroll; ++j) {
+        const int tj = t + j * kReadoutWarps;
+        wt[j] = w[tj];
+        load_vec<T>(U + (long long)pos[tj] * d + col, u[j]);
+      }
+#pragma unroll
+      for (int j = 0; j < kReadoutUnroll; ++j)
+#pragma unroll
+        for (int i = 0; i < V; ++i) acc[i] = fmaf(wt[j], u[j][i], acc[i]);
+    }
+    for (; t < K; t += kReadoutWarps) {
+      float u[V];
+      load_vec<T>(U + (long long)pos[t] * d + col, u);
+      const float wt = w[t];
+#pragma unroll
+      for (int i = 0; i < V; ++i) acc[i] = fmaf(wt, u[i], acc[i]);
     }
   }
-  for (; t < K; ++t) {
-    float u0[V];
-    load_vec<T>(U + (long long)pos[t] * d + col, u0);
-    const float w0 = w[t];
 #pragma unroll
-    for (int i = 0; i < V; ++i) acc[i] = fmaf(w0, u0[i], acc[i]);
+  for (int i = 0; i < V; ++i) part[warp][lane * V + i] = acc[i];
+  __syncthreads();
+  // combine the warps' partial sums in warp order; thread i of the CTA owns
+  // element i of the chunk
+  for (int e = threadIdx.x; e < 32 * V; e += kReadoutThreads) {
+    const int c = blockIdx.y * 32 * V + e;
+    if (c >= d) continue;
+    float sum = 0.0f;
+#pragma unroll
+    for (int wi = 0; wi < kReadoutWarps; ++wi) sum += part[wi][e];
+    if (r_out != nullptr) r_out[(long long)n * d + c] = sum;
+    r_lo[(long long)n * d + c] = from_f32<T>(sum);
   }
-  if (r_out != nullptr) {
-#pragma unroll
-    for (int i = 0; i < V; ++i) r_out[(long long)n * d + col + i] = acc[i];
-  }
-#pragma unroll
-  for (int i = 0; i < V; ++i) r_lo[(long long)n * d + col + i] = from_f32<T>(acc[i]);
 }
 
 cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, const int32_t* sel_pos,
@@ -324,11 +338,11 @@ cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, con
   if (N == 0) return cudaSuccess;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
-    dim3 grid(N, (d / 8 + kReadoutThreads - 1) / kReadoutThreads);
+    dim3 grid(N, (d / 8 + 31) / 32);
     return launch_pdl(readout_kernel<T>, grid, dim3(kReadoutThreads), 0, s, (const T*)U, sel_cnt,
                       sel_pos, sel_w, k_max, d, r_out, (T*)r_lo);
   }
-  dim3 grid(N, (d / 4 + kReadoutThreads - 1) / kReadoutThreads);
+  dim3 grid(N, (d / 4 + 31) / 32);
   return launch_pdl(readout_kernel<float>, grid, dim3(kReadoutThreads), 0, s, (const float*)U,
                     sel_cnt, sel_pos, sel_w, k_max, d, r_out, (float*)r_lo);
 }

@@ -4,17 +4,22 @@
 // K = min(|V|, K_max, max(K_min, K_raw)), and the renormalised weights over
 // I_n = pi_n(1..K)).
 //
-// One CTA per draft state.  The row's scores are staged in shared memory; a
-// 4-pass 8-bit radix select finds the K_eff-th largest score key
+// One CTA per draft state.  The row's scores are staged in shared memory
+// while one pass forms the softmax statistics (running max and rescaled sum).
+// A 4-pass 8-bit radix select finds the K_eff-th largest score key
 // (K_eff = min(K_max, |V|)) without sorting the row; only the K_eff
-// candidates are bitonic-sorted by (score desc, position asc); an fp32
-// inclusive scan of exp(s - s_max) over them gives the cumulative mass, and
-// the first prefix reaching rho sets K.
+// candidates are put in order, by (score desc, position asc): each
+// candidate's rank is its count of larger candidates (one barrier) for
+// K_eff <= 256, a bitonic network above that.  An fp32 inclusive scan of
+// exp(s - s_max) over them gives the cumulative mass, and the first prefix
+// reaching rho sets K.
 #include "common.cuh"
 
 namespace fovea {
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 256;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kRankMax = 256;          // direct ranking up to this many candidates
 
 // Monotone map of a float to uint32 (larger float -> larger key); -0 is
 // mapped like +0 by the caller.
@@ -35,16 +40,29 @@ struct SelectArgs {
   int32_t* sel_cnt;    // [N]
 };
 
+// (max, sum of exp(x - max)) pairs combine as a softmax denominator.
+__device__ __forceinline__ void combine_ms(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s * expf(m - m2) + s2;
+    m = m2;
+  } else if (m2 != -INFINITY) {
+    s = s + s2 * expf(m2 - m);
+  }
+}
+
 __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectArgs a,
-                                                                 const __grid_constant__ SeqTable tab) {
+                                                             const __grid_constant__ SeqTable tab) {
   extern __shared__ float s_sc[];                            // [M] scores of this row
   __shared__ unsigned long long cand[FOVEA_MAX_K];           // (key << 32) | ~position
+  __shared__ unsigned long long sorted[kRankMax];
   __shared__ float cum[FOVEA_MAX_K];                         // inclusive scan of exp(s - s_max)
   __shared__ unsigned int hist[256];
-  __shared__ float scratch[32];
-  __shared__ int warp_tot[kSelThreads / 32];
+  __shared__ float red_m[kSelWarps], red_s[kSelWarps];
+  __shared__ float warp_tot_f[kSelWarps];
+  __shared__ int warp_tot[kSelWarps];
   __shared__ unsigned int sh_digit, sh_above;
   __shared__ int sh_cnt_gt, sh_first;
+  __shared__ float sh_max, sh_sum;
 
   const int n = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -67,18 +85,34 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   const int K_eff = min(k_max, M);
   const float* src = a.scores + tab.score_off[b] + (long long)(n - tab.row_start[b]) * M;
 
-  // ---- stage scores, global max and softmax denominator --------------------
-  float lmax = -INFINITY;
+  // ---- stage scores; softmax statistics in the same pass --------------------
+  float lmax = -INFINITY, lsum = 0.0f;
   for (int i = tid; i < M; i += kSelThreads) {
     float v = src[i];
     if (v == 0.0f) v = 0.0f;              // -0 -> +0 so equal scores get equal keys
     s_sc[i] = v;
-    lmax = fmaxf(lmax, v);
+    combine_ms(lmax, lsum, v, 1.0f);
   }
-  const float smax = block_max(lmax, scratch);
-  float lsum = 0.0f;
-  for (int i = tid; i < M; i += kSelThreads) lsum += expf(s_sc[i] - smax);
-  const float sumexp = block_sum(lsum, scratch);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, lmax, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, lsum, o);
+    combine_ms(lmax, lsum, m2, s2);
+  }
+  if (lane == 0) {
+    red_m[warp] = lmax;
+    red_s[warp] = lsum;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float m = red_m[0], sm = red_s[0];
+    for (int w = 1; w < kSelWarps; ++w) combine_ms(m, sm, red_m[w], red_s[w]);
+    sh_max = m;
+    sh_sum = sm;
+  }
+  __syncthreads();
+  const float smax = sh_max;
+  const float sumexp = sh_sum;
 
   // ---- radix select of the K_eff-th largest key ----------------------------
   uint32_t prefix = 0, pmask = 0;
@@ -133,7 +167,6 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     prefix |= sh_digit << shift;
     pmask |= 255u << shift;
     krem -= (int)sh_above;
-    __syncthreads();
   }
   const uint32_t T = prefix;              // K_eff-th largest key; take krem entries equal to T
 
@@ -177,51 +210,72 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
       }
     }
   }
-  int P = 1;
-  while (P < K_eff) P <<= 1;
-  for (int t = K_eff + tid; t < P; t += kSelThreads) cand[t] = 0ull;
   __syncthreads();
 
-  // ---- bitonic sort of the candidates, descending --------------------------
-  for (int k = 2; k <= P; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < P; i += kSelThreads) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const unsigned long long x = cand[i], y = cand[ixj];
-          const bool desc = (i & k) == 0;
-          if (desc ? (x < y) : (x > y)) {
-            cand[i] = y;
-            cand[ixj] = x;
+  // ---- order the candidates, descending ------------------------------------
+  const unsigned long long* ordered;
+  if (K_eff <= kRankMax) {
+    // keys are distinct (the position is part of the key): rank = #larger
+    for (int c = tid; c < K_eff; c += kSelThreads) {
+      const unsigned long long me = cand[c];
+      int r = 0;
+      for (int j = 0; j < K_eff; ++j) r += cand[j] > me;
+      sorted[r] = me;
+    }
+    ordered = sorted;
+  } else {
+    int P = 1;
+    while (P < K_eff) P <<= 1;
+    for (int t = K_eff + tid; t < P; t += kSelThreads) cand[t] = 0ull;
+    __syncthreads();
+    for (int k = 2; k <= P; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        for (int i = tid; i < P; i += kSelThreads) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long x = cand[i], y = cand[ixj];
+            const bool desc = (i & k) == 0;
+            if (desc ? (x < y) : (x > y)) {
+              cand[i] = y;
+              cand[ixj] = x;
+            }
           }
         }
+        __syncthreads();
       }
-      __syncthreads();
     }
+    ordered = cand;
   }
+  __syncthreads();
 
-  // ---- cumulative mass over the sorted candidates --------------------------
-  // each thread scans a contiguous pair (2 * 512 >= FOVEA_MAX_K)
+  // ---- cumulative mass over the ordered candidates -------------------------
+  // thread tid scans the contiguous quad 4 tid .. 4 tid + 3 (4 x 256 >= FOVEA_MAX_K)
   {
-    const int t0 = 2 * tid, t1 = 2 * tid + 1;
-    float e0 = 0.0f, e1 = 0.0f;
-    if (t0 < K_eff) e0 = expf(s_sc[0xFFFFFFFFu - (uint32_t)(cand[t0] & 0xFFFFFFFFull)] - smax);
-    if (t1 < K_eff) e1 = expf(s_sc[0xFFFFFFFFu - (uint32_t)(cand[t1] & 0xFFFFFFFFull)] - smax);
-    const float pair = e0 + e1;
-    float incl = pair;
+    float e[4];
+    float run = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int t = 4 * tid + q;
+      e[q] = t < K_eff ? expf(s_sc[0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull)] - smax)
+                       : 0.0f;
+      run += e[q];
+    }
+    float incl = run;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const float t = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += t;
     }
+    if (lane == 31) warp_tot_f[warp] = incl;
     __syncthreads();
-    if (lane == 31) scratch[warp] = incl;
-    __syncthreads();
-    float base = 0.0f;
-    for (int w = 0; w < warp; ++w) base += scratch[w];
-    const float before = base + incl - pair;
-    if (t0 < K_eff) cum[t0] = before + e0;
-    if (t1 < K_eff) cum[t1] = before + e0 + e1;
+    float before = incl - run;
+    for (int w = 0; w < warp; ++w) before += warp_tot_f[w];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int t = 4 * tid + q;
+      before += e[q];
+      if (t < K_eff) cum[t] = before;
+    }
   }
   if (tid == 0) sh_first = K_eff;          // K_eff = "not reached within the candidates"
   __syncthreads();
@@ -234,7 +288,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 
   for (int t = tid; t < k_max; t += kSelThreads) {
     if (t < K) {
-      const int pos = (int)(0xFFFFFFFFu - (uint32_t)(cand[t] & 0xFFFFFFFFull));
+      const int pos = (int)(0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull));
       const float e = expf(s_sc[pos] - smax);
       const int row = tab.key_off[b] + pos;
       a.sel_pos[out_row + t] = row;
