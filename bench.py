@@ -303,7 +303,7 @@ def main():
     indices = torch.empty((N, K), dtype=torch.int32, device=dev)
     offs_c = fovea._offsets(w.row_offsets)
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.int32, device=dev)
+    flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.float32, device=dev)
     h_in = torch.empty_like(h)          # the step reads its inputs from here
     depth_in = torch.empty_like(depth)
     h_in.copy_(h)
