@@ -237,9 +237,30 @@ FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(const fovea_params* p, const 
                                                    int32_t* indices, float* readout, float* gate,
                                                    void* stream);
 
+/*
+ * Implementation of the draft step (process-wide; the paper has no
+ * counterpart, both compute the same operator):
+ *   FOVEA_PATH_AUTO     the persistent step kernel where the call fits it
+ *                       (bf16, <= 64 sequences, <= 3072 valid entries per
+ *                       sequence), else one kernel per stage (the default)
+ *   FOVEA_PATH_FUSED    the persistent step kernel only; a call it does not
+ *                       cover returns FOVEA_ERR_UNSUPPORTED
+ *   FOVEA_PATH_KERNELS  one kernel per stage of the step
+ * The persistent kernel is one cooperative launch of one CTA per SM whose
+ * phases meet at device-wide barriers kept in the workspace header; it needs
+ * the whole GPU, so a concurrent kernel on another stream delays its start.
+ * fovea_step_path(path) selects and returns the previous setting; any other
+ * value leaves the setting unchanged and returns it.
+ */
+#define FOVEA_PATH_AUTO 0
+#define FOVEA_PATH_FUSED 1
+#define FOVEA_PATH_KERNELS 2
+FOVEA_API int fovea_step_path(int path);
+
 /* Synchronise `stream`, read and clear the workspace's sticky error word.
  * Returns FOVEA_OK, FOVEA_ERR_INVALID_ARG (a depth outside [0, D] was seen)
- * or FOVEA_ERR_TIMEOUT (a bounded device wait gave up), or FOVEA_ERR_CUDA. */
+ * or FOVEA_ERR_TIMEOUT (a bounded device wait gave up; the whole workspace
+ * header is then cleared, as fovea_workspace_init does), or FOVEA_ERR_CUDA. */
 FOVEA_API fovea_status fovea_sync_errors(void* workspace, void* stream);
 
 /* Message of the last non-OK status returned on this thread ("" if none). */

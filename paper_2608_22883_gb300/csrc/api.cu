@@ -9,7 +9,10 @@
 #include <string>
 #include <vector>
 
+#include <atomic>
+
 #include "common.cuh"
+#include "step_fused.h"
 
 using namespace fovea;
 
@@ -43,6 +46,9 @@ static fovea_status cuda_fail(cudaError_t e, const char* where) {
     cudaError_t e_ = (call);                      \
     if (e_ != cudaSuccess) return cuda_fail(e_, where); \
   } while (0)
+
+// Which implementation of the draft step fovea_retrieve_fuse runs.
+static std::atomic<int> g_step_path{FOVEA_PATH_AUTO};
 
 // ---------------------------------------------------------------------------
 // Per-launch timing (CUDA events on the launching stream)
@@ -403,6 +409,9 @@ namespace {
 // tile counters (pairs of ints).  Zero when the workspace is initialised; the
 // kernels leave the counters at zero after every launch.
 constexpr size_t kWsHeaderBytes = 16384;
+// Words of the persistent step kernel inside the header's first 256 bytes
+// (bytes 128..175): grid-barrier arrival counters, exit counter, abort word.
+constexpr size_t kWsSyncOffset = 128;
 constexpr long long kTileSyncTiles = (kWsHeaderBytes - 256) / 8;
 
 struct WsLayout {
@@ -428,6 +437,22 @@ long long step_partial_floats(int dtype, int d, int H, int N, int ngroups, int m
   need = std::max(need, plan(kEpiBiasF32, H, 0x7fffffff, 1, d, N));
   delete a;
   return need;
+}
+
+// The persistent-kernel plan of a call (false: the call's shape is outside it).
+bool plan_fused_call(const fovea_params* p, const fovea_memory* mem, const int32_t* row_offsets,
+                     int k_max, FusedPlan* plan) {
+  if (g_step_path.load() == FOVEA_PATH_KERNELS) return false;
+  FusedShape sh;
+  sh.bf16 = p->dtype == FOVEA_BF16;
+  sh.N = row_offsets[mem->B];
+  sh.d = p->d_model;
+  sh.H = p->mlp_hidden;
+  sh.B = mem->B;
+  sh.k_max = k_max;
+  sh.row_offsets = row_offsets;
+  sh.m = mem->counts.data();
+  return fused_plan(sh, plan);
 }
 
 WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems,
@@ -498,7 +523,9 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
   int N, mm, mr, ng;
   long long se;
   if ((st = check_rows(mem, row_offsets, &N, &se, &mm, &mr, &ng)) != FOVEA_OK) return st;
-  const long long pf = step_partial_floats(p->dtype, p->d_model, p->mlp_hidden, N, ng, mm, mr);
+  long long pf = step_partial_floats(p->dtype, p->d_model, p->mlp_hidden, N, ng, mm, mr);
+  static thread_local FusedPlan fp;
+  if (N > 0 && plan_fused_call(p, mem, row_offsets, k_max, &fp)) pf = std::max(pf, fp.partial_floats);
   *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se, pf).total;
   return FOVEA_OK;
 }
@@ -523,8 +550,13 @@ FOVEA_API fovea_status fovea_sync_errors(void* workspace, void* stream) {
   FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
   FOVEA_CUDA(cudaMemsetAsync(workspace, 0, sizeof(int), s), "cudaMemsetAsync");
   FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-  if (herr & kErrTimeout)
+  if (herr & kErrTimeout) {
+    // the kernels that gave up may have left barrier counters or the abort
+    // word set: start the next call from a clean header
+    FOVEA_CUDA(cudaMemsetAsync(workspace, 0, kWsHeaderBytes, s), "cudaMemsetAsync");
+    FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
     return fail(FOVEA_ERR_TIMEOUT, "a bounded device wait gave up (error word 0x%x)", herr);
+  }
   if (herr & kErrDepth)
     return fail(FOVEA_ERR_INVALID_ARG, "a draft state had a depth outside [0, max_depth]");
   return FOVEA_OK;
@@ -564,8 +596,15 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   const int d = p->d_model, H = p->mlp_hidden, dt = p->dtype;
-  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems,
-                               step_partial_floats(dt, d, H, N, ngroups, max_m, max_r));
+  static thread_local FusedPlan fplan;
+  const bool use_fused = plan_fused_call(p, mem, row_offsets, k_max, &fplan);
+  if (!use_fused && g_step_path.load() == FOVEA_PATH_FUSED)
+    return fail(FOVEA_ERR_UNSUPPORTED,
+                "the persistent step kernel does not cover this call (bf16, <= %d sequences, "
+                "<= 3072 entries per sequence are required)", fused::kMaxSeq);
+  long long pfloats = step_partial_floats(dt, d, H, N, ngroups, max_m, max_r);
+  if (use_fused) pfloats = std::max(pfloats, fplan.partial_floats);
+  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems, pfloats);
   if (workspace_bytes < L.total)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);
 
@@ -583,6 +622,45 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   float* cbuf = reinterpret_cast<float*>(ws + L.c);
   float* partials = reinterpret_cast<float*>(ws + L.partials);
   int* tile_sync = reinterpret_cast<int*>(ws + L.err + 256);
+
+  if (use_fused) {
+    // the whole step as one persistent cooperative kernel (step_fused.cu)
+    static thread_local std::vector<int32_t> key_off;
+    key_off.resize(mem->B);
+    long long m_sel = 0;
+    for (int b = 0; b < mem->B; ++b) {
+      key_off[b] = (int32_t)mem->offsets[b];
+      const long long R = row_offsets[b + 1] - row_offsets[b];
+      m_sel += std::min<long long>(mem->counts[b], R * k_max);
+    }
+    FusedLaunch fl;
+    memset(&fl, 0, sizeof(fl));
+    fl.N = N; fl.d = d; fl.H = H; fl.B = mem->B; fl.k_max = k_max; fl.k_min = k_min;
+    fl.max_depth = p->max_depth; fl.rho = rho; fl.ln_eps = p->ln_eps; fl.rms_eps = p->rms_eps;
+    fl.row_offsets = row_offsets; fl.key_off = key_off.data(); fl.m = mem->counts.data();
+    fl.total_keys = mem->total;
+    fl.prefetch_values = 2 * m_sel >= mem->total;     // most value rows will be read
+    fl.h = h; fl.ln_gamma = p->ln_h_gamma; fl.ln_beta = p->ln_h_beta; fl.E = p->E_dep;
+    fl.W_Q = p->W_Q; fl.keys = mem->keys; fl.values = mem->values;
+    fl.W_f1 = p->W_f1; fl.W_g1 = p->W_g1; fl.W_f2 = p->W_f2;
+    fl.b_f1 = p->b_f1; fl.b_g1 = p->b_g1; fl.b_f2 = p->b_f2; fl.w_g2 = p->w_g2; fl.b_g2 = p->b_g2;
+    fl.rms_gamma = p->rms_gamma;
+    fl.depth = depth; fl.row_scale = row_scale; fl.orig_index = mem->orig_index;
+    fl.x = ws + L.xh; fl.q_hi = ws + L.q; fl.q_lo = ws + L.q + (size_t)N * d * 2;
+    fl.r = ws + L.r_lo; fl.act = ws + L.act;
+    fl.partials = reinterpret_cast<float*>(ws + L.partials);
+    fl.sel_pos = reinterpret_cast<int32_t*>(ws + L.sel_pos);
+    fl.sel_w = reinterpret_cast<float*>(ws + L.sel_w);
+    fl.sel_cnt = reinterpret_cast<int32_t*>(ws + L.sel_cnt);
+    fl.err = reinterpret_cast<int*>(ws + L.err);
+    fl.sync = reinterpret_cast<int*>(ws + L.err + kWsSyncOffset);
+    fl.h_out = h_out; fl.counts = counts; fl.indices = indices; fl.readout = readout; fl.gate = gate;
+    cudaError_t e;
+    { KernelTimer t("fused_step", s);
+      e = launch_fused_step(fplan, fl, s); }
+    if (e != cudaSuccess) return cuda_fail(e, "fused_step");
+    return FOVEA_OK;
+  }
 
   // Per-sequence table (kernel parameter).
   static thread_local SeqTable tab;
@@ -709,6 +787,12 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                         h_out, gate, s); }
   if (e != cudaSuccess) return cuda_fail(e, "finalize");
   return FOVEA_OK;
+}
+
+FOVEA_API int fovea_step_path(int path) {
+  if (path == FOVEA_PATH_AUTO || path == FOVEA_PATH_FUSED || path == FOVEA_PATH_KERNELS)
+    return g_step_path.exchange(path);
+  return g_step_path.load();
 }
 
 FOVEA_API fovea_status fovea_timing_enable(int enable) {

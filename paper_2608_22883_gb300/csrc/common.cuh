@@ -210,6 +210,10 @@ struct GemmPlan {
   long long tiles;       // output tiles of a split-K launch (counter pairs it needs)
 };
 GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n);
+// Tensor map of a row-major [rows, cols] bf16 matrix (row stride ld
+// elements), 128-byte swizzle, box = 64 columns x box_rows rows.
+bool encode_bf16_map(CUtensorMap* m, const void* base, long long rows, long long cols,
+                     long long ld, int box_rows);
 cudaError_t launch_gemm_tc(int epi, const GemmArgs& a, const TmaOperand& A0, const TmaOperand& A1,
                            const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
                            cudaStream_t s);

@@ -1,8 +1,7 @@
 // Row-wise kernels of the FOVEA path: LayerNorm (+ depth embedding), mask
 // compaction, the gather-and-weighted-sum readout, and the gate + gated
 // residual + RMSNorm finalisation.
-#include "common.cuh"
-#include "dfloat.cuh"
+#include "rowmath.cuh"
 
 namespace fovea {
 
@@ -27,40 +26,6 @@ template <> struct LnVec<__nv_bfloat16> {
 template <> struct LnVec<float> {
   static constexpr int N = 4, MAX = FOVEA_MAX_D / 4 / kLnThreads;
 };
-
-template <class T>
-__device__ __forceinline__ void ln_load(const T* p, float (&v)[LnVec<T>::N]);
-template <>
-__device__ __forceinline__ void ln_load<__nv_bfloat16>(const __nv_bfloat16* p, float (&v)[8]) {
-  const uint4 raw = *reinterpret_cast<const uint4*>(p);
-  const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 f = __bfloat1622float2(h2[i]);
-    v[2 * i] = f.x;
-    v[2 * i + 1] = f.y;
-  }
-}
-template <>
-__device__ __forceinline__ void ln_load<float>(const float* p, float (&v)[4]) {
-  const float4 raw = *reinterpret_cast<const float4*>(p);
-  v[0] = raw.x; v[1] = raw.y; v[2] = raw.z; v[3] = raw.w;
-}
-
-template <class T> __device__ __forceinline__ T df_store(dfloat y);
-template <> __device__ __forceinline__ float df_store<float>(dfloat y) { return y.hi; }
-template <> __device__ __forceinline__ __nv_bfloat16 df_store<__nv_bfloat16>(dfloat y) {
-  return df_to_bf16(y);
-}
-
-__device__ __forceinline__ dfloat warp_sum_df(dfloat v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const dfloat t = {__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)};
-    v = df_add(v, t);
-  }
-  return v;
-}
 
 template <class T>
 __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(

@@ -1,0 +1,314 @@
+// Cumulative-mass selection of one draft state by a group of 256 threads
+// (retrieval section of the paper: the global softmax alpha-tilde over the
+// valid entries, the descending order pi_n, the cardinality
+// K_raw = min{k : sum_{t<=k} alpha-tilde_{pi(t)} >= rho}, its clamp
+// K = min(|V|, K_max, max(K_min, K_raw)), and the renormalised weights over
+// I_n = pi_n(1..K)).
+//
+// The caller stages the row's scores in shared memory (-0 mapped to +0) and
+// forms each thread's running softmax statistics; select_stats combines them
+// over the group and select_finish does the rest.  A 4-pass 8-bit radix
+// select finds the K_eff-th largest score key (K_eff = min(K_max, |V|))
+// without sorting the row; only the K_eff candidates are put in order, by
+// (score desc, position asc): each candidate's rank is its count of larger
+// candidates for K_eff <= 256, a bitonic network above that.  An fp32
+// inclusive scan of exp(s - s_max) over them gives the cumulative mass, and
+// the first prefix reaching rho sets K.
+//
+// Used by the standalone select kernel (a CTA of 256 threads, __syncthreads)
+// and by the persistent step kernel (its 256 worker threads, a named
+// barrier): `sync` is the group barrier, `tid` the thread's index in the
+// group, and the group's warps are whole hardware warps.
+#pragma once
+#include "common.cuh"
+
+namespace fovea {
+
+constexpr int kSelThreads = 256;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kRankMax = 256;          // direct ranking up to this many candidates
+
+// Monotone map of a float to uint32 (larger float -> larger key); -0 is
+// mapped like +0 by the caller.
+__device__ __forceinline__ uint32_t ord_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+struct SelectArgs {
+  const float* scores;
+  const int32_t* orig_index;
+  float rho;
+  int k_min, k_max;
+  int32_t* counts;     // [N] or null
+  int32_t* indices;    // [N, k_max] or null
+  int32_t* sel_pos;    // [N, k_max] compacted memory row of each selected entry
+  float* sel_w;        // [N, k_max] renormalised weight alpha
+  int32_t* sel_cnt;    // [N]
+};
+
+struct SelectSmem {
+  unsigned long long cand[FOVEA_MAX_K];      // (key << 32) | ~position
+  unsigned long long sorted[kRankMax];
+  float cum[FOVEA_MAX_K];                    // inclusive scan of exp(s - s_max)
+  unsigned int hist[256];
+  float red_m[kSelWarps], red_s[kSelWarps];
+  float warp_tot_f[kSelWarps];
+  int warp_tot[kSelWarps];
+  unsigned int sh_digit, sh_above;
+  int sh_cnt_gt, sh_first;
+  float sh_max, sh_sum;
+};
+
+// (max, sum of exp(x - max)) pairs combine as a softmax denominator.
+__device__ __forceinline__ void combine_ms(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s * expf(m - m2) + s2;
+    m = m2;
+  } else if (m2 != -INFINITY) {
+    s = s + s2 * expf(m2 - m);
+  }
+}
+
+// Group-wide combination of the threads' (max, sum) pairs: warps first, then
+// warp 0's lane 0 folds the warps in order.  Every thread returns the result.
+template <class Sync>
+__device__ __forceinline__ void select_stats(float lmax, float lsum, SelectSmem& sm, int tid,
+                                             Sync sync, float& smax, float& sumexp) {
+  const int lane = tid & 31, warp = tid >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, lmax, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, lsum, o);
+    combine_ms(lmax, lsum, m2, s2);
+  }
+  if (lane == 0) {
+    sm.red_m[warp] = lmax;
+    sm.red_s[warp] = lsum;
+  }
+  sync();
+  if (tid == 0) {
+    float m = sm.red_m[0], s = sm.red_s[0];
+    for (int w = 1; w < kSelWarps; ++w) combine_ms(m, s, sm.red_m[w], sm.red_s[w]);
+    sm.sh_max = m;
+    sm.sh_sum = s;
+  }
+  sync();
+  smax = sm.sh_max;
+  sumexp = sm.sh_sum;
+}
+
+// Radix select, candidate ordering, mass scan and the outputs of draft state
+// n, whose M (>= 1) scores are staged in s_sc.  key_off is the compacted row
+// of the sequence's first memory entry.
+template <class Sync>
+__device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, const float* s_sc,
+                              float smax, float sumexp, SelectSmem& sm, int tid, Sync sync) {
+  const int lane = tid & 31, warp = tid >> 5;
+  const int k_max = a.k_max;
+  const long long out_row = (long long)n * k_max;
+  const int K_eff = min(k_max, M);
+
+  // ---- radix select of the K_eff-th largest key ----------------------------
+  uint32_t prefix = 0, pmask = 0;
+  int krem = K_eff;                       // entries still to take at the current prefix
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += kSelThreads) sm.hist[i] = 0;
+    sync();
+    // warp-aggregated histogram: lanes with the same digit add once
+    for (int base = 0; base < M; base += kSelThreads) {
+      const int i = base + tid;
+      uint32_t bin = 0xFFFFFFFFu;
+      if (i < M) {
+        const uint32_t k = ord_key(s_sc[i]);
+        if ((k & pmask) == prefix) bin = (k >> shift) & 255u;
+      }
+      const unsigned int peers = __match_any_sync(0xffffffffu, bin);
+      if (bin != 0xFFFFFFFFu && lane == __ffs(peers) - 1)
+        atomicAdd(&sm.hist[bin], (unsigned)__popc(peers));
+    }
+    sync();
+    if (warp == 0) {
+      // lane l owns bins 255-8l .. 248-8l (lane 0 the largest digits)
+      unsigned int cnt[8], lsum_bins = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        cnt[j] = sm.hist[255 - 8 * lane - j];
+        lsum_bins += cnt[j];
+      }
+      unsigned int incl = lsum_bins;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      const unsigned int ballot = __ballot_sync(0xffffffffu, incl >= (unsigned)krem);
+      const int L = __ffs(ballot) - 1;    // exists: the prefix class holds >= krem entries
+      if (lane == L) {
+        unsigned int running = incl - lsum_bins;
+        unsigned int digit = 0, above = running;
+        for (int j = 0; j < 8; ++j) {
+          if (running + cnt[j] >= (unsigned)krem) {
+            digit = 255 - 8 * lane - j;
+            above = running;
+            break;
+          }
+          running += cnt[j];
+        }
+        sm.sh_digit = digit;
+        sm.sh_above = above;
+      }
+    }
+    sync();
+    prefix |= sm.sh_digit << shift;
+    pmask |= 255u << shift;
+    krem -= (int)sm.sh_above;
+  }
+  const uint32_t T = prefix;              // K_eff-th largest key; take krem entries equal to T
+
+  // ---- collect the K_eff candidates ----------------------------------------
+  if (tid == 0) sm.sh_cnt_gt = 0;
+  sync();
+  for (int base = 0; base < M; base += kSelThreads) {
+    const int i = base + tid;
+    uint32_t k = 0;
+    const bool take = i < M && (k = ord_key(s_sc[i])) > T;
+    const unsigned int bal = __ballot_sync(0xffffffffu, take);
+    int slot0 = 0;
+    if (lane == 0 && bal) slot0 = atomicAdd(&sm.sh_cnt_gt, __popc(bal));
+    slot0 = __shfl_sync(0xffffffffu, slot0, 0);
+    if (take) {
+      const int slot = slot0 + __popc(bal & ((1u << lane) - 1u));
+      sm.cand[slot] = ((unsigned long long)k << 32) | (0xFFFFFFFFu - (uint32_t)i);
+    }
+  }
+  const int c_gt = K_eff - krem;
+  {
+    // entries equal to T: the krem with the smallest positions (ordered scan)
+    const int chunk = (M + kSelThreads - 1) / kSelThreads;
+    const int beg = min(M, tid * chunk), end = min(M, beg + chunk);
+    int c = 0;
+    for (int i = beg; i < end; ++i) c += ord_key(s_sc[i]) == T;
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) sm.warp_tot[warp] = incl;
+    sync();
+    int rank = incl - c;
+    for (int w = 0; w < warp; ++w) rank += sm.warp_tot[w];
+    for (int i = beg; i < end && rank < krem; ++i) {
+      if (ord_key(s_sc[i]) == T) {
+        sm.cand[c_gt + rank] = ((unsigned long long)T << 32) | (0xFFFFFFFFu - (uint32_t)i);
+        ++rank;
+      }
+    }
+  }
+  sync();
+
+  // ---- order the candidates, descending ------------------------------------
+  const unsigned long long* ordered;
+  if (K_eff <= kRankMax) {
+    // keys are distinct (the position is part of the key): rank = #larger
+    for (int c = tid; c < K_eff; c += kSelThreads) {
+      const unsigned long long me = sm.cand[c];
+      int r = 0;
+      for (int j = 0; j < K_eff; ++j) r += sm.cand[j] > me;
+      sm.sorted[r] = me;
+    }
+    ordered = sm.sorted;
+  } else {
+    int P = 1;
+    while (P < K_eff) P <<= 1;
+    for (int t = K_eff + tid; t < P; t += kSelThreads) sm.cand[t] = 0ull;
+    sync();
+    for (int k = 2; k <= P; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        for (int i = tid; i < P; i += kSelThreads) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long x = sm.cand[i], y = sm.cand[ixj];
+            const bool desc = (i & k) == 0;
+            if (desc ? (x < y) : (x > y)) {
+              sm.cand[i] = y;
+              sm.cand[ixj] = x;
+            }
+          }
+        }
+        sync();
+      }
+    }
+    ordered = sm.cand;
+  }
+  sync();
+
+  // ---- cumulative mass over the ordered candidates -------------------------
+  // thread tid scans the contiguous quad 4 tid .. 4 tid + 3 (4 x 256 >= FOVEA_MAX_K)
+  {
+    float e[4];
+    float run = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int t = 4 * tid + q;
+      e[q] = t < K_eff ? expf(s_sc[0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull)] - smax)
+                       : 0.0f;
+      run += e[q];
+    }
+    float incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) sm.warp_tot_f[warp] = incl;
+    sync();
+    float before = incl - run;
+    for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int t = 4 * tid + q;
+      before += e[q];
+      if (t < K_eff) sm.cum[t] = before;
+    }
+  }
+  if (tid == 0) sm.sh_first = K_eff;       // K_eff = "not reached within the candidates"
+  sync();
+  for (int t = tid; t < K_eff; t += kSelThreads)
+    if (sm.cum[t] / sumexp >= a.rho) atomicMin(&sm.sh_first, t);
+  sync();
+  const int first = sm.sh_first;
+  const int K = first < K_eff ? min(K_eff, max(a.k_min, first + 1)) : K_eff;
+  const float denom = sm.cum[K - 1];       // sum over I_n of exp(s - s_max)
+
+  for (int t = tid; t < k_max; t += kSelThreads) {
+    if (t < K) {
+      const int pos = (int)(0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull));
+      const float e = expf(s_sc[pos] - smax);
+      const int row = key_off + pos;
+      a.sel_pos[out_row + t] = row;
+      a.sel_w[out_row + t] = e / denom;
+      if (a.indices) a.indices[out_row + t] = a.orig_index[row];
+    } else if (a.indices) {
+      a.indices[out_row + t] = -1;
+    }
+  }
+  if (tid == 0) {
+    a.sel_cnt[n] = K;
+    if (a.counts) a.counts[n] = K;
+  }
+}
+
+// Outputs of a draft state whose sequence has no valid entry: K = 0.
+__device__ __forceinline__ void select_empty(const SelectArgs& a, int n, int tid) {
+  const long long out_row = (long long)n * a.k_max;
+  for (int t = tid; t < a.k_max; t += kSelThreads)
+    if (a.indices) a.indices[out_row + t] = -1;
+  if (tid == 0) {
+    a.sel_cnt[n] = 0;
+    if (a.counts) a.counts[n] = 0;
+  }
+}
+
+}  // namespace fovea

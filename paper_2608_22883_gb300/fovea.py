@@ -35,9 +35,10 @@ EXPORTS = (
     "fovea_build_memory", "fovea_memory_destroy", "fovea_memory_info", "fovea_memory_tensors",
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
-    "fovea_retrieve_fuse_noalloc",
+    "fovea_retrieve_fuse_noalloc", "fovea_step_path",
 )
 NOALLOC_WORKSPACE_BYTES = 32 << 20
+PATH_AUTO, PATH_FUSED, PATH_KERNELS = 0, 1, 2
 
 
 class FoveaError(RuntimeError):
@@ -90,6 +91,8 @@ def lib() -> ctypes.CDLL:
                                         ctypes.POINTER(ctypes.c_int), ctypes.c_int]
         L.fovea_timing_read.restype = ctypes.c_int
         L.fovea_version.restype = ctypes.c_int
+        L.fovea_step_path.argtypes = [ctypes.c_int]
+        L.fovea_step_path.restype = ctypes.c_int
         for name in ("fovea_build_memory", "fovea_memory_info", "fovea_memory_tensors",
                      "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse",
                      "fovea_sync_errors", "fovea_timing_enable"):
@@ -284,6 +287,13 @@ def retrieve_fuse_noalloc(params: Params, memory: Memory, h: torch.Tensor, depth
 
 def sync_errors(workspace: torch.Tensor, stream=None) -> None:
     _check(lib().fovea_sync_errors(_ptr(workspace), _stream(stream)))
+
+
+def step_path(path: Optional[int] = None) -> int:
+    """Select the draft-step implementation (PATH_AUTO, PATH_FUSED or
+    PATH_KERNELS) and return the previous one; with no argument, return the
+    current one."""
+    return int(lib().fovea_step_path(-1 if path is None else int(path)))
 
 
 def timing_enable(on: bool = True) -> None:

@@ -5,6 +5,10 @@ entry memories, the selection clamps (k_max = 1, k_max > |V|, the paper's
 rho = 0.8 / K_min = 32 / K_max = 256, fixed top-16, dense), per-row
 temperatures, clustered keys and the fp32 path.  The five named workloads run
 at full size (the long-memory one on sampled rows and steps).
+
+Every parity test runs on both implementations of the draft step: "auto"
+(the persistent step kernel wherever a call fits it, which covers every bf16
+case here except the long-memory one) and "kernels" (one kernel per stage).
 """
 
 import dataclasses
@@ -26,6 +30,16 @@ def fovea():
     from paper_2608_22883_gb300 import fovea as f
     f.lib()          # raises if the library was not built: no fallback
     return f
+
+
+PATHS = {"auto": 0, "kernels": 2}
+
+
+@pytest.fixture(params=sorted(PATHS))
+def path(request, fovea):
+    prev = fovea.step_path(PATHS[request.param])
+    yield request.param
+    fovea.step_path(prev)
 
 
 SMALL = {
@@ -56,7 +70,7 @@ def small_workload(name):
 
 
 @pytest.mark.parametrize("name", sorted(SMALL))
-def test_small_parity(fovea, name):
+def test_small_parity(fovea, path, name):
     w = small_workload(name)
     s = store(w)
     gpu = run_gpu(s, fovea)
@@ -92,7 +106,31 @@ def test_memory_build_matches_oracle(fovea, name):
     mem.destroy()
 
 
-def test_zero_gate_returns_rmsnorm_of_h(fovea):
+def test_paths_are_taken(fovea):
+    """AUTO runs the persistent step kernel for a bf16 call and the per-stage
+    kernels for an fp32 one; FUSED refuses a call outside its coverage."""
+    prev = fovea.step_path(fovea.PATH_AUTO)
+    try:
+        for name, want in (("bf16-ragged", {"fused_step"}),
+                           ("fp32-ragged", {"ln_query", "query_proj", "select", "finalize"})):
+            s = store(small_workload(name))
+            fovea.timing_enable(True)
+            run_gpu(s, fovea)
+            names = set(fovea.timing_read())
+            fovea.timing_enable(False)
+            assert want <= names, (name, names)
+            if name.startswith("bf16"):
+                assert "query_proj" not in names
+        fovea.step_path(fovea.PATH_FUSED)
+        s = store(small_workload("fp32-ragged"))
+        with pytest.raises(fovea.FoveaError, match="UNSUPPORTED"):
+            run_gpu(s, fovea)
+    finally:
+        fovea.timing_enable(False)
+        fovea.step_path(prev)
+
+
+def test_zero_gate_returns_rmsnorm_of_h(fovea, path):
     w = small_workload("bf16-ragged")
     w.params["w_g2"] = np.zeros_like(w.params["w_g2"])
     w.params["b_g2"] = np.array([-1000.0], dtype=np.float32)
@@ -104,7 +142,7 @@ def test_zero_gate_returns_rmsnorm_of_h(fovea):
     assert rel_err_rows(gpu["h_out"].astype(np.float64), want).max() <= 2e-2
 
 
-def test_planted_rows_select_one_entry(fovea):
+def test_planted_rows_select_one_entry(fovea, path):
     spec = workloads.Spec(0, "planted-d512", d=512, B=1, rows_per_seq=24, rho=0.9, k_max=32,
                           k_min=1, dtype="bf16", seed=31, m_fixed=300, peaked_rows=6)
     w = workloads.generate(spec)
@@ -116,7 +154,7 @@ def test_planted_rows_select_one_entry(fovea):
     compare(gpu, orc, s, mem=mem)
 
 
-def test_repeat_calls_are_deterministic(fovea):
+def test_repeat_calls_are_deterministic(fovea, path):
     w = small_workload("bf16-temperature")
     s = store(w)
     params = params_for(s, fovea)
@@ -134,7 +172,7 @@ def test_repeat_calls_are_deterministic(fovea):
     fovea.sync_errors(ws)
 
 
-def test_invalid_depth_sets_error_word(fovea):
+def test_invalid_depth_sets_error_word(fovea, path):
     w = small_workload("bf16-ragged")
     w.depth = w.depth.copy()
     w.depth[3] = 9
@@ -147,7 +185,7 @@ def test_invalid_depth_sets_error_word(fovea):
     fovea.sync_errors(o["workspace"])      # the word was cleared
 
 
-def test_bad_row_offsets_and_workspace(fovea):
+def test_bad_row_offsets_and_workspace(fovea, path):
     w = small_workload("bf16-ragged")
     s = store(w)
     params = params_for(s, fovea)
@@ -174,15 +212,26 @@ def test_bad_row_offsets_and_workspace(fovea):
 # The five named workloads at full size
 # ---------------------------------------------------------------------------
 
+_NAMED = {}
+
+
+def _named(idx):
+    """Inputs and oracle result of a named workload, computed once for both paths."""
+    if idx not in _NAMED:
+        w = workloads.generate(workloads.WORKLOADS[idx])
+        s = store(w)
+        orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
+        _NAMED[idx] = (w, s, orc, mem)
+    return _NAMED[idx]
+
+
 @pytest.mark.parametrize("idx", [1, 2, 3, 4])
-def test_named_workload_parity(fovea, idx):
-    w = workloads.generate(workloads.WORKLOADS[idx])
-    s = store(w)
+def test_named_workload_parity(fovea, path, idx):
+    w, s, orc, mem = _named(idx)
     gpu = run_gpu(s, fovea)
     mirror = w.dtype == "bf16"
-    orc, mem = run_oracle(s, mirror=mirror)
     rep = compare(gpu, orc, s, mem=mem, mirror=mirror)
-    print(f"workload {idx}: {rep}")
+    print(f"workload {idx} ({path}): {rep}")
     if idx == 2:
         for row, entry in w.planted.items():
             assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
