@@ -257,6 +257,9 @@ def main():
     ap.add_argument("--workload", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="auto", choices=["auto", "fused", "kernels"],
+                    help="draft-step implementation: the library default (auto), the persistent "
+                         "step kernel (fused) or one kernel per stage (kernels)")
     args = ap.parse_args()
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
@@ -266,6 +269,8 @@ def main():
         return run_reference(args, w)
 
     from paper_2608_22883_gb300 import fovea
+    fovea.step_path({"auto": fovea.PATH_AUTO, "fused": fovea.PATH_FUSED,
+                     "kernels": fovea.PATH_KERNELS}[args.path])
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -425,7 +430,8 @@ def main():
     t_roof = max(t_hbm, t_tc)
     kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
     dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
-    dom_bytes = kernel_bytes(dom, w, uniq)
+    # the persistent step kernel moves the whole step's algorithmic bytes
+    dom_bytes = nbytes if dom == "fused_step" else kernel_bytes(dom, w, uniq)
     achieved = dom_bytes / (kern[dom]["ms_avg"] / 1000.0) / 1e9
     launches_per_step = sum(k["launches"] for k in kern.values()) / max(n_kt, 1)
     launches = int(round(launches_per_step * args.steps))
@@ -450,7 +456,10 @@ def main():
                    "draft_states": N, "sequences": w.B, "rho": w.rho, "k_min": w.k_min,
                    "k_max": K, "mlp_hidden": int(w.params["b_f1"].shape[0]),
                    "l2": "flushed before every step outside the per-step events (512 MB write, then a 256 MB read so the evicted lines are clean)",
-                   "launch": "one CUDA graph replay per step (the kernels of one fovea_retrieve_fuse call)",
+                   "launch": "one CUDA graph replay per step (the kernels of one fovea_retrieve_fuse call: "
+                             + ("one persistent cooperative kernel)" if list(kern) == ["fused_step"]
+                                else f"{len(kern)} kernels)"),
+                   "path": args.path,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved,
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],

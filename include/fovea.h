@@ -240,12 +240,14 @@ FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(const fovea_params* p, const 
 /*
  * Implementation of the draft step (process-wide; the paper has no
  * counterpart, both compute the same operator):
- *   FOVEA_PATH_AUTO     the persistent step kernel where the call fits it
- *                       (bf16, <= 64 sequences, <= 3072 valid entries per
- *                       sequence), else one kernel per stage (the default)
- *   FOVEA_PATH_FUSED    the persistent step kernel only; a call it does not
- *                       cover returns FOVEA_ERR_UNSUPPORTED
+ *   FOVEA_PATH_AUTO     the default: currently one kernel per stage, the
+ *                       faster implementation on every shape measured so far
+ *   FOVEA_PATH_FUSED    the persistent step kernel; it covers bf16 calls with
+ *                       <= 64 sequences and <= 3072 valid entries per
+ *                       sequence, and any other call returns
+ *                       FOVEA_ERR_UNSUPPORTED
  *   FOVEA_PATH_KERNELS  one kernel per stage of the step
+ * A workspace sized by fovea_workspace_size serves every path.
  * The persistent kernel is one cooperative launch of one CTA per SM whose
  * phases meet at device-wide barriers kept in the workspace header; it needs
  * the whole GPU, so a concurrent kernel on another stream delays its start.

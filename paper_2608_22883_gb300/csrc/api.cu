@@ -440,9 +440,9 @@ long long step_partial_floats(int dtype, int d, int H, int N, int ngroups, int m
 }
 
 // The persistent-kernel plan of a call (false: the call's shape is outside it).
+// (Independent of the path setting: a workspace is sized for both paths.)
 bool plan_fused_call(const fovea_params* p, const fovea_memory* mem, const int32_t* row_offsets,
                      int k_max, FusedPlan* plan) {
-  if (g_step_path.load() == FOVEA_PATH_KERNELS) return false;
   FusedShape sh;
   sh.bf16 = p->dtype == FOVEA_BF16;
   sh.N = row_offsets[mem->B];
@@ -597,13 +597,20 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   const int d = p->d_model, H = p->mlp_hidden, dt = p->dtype;
   static thread_local FusedPlan fplan;
-  const bool use_fused = plan_fused_call(p, mem, row_offsets, k_max, &fplan);
-  if (!use_fused && g_step_path.load() == FOVEA_PATH_FUSED)
+  // the persistent kernel runs only when selected; AUTO takes the per-stage
+  // kernels, which are faster on the shapes measured so far
+  const bool want_fused = g_step_path.load() == FOVEA_PATH_FUSED;
+  const bool use_fused = want_fused && plan_fused_call(p, mem, row_offsets, k_max, &fplan);
+  if (!use_fused && want_fused)
     return fail(FOVEA_ERR_UNSUPPORTED,
                 "the persistent step kernel does not cover this call (bf16, <= %d sequences, "
                 "<= 3072 entries per sequence are required)", fused::kMaxSeq);
   long long pfloats = step_partial_floats(dt, d, H, N, ngroups, max_m, max_r);
-  if (use_fused) pfloats = std::max(pfloats, fplan.partial_floats);
+  {
+    static thread_local FusedPlan fp_any;
+    if (plan_fused_call(p, mem, row_offsets, k_max, &fp_any))
+      pfloats = std::max(pfloats, fp_any.partial_floats);
+  }
   const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems, pfloats);
   if (workspace_bytes < L.total)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);

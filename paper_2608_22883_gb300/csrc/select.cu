@@ -1,7 +1,6 @@
 // Cumulative-mass selection kernel: one CTA of 256 threads per draft state
 // (the algorithm is in select_core.cuh).  The row's scores are staged in
-// shared memory while one pass forms the softmax statistics (running max and
-// rescaled sum).
+// shared memory first.
 #include "select_core.cuh"
 
 namespace fovea {
@@ -25,17 +24,13 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     return;
   }
   const float* src = a.scores + tab.score_off[b] + (long long)(n - tab.row_start[b]) * M;
-  // stage scores; softmax statistics in the same pass
-  float lmax = -INFINITY, lsum = 0.0f;
   for (int i = tid; i < M; i += kSelThreads) {
     float v = src[i];
     if (v == 0.0f) v = 0.0f;              // -0 -> +0 so equal scores get equal keys
     s_sc[i] = v;
-    combine_ms(lmax, lsum, v, 1.0f);
   }
-  float smax, sumexp;
-  select_stats(lmax, lsum, sm, tid, BlockSync{}, smax, sumexp);
-  select_finish(a, n, M, tab.key_off[b], s_sc, smax, sumexp, sm, tid, BlockSync{});
+  __syncthreads();
+  select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSync{});
 }
 
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,

@@ -6,8 +6,9 @@
 // I_n = pi_n(1..K)).
 //
 // The caller stages the row's scores in shared memory (-0 mapped to +0) and
-// forms each thread's running softmax statistics; select_stats combines them
-// over the group and select_finish does the rest.  A 4-pass 8-bit radix
+// calls select_row.  Rows of up to 2048 entries take a fast path with few
+// group barriers (select_fast, below).  Otherwise select_stats combines the
+// threads' softmax statistics and select_finish does the rest: a 4-pass 8-bit radix
 // select finds the K_eff-th largest score key (K_eff = min(K_max, |V|))
 // without sorting the row; only the K_eff candidates are put in order, by
 // (score desc, position asc): each candidate's rank is its count of larger
@@ -52,9 +53,10 @@ struct SelectSmem {
   unsigned long long sorted[kRankMax];
   float cum[FOVEA_MAX_K];                    // inclusive scan of exp(s - s_max)
   unsigned int hist[256];
-  float red_m[kSelWarps], red_s[kSelWarps];
+  float red_m[kSelWarps], red_s[kSelWarps], red_lo[kSelWarps];
   float warp_tot_f[kSelWarps];
   int warp_tot[kSelWarps];
+  int warp_first[kSelWarps];
   unsigned int sh_digit, sh_above;
   int sh_cnt_gt, sh_first;
   float sh_max, sh_sum;
@@ -298,6 +300,191 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
     a.sel_cnt[n] = K;
     if (a.counts) a.counts[n] = K;
   }
+}
+
+// Fast path for rows of at most kFastMaxM entries and K_eff <= kRankMax,
+// with six group barriers: the threads keep their scores in registers; one
+// pass gives the softmax statistics and the minimum score; a 256-bin
+// histogram of s_max - s over [0, s_max - s_min] gives the bin b* holding the
+// K_eff-th largest score (the bin index is monotone in the score, so the top
+// K_eff entries all lie in bins <= b*); the entries of bins <= b* are ranked
+// among themselves by (score desc, position asc), which puts the top K_eff in
+// order; the mass scan then runs one ordered entry per thread.  Returns false,
+// having written nothing, when the candidates exceed kFastMaxCand; the caller
+// then runs the radix path.
+constexpr int kFastMaxM = 2048;                   // 8 scores per thread
+constexpr int kFastMaxCand = FOVEA_MAX_K;         // candidates ranked directly
+
+template <class Sync>
+__device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, const float* s_sc,
+                            SelectSmem& sm, int tid, Sync sync) {
+  constexpr int PT = kFastMaxM / kSelThreads;
+  const int lane = tid & 31, warp = tid >> 5;
+  const int k_max = a.k_max;
+  const int K_eff = min(k_max, M);
+  float v[PT];
+  float lmax = -INFINITY, lsum = 0.0f, lmin = INFINITY;
+#pragma unroll
+  for (int j = 0; j < PT; ++j) {
+    const int i = tid + j * kSelThreads;
+    v[j] = i < M ? s_sc[i] : -INFINITY;
+    if (i < M) {
+      combine_ms(lmax, lsum, v[j], 1.0f);
+      lmin = fminf(lmin, v[j]);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, lmax, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, lsum, o);
+    combine_ms(lmax, lsum, m2, s2);
+    lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, o));
+  }
+  for (int i = tid; i < 256; i += kSelThreads) sm.hist[i] = 0;
+  if (lane == 0) {
+    sm.red_m[warp] = lmax;
+    sm.red_s[warp] = lsum;
+    sm.red_lo[warp] = lmin;
+  }
+  if (tid == 0) sm.sh_cnt_gt = 0;
+  sync();                                                     // (1)
+  float smax = sm.red_m[0], sumexp = sm.red_s[0], smin = sm.red_lo[0];
+  for (int w = 1; w < kSelWarps; ++w) {
+    combine_ms(smax, sumexp, sm.red_m[w], sm.red_s[w]);
+    smin = fminf(smin, sm.red_lo[w]);
+  }
+  // ---- histogram of the distance to the maximum ----------------------------
+  const float range = smax - smin;
+  const float inv_w = range > 0.0f ? 255.0f / range : 0.0f;
+  int bin[PT];
+#pragma unroll
+  for (int j = 0; j < PT; ++j) {
+    const int i = tid + j * kSelThreads;
+    bin[j] = 256;
+    if (i < M) {
+      const int b = (int)((smax - v[j]) * inv_w);
+      bin[j] = b < 0 ? 0 : (b > 255 ? 255 : b);
+      atomicAdd(&sm.hist[bin[j]], 1u);
+    }
+  }
+  sync();                                                     // (2)
+  // every warp finds b* itself: lane l owns bins 8l .. 8l + 7
+  int bstar;
+  {
+    unsigned int cnt[8], tot = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      cnt[j] = sm.hist[8 * lane + j];
+      tot += cnt[j];
+    }
+    unsigned int incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    const unsigned int ballot = __ballot_sync(0xffffffffu, incl >= (unsigned)K_eff);
+    const int L = __ffs(ballot) - 1;      // exists: the bins hold M >= K_eff entries
+    int bl = 0;
+    if (lane == L) {
+      unsigned int run = incl - tot;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (bl == 0 && run + cnt[j] >= (unsigned)K_eff) bl = 8 * lane + j + 1;
+        run += cnt[j];
+      }
+    }
+    bstar = __shfl_sync(0xffffffffu, bl, L) - 1;
+  }
+  // ---- candidates: the entries of bins <= b* -------------------------------
+#pragma unroll
+  for (int j = 0; j < PT; ++j) {
+    const int i = tid + j * kSelThreads;
+    const bool take = bin[j] <= bstar;
+    const unsigned int bal = __ballot_sync(0xffffffffu, take);
+    int slot0 = 0;
+    if (lane == 0 && bal) slot0 = atomicAdd(&sm.sh_cnt_gt, __popc(bal));
+    slot0 = __shfl_sync(0xffffffffu, slot0, 0);
+    if (take) {
+      const int slot = slot0 + __popc(bal & ((1u << lane) - 1u));
+      if (slot < kFastMaxCand)
+        sm.cand[slot] = ((unsigned long long)ord_key(v[j]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+    }
+  }
+  sync();                                                     // (3)
+  const int C = sm.sh_cnt_gt;
+  if (C > kFastMaxCand) return false;                         // uniform
+  // ---- rank the candidates: rank = #larger (keys are distinct) -------------
+  for (int c = tid; c < C; c += kSelThreads) {
+    const unsigned long long me = sm.cand[c];
+    int r = 0;
+    for (int j = 0; j < C; ++j) r += sm.cand[j] > me;
+    if (r < K_eff) sm.sorted[r] = me;
+  }
+  sync();                                                     // (4)
+  // ---- cumulative mass, one ordered entry per thread -----------------------
+  const int t = tid;
+  float e = 0.0f;
+  int pos = 0;
+  if (t < K_eff) {
+    pos = (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[t] & 0xFFFFFFFFull));
+    e = expf(s_sc[pos] - smax);
+  }
+  float incl = e;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float u = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += u;
+  }
+  if (lane == 31) sm.warp_tot_f[warp] = incl;
+  sync();                                                     // (5)
+  float before = 0.0f;
+  for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
+  const float cum = before + incl;
+  if (t < K_eff) sm.cum[t] = cum;
+  {
+    const unsigned int bal = __ballot_sync(0xffffffffu, t < K_eff && cum / sumexp >= a.rho);
+    if (lane == 0) sm.warp_first[warp] = bal ? warp * 32 + __ffs(bal) - 1 : K_eff;
+  }
+  sync();                                                     // (6)
+  int first = K_eff;
+  for (int w = 0; w < kSelWarps; ++w) first = min(first, sm.warp_first[w]);
+  const int K = first < K_eff ? min(K_eff, max(a.k_min, first + 1)) : K_eff;
+  const float denom = sm.cum[K - 1];                          // sum over I_n of exp(s - s_max)
+  const long long out_row = (long long)n * k_max;
+  for (int u = tid; u < k_max; u += kSelThreads) {
+    if (u < K) {
+      const int pu = u == t ? pos : (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[u] & 0xFFFFFFFFull));
+      const float eu = u == t ? e : expf(s_sc[pu] - smax);
+      const int row = key_off + pu;
+      a.sel_pos[out_row + u] = row;
+      a.sel_w[out_row + u] = eu / denom;
+      if (a.indices) a.indices[out_row + u] = a.orig_index[row];
+    } else if (a.indices) {
+      a.indices[out_row + u] = -1;
+    }
+  }
+  if (tid == 0) {
+    a.sel_cnt[n] = K;
+    if (a.counts) a.counts[n] = K;
+  }
+  return true;
+}
+
+// Selection of draft state n from its staged scores (s_sc, M >= 1 entries,
+// staged and visible to the group): the fast path where it applies, else the
+// radix path.
+template <class Sync>
+__device__ __forceinline__ void select_row(const SelectArgs& a, int n, int M, int key_off,
+                                           const float* s_sc, SelectSmem& sm, int tid, Sync sync) {
+  if (M <= kFastMaxM && min(a.k_max, M) <= kRankMax &&
+      select_fast(a, n, M, key_off, s_sc, sm, tid, sync))
+    return;
+  float lmax = -INFINITY, lsum = 0.0f;
+  for (int i = tid; i < M; i += kSelThreads) combine_ms(lmax, lsum, s_sc[i], 1.0f);
+  float smax, sumexp;
+  select_stats(lmax, lsum, sm, tid, sync, smax, sumexp);
+  select_finish(a, n, M, key_off, s_sc, smax, sumexp, sm, tid, sync);
 }
 
 // Outputs of a draft state whose sequence has no valid entry: K = 0.

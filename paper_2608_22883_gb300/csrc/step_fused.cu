@@ -116,8 +116,11 @@ __device__ bool spin_barrier(const FusedArgs& a, int k) {
   if (ld_acquire_gpu(ctr) >= G) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
-    for (int i = 0; i < 32; ++i)
+    // poll with a short sleep: every SM polls the same line
+    for (int i = 0; i < 32; ++i) {
+      __nanosleep(40);
       if (ld_acquire_gpu(ctr) >= G) return true;
+    }
     if (ld_acquire_gpu(a.sync + kSyncAbort) != 0) return false;
     if (globaltimer_ns() - t0 > kWaitNs) {
       atomicOr(a.err, kErrTimeout);
@@ -168,6 +171,32 @@ __device__ __forceinline__ UnitPos decode_unit(const PhaseGemm& p, int u) {
 }
 __device__ __forceinline__ float* partial_tile(const FusedArgs& a, const PhaseGemm& p, int u) {
   return a.partials + (long long)u * 128 * p.bn;
+}
+
+// Sum in split order of the S partial float4 at base + s * stride (floats),
+// with the loads of up to 16 splits in flight together.
+__device__ __forceinline__ float4 sum_splits(const float* base, long long stride, int S) {
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s0 = 0; s0 < S; s0 += 16) {
+    float4 t[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (s0 + i < S) t[i] = __ldcg(reinterpret_cast<const float4*>(base + (s0 + i) * stride));
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (s0 + i < S) {
+        if (s0 + i == 0) {
+          acc = t[i];
+        } else {
+          acc.x += t[i].x;
+          acc.y += t[i].y;
+          acc.z += t[i].z;
+          acc.w += t[i].w;
+        }
+      }
+    }
+  }
+  return acc;
 }
 
 // k-block cursor over (phase, unit of this CTA, k-block)
@@ -240,7 +269,7 @@ __device__ void producer(const FusedArgs& a, const FusedMaps& maps, uint8_t* rin
       const UnitPos up = decode_unit(p, cf.u);
       const int rbytes = p.dual ? 2 * kRTile : kRTile;
       uint8_t* stage = ring + st * kStageBytes;
-      mbar_expect_tx(&full[st], (uint32_t)(rbytes + p.bn * 128));
+      mbar_expect_tx(&full[st], (uint32_t)((p.dual ? 2 : 1) * p.rbox * 128 + p.bn * 128));
       const int f = up.ft * p.bn;
       const bool second = f >= p.f_split;
       tma_load_2d(stage + rbytes, &maps.m[second ? p.fmap1 : p.fmap0], &full[st], cf.kb * 64,
@@ -367,10 +396,14 @@ __device__ void mma_issuer(const FusedArgs& a, uint8_t* ring, uint64_t* full, ui
 // worker phases
 // ---------------------------------------------------------------------------
 
-// LN_h(h_n) + E_dep[l_n] -> x (bf16), one row per CTA iteration (query equation).
+// LN_h(h_n) + E_dep[l_n] -> x (bf16), one row per CTA iteration (query
+// equation).  The row stays in registers between the statistics and the
+// affine map; gamma, beta and the depth embedding are loaded per vector in
+// the second pass, so few values are live at once.  Four independent
+// double-float accumulators per sum keep the dependency chains short.
 __device__ void phase_ln(const FusedArgs& a, const WorkerCtx& w, uint8_t* scr) {
   constexpr int MV = FOVEA_MAX_D / 8 / kWorkers;     // 16-byte vectors per thread
-  dfloat* red = reinterpret_cast<dfloat*>(scr);      // [2][8]
+  dfloat* red = reinterpret_cast<dfloat*>(scr);      // [2][8], then mean, rstd
   const int d = a.d, nvec = d / 8;
   for (int n = blockIdx.x; n < a.N; n += gridDim.x) {
     int dep = a.depth[n];
@@ -380,27 +413,29 @@ __device__ void phase_ln(const FusedArgs& a, const WorkerCtx& w, uint8_t* scr) {
     }
     const bf16* xr = a.h + (long long)n * d;
     const bf16* er = a.E + (long long)dep * d;
-    float xv[MV][8], gv[MV][8], bv[MV][8], ev[MV][8];
+    float xv[MV][8];
 #pragma unroll
     for (int j = 0; j < MV; ++j) {
       const int vi = w.wtid + j * kWorkers;
-      if (vi < nvec) {
-        ln_load<bf16>(xr + vi * 8, xv[j]);
-        ln_load<bf16>(a.ln_gamma + vi * 8, gv[j]);
-        ln_load<bf16>(a.ln_beta + vi * 8, bv[j]);
-        ln_load<bf16>(er + vi * 8, ev[j]);
-      }
+      if (vi < nvec) ln_load<bf16>(xr + vi * 8, xv[j]);
     }
-    dfloat s1 = {0.0f, 0.0f}, s2 = {0.0f, 0.0f};
+    dfloat s1, s2;
+    {
+      dfloat a1[4], a2[4];
 #pragma unroll
-    for (int j = 0; j < MV; ++j) {
-      if (w.wtid + j * kWorkers < nvec) {
+      for (int q = 0; q < 4; ++q) a1[q] = a2[q] = dfloat{0.0f, 0.0f};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          s1 = df_add_f(s1, xv[j][i]);
-          s2 = df_add(s2, df_two_prod(xv[j][i], xv[j][i]));
+      for (int j = 0; j < MV; ++j) {
+        if (w.wtid + j * kWorkers < nvec) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            a1[i & 3] = df_add_f(a1[i & 3], xv[j][i]);
+            a2[i & 3] = df_add(a2[i & 3], df_two_prod(xv[j][i], xv[j][i]));
+          }
         }
       }
+      s1 = df_add(df_add(a1[0], a1[1]), df_add(a1[2], a1[3]));
+      s2 = df_add(df_add(a2[0], a2[1]), df_add(a2[2], a2[3]));
     }
     s1 = warp_sum_df(s1);
     s2 = warp_sum_df(s2);
@@ -431,12 +466,16 @@ __device__ void phase_ln(const FusedArgs& a, const WorkerCtx& w, uint8_t* scr) {
     for (int j = 0; j < MV; ++j) {
       const int vi = w.wtid + j * kWorkers;
       if (vi < nvec) {
+        float gv[8], bv[8], ev[8];
+        ln_load<bf16>(a.ln_gamma + vi * 8, gv);
+        ln_load<bf16>(a.ln_beta + vi * 8, bv);
+        ln_load<bf16>(er + vi * 8, ev);
         bf16 res[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           dfloat y = df_mul(df_add_f(neg_mean, xv[j][i]), rstd);
-          y = df_add_f(df_mul_f(y, gv[j][i]), bv[j][i]);
-          y = df_add_f(y, ev[j][i]);
+          y = df_add_f(df_mul_f(y, gv[i]), bv[i]);
+          y = df_add_f(y, ev[i]);
           res[i] = df_to_bf16(y);
         }
         *reinterpret_cast<uint4*>(o + vi * 8) = *reinterpret_cast<const uint4*>(res);
@@ -521,29 +560,8 @@ __device__ void phase_reduce(const FusedArgs& a, const WorkerCtx& w) {
     const int rt = n >> 7, rit = n & 127;
     const int ft = c / p.bn, j = c - ft * p.bn;
     const int u0 = p.unit0[0] + (rt * p.ftiles[0] + ft) * p.splits;
-    float4 part[16];
-#pragma unroll
-    for (int s = 0; s < 16; ++s)
-      if (s < p.splits)
-        part[s] = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u0 + s) +
-                                                         (long long)rit * p.bn + j));
-    float4 acc = part[0];
-#pragma unroll
-    for (int s = 1; s < 16; ++s)
-      if (s < p.splits) {
-        acc.x += part[s].x;
-        acc.y += part[s].y;
-        acc.z += part[s].z;
-        acc.w += part[s].w;
-      }
-    for (int s = 16; s < p.splits; ++s) {
-      const float4 t = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u0 + s) +
-                                                              (long long)rit * p.bn + j));
-      acc.x += t.x;
-      acc.y += t.y;
-      acc.z += t.z;
-      acc.w += t.w;
-    }
+    const float4 acc = sum_splits(partial_tile(a, p, u0) + (long long)rit * p.bn + j,
+                                  128ll * p.bn, p.splits);
     const float v[4] = {acc.x, acc.y, acc.z, acc.w};
     if constexpr (PH == kPhaseQuery) {
       bf16 hi[4], lo[4];
@@ -598,19 +616,8 @@ __device__ void phase_select(const FusedArgs& a, const WorkerCtx& w, uint8_t* sc
       const int i0 = q * 4;
       const int ft = i0 / p.bn, j = i0 - ft * p.bn;
       const int u0 = p.unit0[g] + (rt * p.ftiles[g] + ft) * p.splits;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int s = 0; s < p.splits; ++s) {
-        const float4 t = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u0 + s) +
-                                                                (long long)rit * p.bn + j));
-        if (s == 0) {
-          acc = t;
-        } else {
-          acc.x += t.x;
-          acc.y += t.y;
-          acc.z += t.z;
-          acc.w += t.w;
-        }
-      }
+      const float4 acc = sum_splits(partial_tile(a, p, u0) + (long long)rit * p.bn + j,
+                                    128ll * p.bn, p.splits);
       const float v[4] = {acc.x, acc.y, acc.z, acc.w};
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -622,11 +629,7 @@ __device__ void phase_select(const FusedArgs& a, const WorkerCtx& w, uint8_t* sc
       }
     }
     wsync();
-    float lmax = -INFINITY, lsum = 0.0f;
-    for (int i = w.wtid; i < M; i += kWorkers) combine_ms(lmax, lsum, s_sc[i], 1.0f);
-    float smax, sumexp;
-    select_stats(lmax, lsum, sm, w.wtid, WorkerSync{}, smax, sumexp);
-    select_finish(sa, n, M, a.key_off[b], s_sc, smax, sumexp, sm, w.wtid, WorkerSync{});
+    select_row(sa, n, M, a.key_off[b], s_sc, sm, w.wtid, WorkerSync{});
   }
 }
 
@@ -651,19 +654,51 @@ __device__ void phase_readout(const FusedArgs& a, const WorkerCtx& w, uint8_t* s
     wsync();                          // the previous item's readers are done
     if (M > 0) {
       const int pieces = W >> 3;      // 16-byte pieces per value row slice
-      for (int i = w.wtid; i < M * pieces; i += kWorkers) {
-        const int r = i / pieces, pc = i - r * pieces;
-        const uint4 v = __ldg(reinterpret_cast<const uint4*>(a.U + (long long)(koff + r) * a.d + c0 + pc * 8));
-        *reinterpret_cast<uint4*>(us + r * W + pc * 8) = v;
+      const int tot = M * pieces;
+      for (int i0 = w.wtid; i0 < tot; i0 += 8 * kWorkers) {
+        uint4 v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int i = i0 + k * kWorkers;
+          if (i < tot) {
+            const int r = i / pieces, pc = i - r * pieces;
+            v[k] = __ldg(reinterpret_cast<const uint4*>(a.U + (long long)(koff + r) * a.d + c0 + pc * 8));
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int i = i0 + k * kWorkers;
+          if (i < tot) {
+            const int r = i / pieces, pc = i - r * pieces;
+            *reinterpret_cast<uint4*>(us + r * W + pc * 8) = v[k];
+          }
+        }
       }
     }
     for (int rb = 0; rb < R; rb += a.ro_rows) {
       const int nb = min(a.ro_rows, R - rb);
       if (rb > 0) wsync();
-      for (int i = w.wtid; i < nb * k_max; i += kWorkers) {
-        const long long gi = (long long)(row0 + rb) * k_max + i;
-        spos[i] = __ldcg(a.sel_pos + gi) - koff;
-        sw[i] = __ldcg(a.sel_w + gi);
+      const int tot = nb * k_max;
+      const long long g0 = (long long)(row0 + rb) * k_max;
+      for (int i0 = w.wtid; i0 < tot; i0 += 8 * kWorkers) {
+        int pv[8];
+        float wv[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int i = i0 + k * kWorkers;
+          if (i < tot) {
+            pv[k] = __ldcg(a.sel_pos + g0 + i);
+            wv[k] = __ldcg(a.sel_w + g0 + i);
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int i = i0 + k * kWorkers;
+          if (i < tot) {
+            spos[i] = pv[k] - koff;
+            sw[i] = wv[k];
+          }
+        }
       }
       for (int i = w.wtid; i < nb; i += kWorkers) scnt[i] = __ldcg(a.sel_cnt + row0 + rb + i);
       wsync();
@@ -673,17 +708,45 @@ __device__ void phase_readout(const FusedArgs& a, const WorkerCtx& w, uint8_t* s
         const int K = scnt[rr];
         const int* pp = spos + rr * k_max;
         const float* ww = sw + rr * k_max;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int t = 0; t < K; ++t) {
+        // four entries per step with their loads issued together; the four
+        // partial sums are combined in a fixed order
+        float acc4[4][4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) acc4[q][i] = 0.f;
+        int t = 0;
+        for (; t + 4 <= K; t += 4) {
+          uint2 raw[4];
+          float wt[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            wt[q] = ww[t + q];
+            raw[q] = *reinterpret_cast<const uint2*>(us + pp[t + q] * W + cq * 4);
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&raw[q]);
+            const float2 f0 = __bfloat1622float2(h2[0]), f1 = __bfloat1622float2(h2[1]);
+            acc4[q][0] = fmaf(wt[q], f0.x, acc4[q][0]);
+            acc4[q][1] = fmaf(wt[q], f0.y, acc4[q][1]);
+            acc4[q][2] = fmaf(wt[q], f1.x, acc4[q][2]);
+            acc4[q][3] = fmaf(wt[q], f1.y, acc4[q][3]);
+          }
+        }
+        for (; t < K; ++t) {
           const float wt = ww[t];
           const uint2 raw = *reinterpret_cast<const uint2*>(us + pp[t] * W + cq * 4);
           const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
           const float2 f0 = __bfloat1622float2(h2[0]), f1 = __bfloat1622float2(h2[1]);
-          acc[0] = fmaf(wt, f0.x, acc[0]);
-          acc[1] = fmaf(wt, f0.y, acc[1]);
-          acc[2] = fmaf(wt, f1.x, acc[2]);
-          acc[3] = fmaf(wt, f1.y, acc[3]);
+          acc4[0][0] = fmaf(wt, f0.x, acc4[0][0]);
+          acc4[0][1] = fmaf(wt, f0.y, acc4[0][1]);
+          acc4[0][2] = fmaf(wt, f1.x, acc4[0][2]);
+          acc4[0][3] = fmaf(wt, f1.y, acc4[0][3]);
         }
+        float acc[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[i] = (acc4[0][i] + acc4[1][i]) + (acc4[2][i] + acc4[3][i]);
         const long long n = row0 + rb + rr;
         const int col = c0 + cq * 4;
         bf16 o[4];
@@ -698,7 +761,8 @@ __device__ void phase_readout(const FusedArgs& a, const WorkerCtx& w, uint8_t* s
 }
 
 // Gate, gated residual and RMSNorm (Eq. hidden_correction), with c summed
-// from the last fusion layer's partial tiles in split order plus b_f2.
+// from the last fusion layer's partial tiles in split order plus b_f2.  The
+// gate comes first; y = h + g c stays in registers for the second pass.
 __device__ void phase_finalize(const FusedArgs& a, const WorkerCtx& w, uint8_t* scr) {
   constexpr int MV = FOVEA_MAX_D / 8 / kWorkers;
   float* red = reinterpret_cast<float*>(scr);
@@ -706,55 +770,57 @@ __device__ void phase_finalize(const FusedArgs& a, const WorkerCtx& w, uint8_t* 
   const int d = a.d, H = a.H, nvec = d / 8;
   for (int n = blockIdx.x; n < a.N; n += gridDim.x) {
     const int rt = n >> 7, rit = n & 127;
-    float hv[MV][8], gv[MV][8];
-#pragma unroll
-    for (int j = 0; j < MV; ++j) {
-      const int vi = w.wtid + j * kWorkers;
-      if (vi < nvec) {
-        ln_load<bf16>(a.h + (long long)n * d + vi * 8, hv[j]);
-        ln_load<bf16>(a.rms_gamma + vi * 8, gv[j]);
-      }
-    }
-    float cv[MV][8];
-#pragma unroll
-    for (int j = 0; j < MV; ++j) {
-      const int vi = w.wtid + j * kWorkers;
-      if (vi < nvec) {
-#pragma unroll
-        for (int h4 = 0; h4 < 2; ++h4) {
-          const int c = vi * 8 + h4 * 4;
-          const int ft = c / p.bn, jj = c - ft * p.bn;
-          const int u0 = p.unit0[0] + (rt * p.ftiles[0] + ft) * p.splits;
-          float4 acc = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u0) + (long long)rit * p.bn + jj));
-          for (int s = 1; s < p.splits; ++s) {
-            const float4 t = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u0 + s) +
-                                                                    (long long)rit * p.bn + jj));
-            acc.x += t.x;
-            acc.y += t.y;
-            acc.z += t.z;
-            acc.w += t.w;
-          }
-          cv[j][h4 * 4 + 0] = acc.x + __bfloat162float(a.b_f2[c + 0]);
-          cv[j][h4 * 4 + 1] = acc.y + __bfloat162float(a.b_f2[c + 1]);
-          cv[j][h4 * 4 + 2] = acc.z + __bfloat162float(a.b_f2[c + 2]);
-          cv[j][h4 * 4 + 3] = acc.w + __bfloat162float(a.b_f2[c + 3]);
-        }
-      }
-    }
     const bf16* a_g = a.act + (long long)n * 2 * H + H;
     float part = 0.0f;
     for (int k = w.wtid; k < H; k += kWorkers)
       part = fmaf(__bfloat162float(__ldcg(a_g + k)), __bfloat162float(a.w_g2[k]), part);
     const float z = worker_sum(part, red, w.wtid) + __bfloat162float(a.b_g2[0]);
     const float g = sigmoidf_(z);
+    // c = sum of the partial tiles in split order (every quad's load of one
+    // split in flight together)
+    float yv[MV][8];
+    for (int s = 0; s < p.splits; ++s) {
+      float4 t[MV][2];
+#pragma unroll
+      for (int j = 0; j < MV; ++j) {
+        const int vi = w.wtid + j * kWorkers;
+        if (vi < nvec) {
+#pragma unroll
+          for (int h4 = 0; h4 < 2; ++h4) {
+            const int c = vi * 8 + h4 * 4;
+            const int ft = c / p.bn, jj = c - ft * p.bn;
+            const int u = p.unit0[0] + (rt * p.ftiles[0] + ft) * p.splits + s;
+            t[j][h4] = __ldcg(reinterpret_cast<const float4*>(partial_tile(a, p, u) +
+                                                               (long long)rit * p.bn + jj));
+          }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < MV; ++j) {
+        if (w.wtid + j * kWorkers < nvec) {
+#pragma unroll
+          for (int h4 = 0; h4 < 2; ++h4) {
+            const float e[4] = {t[j][h4].x, t[j][h4].y, t[j][h4].z, t[j][h4].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              yv[j][h4 * 4 + i] = s == 0 ? e[i] : yv[j][h4 * 4 + i] + e[i];
+          }
+        }
+      }
+    }
     float ss = 0.0f;
 #pragma unroll
     for (int j = 0; j < MV; ++j) {
-      if (w.wtid + j * kWorkers < nvec) {
+      const int vi = w.wtid + j * kWorkers;
+      if (vi < nvec) {
+        float hv[8], bf[8];
+        ln_load<bf16>(a.h + (long long)n * d + vi * 8, hv);
+        ln_load<bf16>(a.b_f2 + vi * 8, bf);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          hv[j][i] = fmaf(g, cv[j][i], hv[j][i]);     // y = h + g c
-          ss = fmaf(hv[j][i], hv[j][i], ss);
+          const float c = yv[j][i] + bf[i];
+          yv[j][i] = fmaf(g, c, hv[i]);          // y = h + g c
+          ss = fmaf(yv[j][i], yv[j][i], ss);
         }
       }
     }
@@ -765,9 +831,11 @@ __device__ void phase_finalize(const FusedArgs& a, const WorkerCtx& w, uint8_t* 
     for (int j = 0; j < MV; ++j) {
       const int vi = w.wtid + j * kWorkers;
       if (vi < nvec) {
+        float gv[8];
+        ln_load<bf16>(a.rms_gamma + vi * 8, gv);
         bf16 res[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) res[i] = __float2bfloat16_rn(hv[j][i] * inv * gv[j][i]);
+        for (int i = 0; i < 8; ++i) res[i] = __float2bfloat16_rn(yv[j][i] * inv * gv[i]);
         *reinterpret_cast<uint4*>(o + vi * 8) = *reinterpret_cast<const uint4*>(res);
       }
     }
@@ -889,8 +957,9 @@ void plan_phase(fused::PhaseGemm& p, int G, int kb_total, const int* m, const in
     if (dual && bn > 128) continue;
     if (f_split_hint > 0 && f_split_hint % bn != 0) continue;
     long long tiles = 0, outs = 0;
-    int rtiles_max = 0;
+    int rtiles_max = 0, rows_max = 0;
     for (int g = 0; g < ngroups; ++g) {
+      rows_max = std::max(rows_max, n[g]);
       tiles += (long long)((n[g] + 127) / 128) * ((m[g] + bn - 1) / bn);
       outs += (long long)n[g] * m[g];
       rtiles_max = std::max(rtiles_max, (n[g] + 127) / 128);
@@ -902,7 +971,11 @@ void plan_phase(fused::PhaseGemm& p, int G, int kb_total, const int* m, const in
     const long long waves = (units + G - 1) / G;
     const int nkb = (kb_total + S - 1) / S;
     const double t_mma = nkb * 4.0 * mma_cycles(bn) * (dual ? 2 : 1) / 2000.0;
-    const double t_bytes = nkb * (double)bn * 128.0 / (rtiles_max > 1 ? 150e3 : 50e3);
+    // feature bytes from HBM (from L2 when several row tiles reuse them), row
+    // bytes from L2; per-SM shares of the bandwidth in bytes per microsecond
+    const double rbytes = (dual ? 2.0 : 1.0) * std::min(128, (rows_max + 7) / 8 * 8) * 128.0;
+    const double t_bytes = nkb * ((double)bn * 128.0 / (rtiles_max > 1 ? 150e3 : 45e3) +
+                                  rbytes / 150e3);
     const double t_red = (double)S * outs * 4.0 / (G * 100e3);
     const double t = waves * std::max(t_mma, t_bytes) + t_red;
     if (t < best - 1e-9) {
@@ -911,6 +984,9 @@ void plan_phase(fused::PhaseGemm& p, int G, int kb_total, const int* m, const in
       best_s = S;
     }
   }
+  int rows_max = 0;
+  for (int g = 0; g < ngroups; ++g) rows_max = std::max(rows_max, n[g]);
+  p.rbox = std::min(128, (rows_max + 7) / 8 * 8);
   p.bn = best_bn;
   p.splits = best_s;
   p.kb_total = kb_total;
@@ -1033,16 +1109,16 @@ cudaError_t launch_fused_step(const FusedPlan& pl, const FusedLaunch& L, cudaStr
             bn2 = pl.g[kPhaseFuse2].bn;
   const Op ops[kNumMaps] = {
       {L.W_Q, d, d, d, bnQ},                       // 0 F: query weights
-      {L.x, N, d, d, 128},                         // 1 R: LN(h) + E
+      {L.x, N, d, d, pl.g[kPhaseQuery].rbox},      // 1 R: LN(h) + E
       {L.keys, std::max<long long>(L.total_keys, 1), d, d, bnS},   // 2 F: keys
-      {L.q_hi, N, d, d, 128},                      // 3 R: q hi
-      {L.q_lo, N, d, d, 128},                      // 4 R: q lo
+      {L.q_hi, N, d, d, std::max(8, pl.g[kPhaseScore].rbox)},   // 3 R: q hi
+      {L.q_lo, N, d, d, std::max(8, pl.g[kPhaseScore].rbox)},   // 4 R: q lo
       {L.W_f1, H, 2 * d, 2 * d, bn1},              // 5 F: W_f1
       {L.W_g1, H, 2 * d, 2 * d, bn1},              // 6 F: W_g1
-      {L.h, N, d, d, 128},                         // 7 R: h
-      {L.r, N, d, d, 128},                         // 8 R: r
+      {L.h, N, d, d, pl.g[kPhaseFuse1].rbox},      // 7 R: h
+      {L.r, N, d, d, pl.g[kPhaseFuse1].rbox},      // 8 R: r
       {L.W_f2, d, H, H, bn2},                      // 9 F: W_f2
-      {L.act, N, H, 2 * H, 128},                   // 10 R: a_f (columns 0..H-1 of act)
+      {L.act, N, H, 2 * H, pl.g[kPhaseFuse2].rbox},   // 10 R: a_f (columns 0..H-1 of act)
   };
   for (int i = 0; i < kNumMaps; ++i) {
     if (!encode_bf16_map(&maps.m[i], ops[i].base, ops[i].rows, ops[i].cols, ops[i].ld,

@@ -24,6 +24,7 @@ struct PhaseGemm {
   int r_split_kb;    // k-blocks >= r_split_kb read the row operand from rmap1
   int f_split;       // features >= f_split come from fmap1 (a multiple of bn)
   int dual;          // scores: the row stage holds q_hi and q_lo tiles (rmap0, rmap1)
+  int rbox;          // rows per row-operand load (<= 128; the MMA's rows beyond it are unused)
   int fmap0, fmap1, rmap0, rmap1;   // tensor-map indices
   int wait_r0, wait_r1;             // grid barrier the row loads from rmap0 / rmap1 wait for
   int ngroups, units;

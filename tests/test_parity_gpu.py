@@ -6,9 +6,10 @@ rho = 0.8 / K_min = 32 / K_max = 256, fixed top-16, dense), per-row
 temperatures, clustered keys and the fp32 path.  The five named workloads run
 at full size (the long-memory one on sampled rows and steps).
 
-Every parity test runs on both implementations of the draft step: "auto"
-(the persistent step kernel wherever a call fits it, which covers every bf16
-case here except the long-memory one) and "kernels" (one kernel per stage).
+Every parity test runs on both implementations of the draft step: "fused"
+(the persistent step kernel, which covers every bf16 case here except the
+long-memory one; fp32 cases skip it) and "kernels" (one kernel per stage,
+the default).
 """
 
 import dataclasses
@@ -32,7 +33,7 @@ def fovea():
     return f
 
 
-PATHS = {"auto": 0, "kernels": 2}
+PATHS = {"fused": 1, "kernels": 2}
 
 
 @pytest.fixture(params=sorted(PATHS))
@@ -40,6 +41,11 @@ def path(request, fovea):
     prev = fovea.step_path(PATHS[request.param])
     yield request.param
     fovea.step_path(prev)
+
+
+def skip_fp32_on_fused(path, dtype):
+    if path == "fused" and dtype != "bf16":
+        pytest.skip("the persistent step kernel covers bf16 calls only")
 
 
 SMALL = {
@@ -72,6 +78,7 @@ def small_workload(name):
 @pytest.mark.parametrize("name", sorted(SMALL))
 def test_small_parity(fovea, path, name):
     w = small_workload(name)
+    skip_fp32_on_fused(path, w.dtype)
     s = store(w)
     gpu = run_gpu(s, fovea)
     orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
@@ -107,20 +114,21 @@ def test_memory_build_matches_oracle(fovea, name):
 
 
 def test_paths_are_taken(fovea):
-    """AUTO runs the persistent step kernel for a bf16 call and the per-stage
-    kernels for an fp32 one; FUSED refuses a call outside its coverage."""
+    """AUTO runs the per-stage kernels; FUSED runs the persistent step kernel
+    for a bf16 call and refuses an fp32 one (outside its coverage)."""
     prev = fovea.step_path(fovea.PATH_AUTO)
     try:
-        for name, want in (("bf16-ragged", {"fused_step"}),
-                           ("fp32-ragged", {"ln_query", "query_proj", "select", "finalize"})):
+        for path, name, want, absent in (
+                (fovea.PATH_AUTO, "bf16-ragged", {"ln_query", "query_proj", "select", "finalize"},
+                 "fused_step"),
+                (fovea.PATH_FUSED, "bf16-ragged", {"fused_step"}, "query_proj")):
+            fovea.step_path(path)
             s = store(small_workload(name))
             fovea.timing_enable(True)
             run_gpu(s, fovea)
             names = set(fovea.timing_read())
             fovea.timing_enable(False)
-            assert want <= names, (name, names)
-            if name.startswith("bf16"):
-                assert "query_proj" not in names
+            assert want <= names and absent not in names, (path, names)
         fovea.step_path(fovea.PATH_FUSED)
         s = store(small_workload("fp32-ragged"))
         with pytest.raises(fovea.FoveaError, match="UNSUPPORTED"):
@@ -227,6 +235,8 @@ def _named(idx):
 
 @pytest.mark.parametrize("idx", [1, 2, 3, 4])
 def test_named_workload_parity(fovea, path, idx):
+    if path == "fused" and workloads.WORKLOADS[idx].dtype != "bf16":
+        pytest.skip("the persistent step kernel covers bf16 calls only")
     w, s, orc, mem = _named(idx)
     gpu = run_gpu(s, fovea)
     mirror = w.dtype == "bf16"
