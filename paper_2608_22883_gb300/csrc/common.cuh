@@ -117,6 +117,8 @@ struct GemmArgs {
   KeyFix* fix_list; int* fix_count; int fix_cap;   // kEpiStoreKeys
   int splits;         // tensor-core path: CTAs of a cluster sharing one output tile (split K)
   int stages;         // tensor-core path: depth of the shared-memory ring
+  int tx_bytes;       // tensor-core path: bytes one ring stage receives (row box + feature tile)
+  int region;         // tensor-core path: bytes of the ring / partial-tile staging region
   float* partials;    // tensor-core split K: fp32 partial tiles (scratch)
   long long partials_floats;
   int* tile_sync;     // tensor-core split K: per tile {arrivals, departures}, zero between launches
@@ -206,8 +208,10 @@ struct TmaOperand {     // a row-major [rows, cols] bf16 matrix with a row strid
 // the fp32 scratch (partial tiles) that split needs.
 struct GemmPlan {
   int bn, splits, stages;
-  long long partial_floats;
-  long long tiles;       // output tiles of a split-K launch (counter pairs it needs)
+  long long partial_floats;   // global fp32 scratch the launch needs (0: none)
+  long long tiles;            // output tiles
+  int rbox;                   // rows of a row-operand load (<= 128)
+  int region;                 // bytes of the ring / partial-tile staging region
 };
 GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n);
 // Tensor map of a row-major [rows, cols] bf16 matrix (row stride ld

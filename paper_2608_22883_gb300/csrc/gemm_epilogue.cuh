@@ -34,4 +34,76 @@ __device__ __forceinline__ void gemm_epilogue(const GemmArgs& a, const GemmGroup
   }
 }
 
+// Epilogue of four consecutive columns m .. m+3 (nv <= 4 of them in range) of
+// output row n: one 8-byte (bf16) or 16-byte (fp32) store per output array
+// where the four are contiguous and aligned, else per element.
+template <int EPI>
+__device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGroup& g, int m, int n,
+                                               const float (&v)[4], int nv) {
+  typedef __nv_bfloat16 T;
+  const long long row = (long long)g.b_row0 + n;
+  bool vec = nv == 4;
+  if constexpr (EPI == kEpiStore || EPI == kEpiBiasSilu)
+    vec = vec && (m + 3 < a.epi_split || m >= a.epi_split);
+  if constexpr (EPI == kEpiScores) {
+    const long long o = g.c_off + (long long)n * g.m + m;
+    if (vec && (o & 3) == 0) {
+      const float rs = a.row_scale ? a.row_scale[g.b_row0 + n] : 1.0f;
+      *reinterpret_cast<float4*>(static_cast<float*>(a.out0) + o) =
+          make_float4(v[0] * a.scale * rs, v[1] * a.scale * rs, v[2] * a.scale * rs,
+                      v[3] * a.scale * rs);
+      return;
+    }
+  } else if constexpr (EPI == kEpiBiasF32) {
+    const long long o = row * a.ldc + m;
+    if (vec && (o & 3) == 0) {
+      const T* b = static_cast<const T*>(a.bias0) + m;
+      *reinterpret_cast<float4*>(static_cast<float*>(a.out0) + o) =
+          make_float4(v[0] + to_f32(b[0]), v[1] + to_f32(b[1]), v[2] + to_f32(b[2]),
+                      v[3] + to_f32(b[3]));
+      return;
+    }
+  } else if constexpr (EPI == kEpiStoreHiLo) {
+    const long long o = row * a.ldc + m;
+    if (vec && (o & 3) == 0) {
+      T hi[4], lo[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        hi[j] = from_f32<T>(v[j]);
+        lo[j] = from_f32<T>(v[j] - to_f32(hi[j]));
+      }
+      *reinterpret_cast<uint2*>(static_cast<T*>(a.out0) + o) = *reinterpret_cast<const uint2*>(hi);
+      *reinterpret_cast<uint2*>(static_cast<T*>(a.out1) + o) = *reinterpret_cast<const uint2*>(lo);
+      return;
+    }
+  } else if constexpr (EPI == kEpiBiasSilu) {
+    const long long o = row * a.ldc + m;
+    if (vec && (o & 3) == 0) {
+      const T* b = m < a.epi_split ? static_cast<const T*>(a.bias0) + m
+                                   : static_cast<const T*>(a.bias1) + (m - a.epi_split);
+      T r[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float z = v[j] + to_f32(b[j]);
+        r[j] = from_f32<T>(z * sigmoidf_(z));
+      }
+      *reinterpret_cast<uint2*>(static_cast<T*>(a.out0) + o) = *reinterpret_cast<const uint2*>(r);
+      return;
+    }
+  } else if constexpr (EPI == kEpiStore) {
+    const long long o = m < a.epi_split ? row * a.ldc + m : row * a.ldc + (m - a.epi_split);
+    if (vec && (o & 3) == 0) {
+      T r[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) r[j] = from_f32<T>(v[j]);
+      T* out = m < a.epi_split ? static_cast<T*>(a.out0) : static_cast<T*>(a.out1);
+      *reinterpret_cast<uint2*>(out + o) = *reinterpret_cast<const uint2*>(r);
+      return;
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (j < nv) gemm_epilogue<T, EPI>(a, g, m + j, n, v[j]);
+}
+
 }  // namespace fovea

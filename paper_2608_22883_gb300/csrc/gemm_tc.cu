@@ -26,14 +26,13 @@
 // the CTA unwinds.
 //
 // Split K: when the output tiles cannot fill the GPU (a 64-row batch against
-// a weight matrix), S CTAs share one output tile, each contracting a slice of
-// K and writing its fp32 partial tile (column-major, so the 32 rows a warp
-// holds land in one 128-byte line) to global scratch.  The grid is a
-// cooperative launch, so all its CTAs are resident together: the S CTAs of a
-// tile meet on a per-tile arrival counter (a bounded spin), then CTA r sums
-// the S partials of columns [r BN/S, (r+1) BN/S) in rank order (so the result
-// does not depend on timing) and runs the epilogue for them.  The last CTA to
-// leave resets the tile's counters for the next launch.
+// a weight matrix), S <= 8 CTAs share one output tile, each contracting a
+// slice of K.  The S CTAs of a tile form a thread-block cluster: each stages
+// its fp32 partial tile row-major in its own shared memory (over the idle
+// stage ring), the cluster synchronises, and CTA r sums the S partials of
+// columns [r BN/S, (r+1) BN/S) in rank order through distributed shared
+// memory (so the result does not depend on timing) and runs the epilogue for
+// them; a second cluster barrier keeps every partial alive until it is read.
 //
 // Launch overlap: kernels are launched with programmatic dependent launch.
 // The producer issues the feature-operand (weight / key) loads of the first
@@ -48,7 +47,7 @@ namespace tc {
 constexpr int BM = 128;          // UMMA M: rows per tile
 constexpr int BK = 64;           // contraction elements per stage (128 bytes bf16)
 constexpr int UMMA_K = 16;       // contraction elements per tcgen05.mma (kind::f16)
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
 constexpr int kSmemBudget = 200 * 1024;   // shared-memory stages, one CTA per SM
 constexpr int kSmemBudgetPair = 100 * 1024;  // two CTAs per SM
 constexpr int kSmemExtra = 1024 /*alignment*/ + 256 /*barriers*/;
@@ -129,7 +128,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                              ~uintptr_t(1023));
   uint8_t* sR = smem;                                  // [stages][R_BYTES]
   uint8_t* sF = smem + stages * C::R_BYTES;            // [stages][F_BYTES]
-  uint64_t* full = reinterpret_cast<uint64_t*>(sF + stages * C::F_BYTES);
+  // barriers after the ring, or after the partial-tile staging area when that
+  // is larger (split K)
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + args.region);
   uint64_t* empty = full + stages;
   uint64_t* accum = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
@@ -169,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // weights / keys of the first stages: independent of the previous kernel
     const int pre = nkb < stages ? nkb : stages;
     for (int i = 0; i < pre; ++i) {
-      mbar_expect_tx(&full[i], C::STAGE_BYTES);
+      mbar_expect_tx(&full[i], (uint32_t)args.tx_bytes);
       tma_load_2d(sF + i * C::F_BYTES, mapF, &full[i], (kb_lo + i) * BK, fy);
     }
     pdl_wait();
@@ -184,7 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           *abort_flag = 1;
           break;
         }
-        mbar_expect_tx(&full[st], C::STAGE_BYTES);
+        mbar_expect_tx(&full[st], (uint32_t)args.tx_bytes);
         tma_load_2d(sF + st * C::F_BYTES, mapF, &full[st], kb * BK, fy);
       }
       if constexpr (DUAL) {
@@ -197,11 +198,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ++issued;
     }
-    if (*abort_flag) {
-      // let copies already in flight land before the CTA gives up its shared memory
-      for (int i = issued > stages ? issued - stages : 0; i < issued; ++i)
-        mbar_wait(&full[i % stages], (uint32_t)(i / stages) & 1u, nullptr, 20000000ull);
-    }
+    // every copy in flight has landed before the ring is reused or the CTA
+    // leaves (in the normal case these stages completed long ago)
+    for (int i = issued > stages ? issued - stages : 0; i < issued; ++i)
+      mbar_wait(&full[i % stages], (uint32_t)(i / stages) & 1u, nullptr, 20000000ull);
   } else if (warp == 1 && lane == 0 && nkb > 0) {
     // ---- MMA issuer (single elected thread) ----
     for (int i = 0; i < nkb; ++i) {
@@ -230,7 +230,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     umma_commit(accum);             // all issued MMAs complete -> accumulator ready
   }
 
-  // ---- epilogue: all warps; thread = one row of the tile ----
+  // ---- epilogue: all eight warps.  Warp w reads accumulator lanes (rows)
+  // 32 (w % 4) .. +31; warps w and w + 4 take the two halves of the columns.
   pdl_wait();
   __syncwarp();
   bool ok = true;
@@ -241,27 +242,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (!ok && lane == 0) atomicOr(args.err, kErrTimeout);
   tc_fence_after();
-  const int row_in_tile = warp * 32 + lane;
+  const int quarter = warp & 3, half = warp >> 2;
+  const int row_in_tile = quarter * 32 + lane;
   const int n = n0 + row_in_tile;
   const bool row_ok = n < g.n;
-  const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16);
+  const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16);
   const int n_cols = min(BN, m_end - m0);
 
-  if (S == 1) {
-    if (ok) {
-      float key_scale = 0.0f;
-      if constexpr (EPI == kEpiStoreKeys) {
-        float ss = 0.0f;
+  if constexpr (EPI == kEpiStoreKeys) {
+    // keys (never split): each thread of warps 0-3 owns one token's row
+    if (ok && half == 0) {
+      float ss = 0.0f;
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 32) {
-          float v[32];
-          tmem_ld32(taddr + (uint32_t)c0, v);
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        float v[32];
+        tmem_ld32(taddr + (uint32_t)c0, v);
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (c0 + j < n_cols) ss = fmaf(v[j], v[j], ss);
-        }
-        key_scale = sqrtf(ss / (float)max(n_cols, 1));
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < n_cols) ss = fmaf(v[j], v[j], ss);
       }
+      const float key_scale = sqrtf(ss / (float)max(n_cols, 1));
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
         if (c0 >= n_cols) break;                    // uniform across the warp
@@ -269,99 +269,89 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32(taddr + (uint32_t)c0, v);
         if (row_ok) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            if (c0 + j < n_cols) {
-              if constexpr (EPI == kEpiStoreKeys) store_key(args, g, m0 + c0 + j, n, v[j], key_scale);
-              else gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + c0 + j, n, v[j]);
-            }
-          }
+          for (int j = 0; j < 32; ++j)
+            if (c0 + j < n_cols) store_key(args, g, m0 + c0 + j, n, v[j], key_scale);
         }
       }
     }
   } else {
-    // ---- split K: partial tiles through global scratch ----
-    const long long tile_id =
-        ((long long)blockIdx.z * gridDim.y + blockIdx.y) * (gridDim.x / S) + tx;
-    float* base = args.partials + tile_id * S * (long long)(BM * BN);   // [S][BN][BM]
-    float* mine = base + (long long)rank * BN * BM;
+    // The accumulator tile goes row-major [rows_real][BN + 4] fp32 into shared
+    // memory over the stage ring (idle: every MMA has completed, every copy
+    // has landed); the pitch of BN + 4 floats spreads a warp's 16-byte stores
+    // over all banks.  Without split K the CTA then writes it out with
+    // consecutive threads on consecutive columns; with split K the S CTAs of
+    // the tile's cluster meet, and CTA `rank` sums columns [rank cpo,
+    // (rank+1) cpo) of the S partial tiles in rank order through distributed
+    // shared memory before writing them.
+    float* part = reinterpret_cast<float*>(smem);
+    const int ldp = BN + 4;
+    const int rows_real = min(BM, g.n - n0);
     const bool have_acc = ok && nkb > 0;          // warp-uniform
+    if (quarter * 32 < rows_real) {               // warp-uniform
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 32) {
-      float v[32];
-      if (have_acc) {
-        tmem_ld32(taddr + (uint32_t)c0, v);       // the whole warp, converged
-      } else {
+      for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+        float v[32];
+        if (have_acc) {
+          tmem_ld32(taddr + (uint32_t)c0, v);     // the whole warp, converged
+        } else {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-      }
-      if (row_ok) {
+          for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+        }
+        if (row_in_tile < rows_real) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) mine[(c0 + j) * BM + row_in_tile] = v[j];
+          for (int q = 0; q < 8; ++q)
+            *reinterpret_cast<float4*>(part + row_in_tile * ldp + c0 + 4 * q) =
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
       }
     }
-    // arrive, then wait (bounded) until the tile's S partials are written
-    __threadfence();
-    __syncthreads();
-    int* arrive = args.tile_sync + 2 * tile_id;
-    __shared__ int s_go;
-    if (threadIdx.x == 0) {
-      atomicAdd(arrive, 1);
-      int go = 1;
-      if (ld_acquire_gpu(arrive) < S) {
-        const uint64_t t0 = globaltimer_ns();
-        while (ld_acquire_gpu(arrive) < S) {
-          if (globaltimer_ns() - t0 > 2000000000ull) {
-            go = 0;
-            atomicOr(args.err, kErrTimeout);
-            break;
+    __syncwarp();
+    if (S > 1) cluster_sync(); else __syncthreads();
+    const int cpo = BN / S;
+    const int q4 = cpo >> 2;
+    const int items = rows_real * q4;
+    // two items per thread and round, all their loads in flight together
+    for (int it0 = threadIdx.x; it0 < items; it0 += 2 * kThreads) {
+      float4 t[2][8];
+      int rr[2], cc[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int it = it0 + k * kThreads;
+        rr[k] = -1;
+        if (it < items) {
+          rr[k] = it / q4;
+          cc[k] = (int)rank * cpo + (it - rr[k] * q4) * 4;
+          const float* src = part + rr[k] * ldp + cc[k];
+          if (S == 1) {
+            t[k][0] = *reinterpret_cast<const float4*>(src);
+          } else {
+            const uint32_t laddr = smem_u32(src);
+#pragma unroll
+            for (int sidx = 0; sidx < 8; ++sidx)
+              if (sidx < S) t[k][sidx] = ld_dsmem_f4(map_dsmem(laddr, (uint32_t)sidx));
           }
         }
       }
-      s_go = go;
-    }
-    __syncthreads();
-    // CTA `rank` owns columns [rank cpo, (rank+1) cpo); work items are
-    // (column, 4 rows); each item issues its S independent loads first, then
-    // sums them in rank order.
-    const int cpo = BN / S;
-    const int rows_real = min(BM, g.n - n0);
-    const int rgroups = (rows_real + 3) / 4;
-    if (ok && s_go) {
-      for (int it = threadIdx.x; it < cpo * rgroups; it += kThreads) {
-        const int cl = it / rgroups;
-        const int r4 = (it - cl * rgroups) * 4;
-        const int col = (int)rank * cpo + cl;
-        if (col >= n_cols) continue;
-        float4 part[16];
 #pragma unroll
-        for (int src = 0; src < 16; ++src)
-          if (src < S)
-            part[src] = __ldcg(reinterpret_cast<const float4*>(
-                base + ((long long)src * BN + col) * BM + r4));
-        float4 acc = part[0];
+      for (int k = 0; k < 2; ++k) {
+        if (rr[k] < 0) continue;
+        float4 acc = t[k][0];
 #pragma unroll
-        for (int src = 1; src < 16; ++src)
-          if (src < S) {
-            acc.x += part[src].x;
-            acc.y += part[src].y;
-            acc.z += part[src].z;
-            acc.w += part[src].w;
+        for (int sidx = 1; sidx < 8; ++sidx)
+          if (sidx < S) {
+            acc.x += t[k][sidx].x;
+            acc.y += t[k][sidx].y;
+            acc.z += t[k][sidx].z;
+            acc.w += t[k][sidx].w;
           }
-        const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (r4 + j < rows_real)
-            gemm_epilogue<__nv_bfloat16, EPI>(args, g, m0 + col, n0 + r4 + j, vals[j]);
+        if (ok && cc[k] < n_cols) {
+          const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+          gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]));
+        }
       }
     }
-    // leave; the last CTA of the tile resets its counters for the next launch
-    __syncthreads();
-    if (threadIdx.x == 0 && s_go) {
-      if (atomicAdd(arrive + 1, 1) == S - 1) {
-        atomicExch(arrive, 0);
-        atomicExch(arrive + 1, 0);
-      }
-    }
+    __syncwarp();
+    if (S > 1) cluster_sync();   // no CTA leaves while another still reads its partial tile
   }
   tc_fence_before();
   __syncthreads();
@@ -444,7 +434,7 @@ static int stages_for(int nkb, int budget) {
   return st < 1 ? 1 : st;
 }
 
-// CTAs of this kernel that can be resident on the GPU at once.
+// CTAs of this kernel resident on the GPU at once.
 template <int BN, int EPI>
 static int resident_ctas(int smem) {
   static int cache[64];      // by smem / 4 KB
@@ -461,27 +451,58 @@ static int resident_ctas(int smem) {
   return cache[mi];
 }
 
+// Clusters of S CTAs of this kernel resident on the GPU at once.
+template <int BN, int EPI>
+static int resident_clusters(int smem, int S) {
+  static int cache[64][4];   // by smem / 4 KB, log2 S
+  const int mi = (smem >> 12) & 63, si = S == 2 ? 1 : S == 4 ? 2 : 3;
+  if (cache[mi][si] != 0) return cache[mi][si];
+  auto kern = tc_kernel<BN, EPI>();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(S, 1, 1);
+  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = -1;                  // cannot be launched with this configuration
+  }
+  cache[mi][si] = n;
+  return n;
+}
+
 template <int BN, int EPI>
 static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tiles_x, int max_n,
-                                  int splits, int stages, cudaStream_t s) {
-  using C = tc::Cfg<BN, EPI == kEpiScores>;
+                                  const GemmPlan& p, cudaStream_t s) {
+  constexpr bool DUAL = EPI == kEpiScores;
   auto kern = tc_kernel<BN, EPI>();
-  a.splits = splits;
-  a.stages = stages;
+  a.splits = p.splits;
+  a.stages = p.stages;
+  a.region = p.region;
+  a.tx_bytes = p.rbox * 128 * (DUAL ? 2 : 1) + BN * 128;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(tiles_x * splits, (max_n + tc::BM - 1) / tc::BM, a.ngroups);
+  cfg.gridDim = dim3(tiles_x * p.splits, (max_n + tc::BM - 1) / tc::BM, a.ngroups);
   cfg.blockDim = dim3(tc::kThreads, 1, 1);
-  cfg.dynamicSmemBytes = stages * C::STAGE_BYTES + tc::kSmemExtra;
+  cfg.dynamicSmemBytes = p.region + tc::kSmemExtra;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (splits > 1) {
-    // the CTAs of a tile wait for one another: the whole grid must be resident
-    attr[1].id = cudaLaunchAttributeCooperative;
-    attr[1].val.cooperative = 1;
+  if (p.splits > 1) {
+    // the S CTAs of an output tile form one cluster
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = p.splits;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
   }
   return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], a);
@@ -491,9 +512,9 @@ template <int EPI>
 static cudaError_t launch_tc_epi(GemmArgs& a, const CUtensorMap* maps, const GemmPlan& p,
                                  int tiles_x, int max_n, cudaStream_t s) {
   switch (p.bn) {
-    case 64: return launch_tc_inst<64, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
-    case 128: return launch_tc_inst<128, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
-    default: return launch_tc_inst<256, EPI>(a, maps, tiles_x, max_n, p.splits, p.stages, s);
+    case 64: return launch_tc_inst<64, EPI>(a, maps, tiles_x, max_n, p, s);
+    case 128: return launch_tc_inst<128, EPI>(a, maps, tiles_x, max_n, p, s);
+    default: return launch_tc_inst<256, EPI>(a, maps, tiles_x, max_n, p, s);
   }
 }
 
@@ -502,31 +523,53 @@ static int feature_tiles(const GemmArgs& a, int max_m, int bn) {
                             : (a.a_split + bn - 1) / bn + (max_m - a.a_split + bn - 1) / bn;
 }
 
+// Issue time of one tcgen05.mma (M = 128, K = 16) by feature-tile width, in
+// cycles, measured on GB300 with back-to-back instructions.
+static int mma_cycles(int bn) { return bn <= 64 ? 50 : bn <= 128 ? 66 : bn <= 192 ? 98 : 129; }
+
+// Estimated time (us) of a plan: the slower of the MMA issue time of a CTA's
+// k-blocks (CTAs sharing an SM share its tensor core) and the load rounds its
+// ring needs (~1.5 us per round of `stages` k-blocks), per wave of resident
+// CTAs, against the feature bytes at HBM speed, plus the split-K tail.
 template <int BN, int EPI>
-static void plan_for(const GemmArgs& a, int max_m, long long row_tiles, GemmPlan& best,
-                     long long& best_score) {
+static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tiles,
+                     GemmPlan& best, double& best_t) {
   constexpr bool DUAL = EPI == kEpiScores;
+  using C = tc::Cfg<BN, DUAL>;
   const int kb_total = a.k_total / tc::BK;
-  const long long tiles = (long long)feature_tiles(a, max_m, BN) * row_tiles;
-  const long long useful = BN < max_m ? BN : max_m;      // real features per tile (bound)
+  const long long ftiles = feature_tiles(a, max_m, BN);
+  const long long tiles = ftiles * row_tiles;
+  const int rows = max_n < tc::BM ? max_n : tc::BM;
+  const int rbox = std::min(tc::BM, (max_n + 7) / 8 * 8);
   const int sms = num_sms();
-  for (int splits = 1; splits <= 16; splits *= 2) {
-    if (splits > 1 && (EPI == kEpiStoreKeys || splits > kb_total || splits > BN)) break;
-    const int nkb = (kb_total + splits - 1) / splits;
-    const long long ctas = tiles * splits;
-    // one CTA per SM while the grid fits on the SMs, else the pair budget
-    int stages = stages_for<BN, DUAL>(nkb, ctas <= sms ? tc::kSmemBudget : tc::kSmemBudgetPair);
-    if (stages < 2 && nkb >= 2) stages = stages_for<BN, DUAL>(nkb, tc::kSmemBudget);
-    const int smem = stages * tc::Cfg<BN, DUAL>::STAGE_BYTES + tc::kSmemExtra;
-    const long long cap = resident_ctas<BN, EPI>(smem);
-    if (splits > 1 && ctas > cap) break;               // a cooperative grid must be resident
-    // weight bytes consumable per MMA time over the CTAs that run at once; a
-    // tie goes to more CTAs (more bytes in flight)
-    const long long run = ctas < sms ? ctas : sms;
-    const long long score = (run * useful) * 4096 + run;
-    if (score > best_score) {
-      best_score = score;
-      best = GemmPlan{BN, splits, stages, 0, 0};
+  const double feat_bytes = (double)ftiles * BN * a.k_total * 2.0 * a.ngroups;
+  for (int S = 1; S <= 8; S *= 2) {
+    if (S > 1 && (EPI == kEpiStoreKeys || S > kb_total)) break;
+    const int nkb = (kb_total + S - 1) / S;
+    const long long ctas = tiles * S;
+    const int staging = EPI == kEpiStoreKeys ? 0 : rows * (BN + 4) * 4;
+    for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
+      const int stages = stages_for<BN, DUAL>(nkb, budget);
+      const int region = std::max(stages * C::STAGE_BYTES, staging);
+      const int smem = region + tc::kSmemExtra;
+      if (region > tc::kSmemBudget) continue;
+      long long cap = resident_ctas<BN, EPI>(smem);
+      if (S > 1) {
+        const int nc = resident_clusters<BN, EPI>(smem, S);
+        if (nc <= 0) continue;
+        cap = std::min<long long>(cap, (long long)nc * S);
+      }
+      if (cap <= 0) continue;
+      const long long waves = (ctas + cap - 1) / cap;
+      const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
+      const double t_mma = nkb * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2000.0 * per_sm;
+      const double t_lat = ((nkb + stages - 1) / stages) * 1.5;
+      const double t_tail = S > 1 ? 1.0 + 0.1 * S : 0.3;
+      const double t = std::max(waves * std::max(t_mma, t_lat), feat_bytes / 6.0e6) + t_tail;
+      if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
+        best_t = t;
+        best = GemmPlan{BN, S, stages, 0, tiles, rbox, region};
+      }
     }
   }
 }
@@ -534,15 +577,11 @@ static void plan_for(const GemmArgs& a, int max_m, long long row_tiles, GemmPlan
 template <int EPI>
 static GemmPlan plan_epi(const GemmArgs& a, int max_m, int max_n) {
   const long long row_tiles = (long long)(max_n + tc::BM - 1) / tc::BM * a.ngroups;
-  GemmPlan best{256, 1, 2, 0, 0};
-  long long best_score = -1;
-  plan_for<256, EPI>(a, max_m, row_tiles, best, best_score);
-  plan_for<128, EPI>(a, max_m, row_tiles, best, best_score);
-  plan_for<64, EPI>(a, max_m, row_tiles, best, best_score);
-  if (best.splits > 1) {
-    best.tiles = (long long)feature_tiles(a, max_m, best.bn) * row_tiles;
-    best.partial_floats = best.tiles * best.splits * tc::BM * best.bn;
-  }
+  GemmPlan best{256, 1, 2, 0, 1 << 30, 128, 0};
+  double best_t = 1e30;
+  plan_for<256, EPI>(a, max_m, max_n, row_tiles, best, best_t);
+  plan_for<128, EPI>(a, max_m, max_n, row_tiles, best, best_t);
+  plan_for<64, EPI>(a, max_m, max_n, row_tiles, best, best_t);
   return best;
 }
 
@@ -564,14 +603,12 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
   static thread_local GemmArgs a;
   a = args;
   const GemmPlan plan = plan_gemm_tc(epi, a, max_m, max_n);
-  if (plan.splits > 1 && (a.partials == nullptr || a.partials_floats < plan.partial_floats ||
-                          a.tile_sync == nullptr || a.tile_sync_tiles < plan.tiles))
-    return cudaErrorInvalidValue;             // the caller sized the scratch with plan_gemm_tc
+  if (plan.region <= 0) return cudaErrorInvalidConfiguration;
   CUtensorMap maps[4];
   const TmaOperand& a1 = A1.base ? A1 : A0;
   const TmaOperand& b1 = B1.base ? B1 : B0;
   if (!make_map(&maps[0], A0, plan.bn) || !make_map(&maps[1], a1, plan.bn) ||
-      !make_map(&maps[2], B0, tc::BM) || !make_map(&maps[3], b1, tc::BM))
+      !make_map(&maps[2], B0, plan.rbox) || !make_map(&maps[3], b1, plan.rbox))
     return cudaErrorInvalidValue;
   const int tiles_x = feature_tiles(a, max_m, plan.bn);
   switch (epi) {
