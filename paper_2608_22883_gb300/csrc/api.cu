@@ -706,6 +706,18 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
+  if (bf) {
+    // the keys (scores, next), and the values when most will be read
+    long long m_sel = 0;
+    for (int b = 0; b < mem->B; ++b)
+      m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
+    a.pf_ptr[a.n_prefetch] = mem->keys;
+    a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+    if (2 * m_sel >= mem->total) {
+      a.pf_ptr[a.n_prefetch] = mem->values;
+      a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+    }
+  }
   { KernelTimer t("query_proj", s);
     e = run_gemm(dt, bf ? kEpiStoreHiLo : kEpiStore, a, TmaOperand{p->W_Q, d, d, d},
                  TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
@@ -732,6 +744,16 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     }
     a.ngroups = g;
     a.dual_b = bf ? 1 : 0;
+    if (bf) {
+      // the fusion weights, read after selection and readout
+      a.pf_ptr[0] = p->W_f1;
+      a.pf_bytes[0] = (long long)H * 2 * d * 2;
+      a.pf_ptr[1] = p->W_g1;
+      a.pf_bytes[1] = (long long)H * 2 * d * 2;
+      a.pf_ptr[2] = p->W_f2;
+      a.pf_bytes[2] = (long long)d * H * 2;
+      a.n_prefetch = 3;
+    }
     { KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
                    TmaOperand{nullptr, 0, 0, 0}, TmaOperand{q, N, d, d},

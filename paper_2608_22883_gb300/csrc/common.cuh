@@ -118,12 +118,19 @@ struct GemmArgs {
   int splits;         // tensor-core path: CTAs of a cluster sharing one output tile (split K)
   int stages;         // tensor-core path: depth of the shared-memory ring
   int tx_bytes;       // tensor-core path: bytes one ring stage receives (row box + feature tile)
+  int kps;            // tensor-core path: k-blocks of 64 per ring stage
+  int rbox;           // tensor-core path: rows of a row-operand tile (64 or 128)
   int region;         // tensor-core path: bytes of the ring / partial-tile staging region
   float* partials;    // tensor-core split K: fp32 partial tiles (scratch)
   long long partials_floats;
   int* tile_sync;     // tensor-core split K: per tile {arrivals, departures}, zero between launches
   long long tile_sync_tiles;
   int* err;
+  // tensor-core path: byte ranges whose share each CTA prefetches into L2 once
+  // it has requested its own operands (data a later kernel of the step reads)
+  int n_prefetch;
+  const void* pf_ptr[4];
+  long long pf_bytes[4];
   int ngroups;
   GemmGroup groups[FOVEA_MAX_SEQ];
 };
@@ -210,8 +217,9 @@ struct GemmPlan {
   int bn, splits, stages;
   long long partial_floats;   // global fp32 scratch the launch needs (0: none)
   long long tiles;            // output tiles
-  int rbox;                   // rows of a row-operand load (<= 128)
+  int rbox;                   // rows of a row-operand load (64 or 128)
   int region;                 // bytes of the ring / partial-tile staging region
+  int kps;                    // k-blocks of 64 per ring stage
 };
 GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n);
 // Tensor map of a row-major [rows, cols] bf16 matrix (row stride ld

@@ -56,13 +56,21 @@ constexpr int kMaxStages = 8;
 // BN features per tile; DUAL: the row stage holds two tiles (hi and lo parts
 // of the row operand), and each feature tile is multiplied by both into the
 // same accumulator.
+//
+// A ring stage holds KPS consecutive k-blocks of 64, loaded with one 3-D TMA
+// box per operand (k within the block, row, k-block), because the TMA engine
+// of an SM costs about the same time per copy for any box up to ~32 KB: few
+// large copies keep the ring fed.  Stage layout: row tiles [KPS][rbox][128 B]
+// (twice for DUAL: hi, then lo), then feature tiles [KPS][BN][128 B].  The MMA
+// reads 128 rows from each row tile's start; rows past rbox (>= 64, so the
+// read stays inside the stage) only feed accumulator rows that are never
+// stored.
 template <int BN, bool DUAL = false>
 struct Cfg {
-  static constexpr int R_TILE = BM * BK * 2;                 // one row tile
-  static constexpr int R_BYTES = R_TILE * (DUAL ? 2 : 1);
-  static constexpr int F_BYTES = BN * BK * 2;                // one feature tile
-  static constexpr int STAGE_BYTES = R_BYTES + F_BYTES;
   static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  __host__ __device__ static constexpr int stage_bytes(int kps, int rbox) {
+    return kps * (rbox * (DUAL ? 2 : 1) + BN) * 128;
+  }
   // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9
   // = 1), B bf16 (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at
   // bits 17-22, M >> 4 at bits 24-28.
@@ -123,11 +131,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (m0 >= m_end || n0 >= g.n) return;
 
   const int stages = args.stages;
+  const int KPS = args.kps, rbox = args.rbox;
+  const int r_tile = rbox * 128;                       // one k-block of the row operand
+  const int r_bytes = KPS * r_tile * (DUAL ? 2 : 1);
+  const int f_tile = BN * 128;                         // one k-block of the feature operand
+  const int stage_bytes = C::stage_bytes(KPS, rbox);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint8_t* sR = smem;                                  // [stages][R_BYTES]
-  uint8_t* sF = smem + stages * C::R_BYTES;            // [stages][F_BYTES]
+  // stage st: row tiles at smem + st * stage_bytes, feature tiles r_bytes later
   // barriers after the ring, or after the partial-tile staging area when that
   // is larger (split K)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + args.region);
@@ -158,9 +170,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int kb_total = args.k_total / BK;
   const int r_split_kb = args.b_split / BK;
-  const int kb_lo = (int)((long long)rank * kb_total / S);
-  const int kb_hi = (int)((long long)(rank + 1) * kb_total / S);
-  const int nkb = kb_hi - kb_lo;
+  const int su_total = kb_total / KPS;                 // stage units (KPS k-blocks each)
+  const int su_lo = (int)((long long)rank * su_total / S);
+  const int su_hi = (int)((long long)(rank + 1) * su_total / S);
+  const int nkb = su_hi - su_lo;                       // stages of this CTA
 
   if (warp == 0 && lane == 0) {
     // ---- TMA producer ----
@@ -171,30 +184,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int pre = nkb < stages ? nkb : stages;
     for (int i = 0; i < pre; ++i) {
       mbar_expect_tx(&full[i], (uint32_t)args.tx_bytes);
-      tma_load_2d(sF + i * C::F_BYTES, mapF, &full[i], (kb_lo + i) * BK, fy);
+      tma_load_3d(smem + i * stage_bytes + r_bytes, mapF, &full[i], 0, fy, (su_lo + i) * KPS);
     }
     pdl_wait();
     pdl_trigger();
     int issued = 0;
     for (int i = 0; i < nkb; ++i) {
-      const int kb = kb_lo + i;
+      const int kb = (su_lo + i) * KPS;
       const int st = i % stages;
       const uint32_t ph = (uint32_t)(i / stages) & 1u;
+      uint8_t* stg = smem + st * stage_bytes;
       if (i >= pre) {
         if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
           *abort_flag = 1;
           break;
         }
         mbar_expect_tx(&full[st], (uint32_t)args.tx_bytes);
-        tma_load_2d(sF + st * C::F_BYTES, mapF, &full[st], kb * BK, fy);
+        tma_load_3d(stg + r_bytes, mapF, &full[st], 0, fy, kb);
       }
       if constexpr (DUAL) {
-        tma_load_2d(sR + st * C::R_BYTES, &tmR0, &full[st], kb * BK, ry);
-        tma_load_2d(sR + st * C::R_BYTES + C::R_TILE, &tmR1, &full[st], kb * BK, ry);
+        tma_load_3d(stg, &tmR0, &full[st], 0, ry, kb);
+        tma_load_3d(stg + KPS * r_tile, &tmR1, &full[st], 0, ry, kb);
       } else {
         const bool r_second = kb >= r_split_kb;
-        tma_load_2d(sR + st * C::R_BYTES, r_second ? &tmR1 : &tmR0, &full[st],
-                    (r_second ? kb - r_split_kb : kb) * BK, ry);
+        tma_load_3d(stg, r_second ? &tmR1 : &tmR0, &full[st], 0, ry,
+                    r_second ? kb - r_split_kb : kb);
       }
       ++issued;
     }
@@ -211,18 +225,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 1;
         break;
       }
-      tc_fence_after();
-      const uint64_t adesc = sw128_desc(smem_u32(sR + st * C::R_BYTES));
-      const uint64_t bdesc = sw128_desc(smem_u32(sF + st * C::F_BYTES));
+      // no tcgen05 fence here: the stage was written by TMA and published by
+      // the mbarrier
+      const uint32_t stg = smem_u32(smem + st * stage_bytes);
+      for (int j = 0; j < KPS; ++j) {
+        const uint64_t adesc = sw128_desc(stg + (uint32_t)(j * r_tile));
+        const uint64_t bdesc = sw128_desc(stg + (uint32_t)(r_bytes + j * f_tile));
 #pragma unroll
-      for (int k = 0; k < BK / UMMA_K; ++k) {
-        // advance the start address by k * 32 bytes inside the swizzle atom
-        umma_bf16(tmem_base, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
-                  (i > 0 || k > 0) ? 1u : 0u);
-        if constexpr (DUAL) {
-          const uint64_t adesc_lo = sw128_desc(smem_u32(sR + st * C::R_BYTES + C::R_TILE));
-          umma_bf16(tmem_base, adesc_lo + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
-                    1u);
+        for (int k = 0; k < BK / UMMA_K; ++k) {
+          // advance the start address by k * 32 bytes inside the swizzle atom
+          umma_bf16(tmem_base, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
+                    (i > 0 || j > 0 || k > 0) ? 1u : 0u);
+          if constexpr (DUAL) {
+            const uint64_t adesc_lo = sw128_desc(stg + (uint32_t)((KPS + j) * r_tile));
+            umma_bf16(tmem_base, adesc_lo + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
+                      1u);
+          }
         }
       }
       umma_commit(&empty[st]);      // frees this stage once its MMAs have read it
@@ -397,6 +415,23 @@ static bool make_map(CUtensorMap* m, const TmaOperand& op, int box_rows) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// [rows, cols] bf16 (row stride ld elements, cols a multiple of 64) viewed as
+// (64 k, rows, cols / 64 k-blocks); box = 64 x box_rows x kps: kps
+// consecutive k-blocks of box_rows rows per copy, one 128-byte-swizzled
+// [box_rows][128 B] tile per k-block in shared memory.
+static bool make_map3(CUtensorMap* m, const TmaOperand& op, int box_rows, int kps) {
+  EncodeTiledFn enc = encoder();
+  if (enc == nullptr || op.base == nullptr || op.rows <= 0 || op.cols <= 0 || op.cols % 64 != 0)
+    return false;
+  cuuint64_t dims[3] = {64, (cuuint64_t)op.rows, (cuuint64_t)(op.cols / 64)};
+  cuuint64_t strides[2] = {(cuuint64_t)op.ld * 2, 128};
+  cuuint32_t box[3] = {64, (cuuint32_t)box_rows, (cuuint32_t)kps};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(op.base), dims, strides, box,
+             es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool encode_bf16_map(CUtensorMap* m, const void* base, long long rows, long long cols,
                      long long ld, int box_rows) {
   return make_map(m, TmaOperand{base, rows, cols, ld}, box_rows);
@@ -426,9 +461,9 @@ static auto tc_kernel() {
 }
 
 template <int BN, bool DUAL>
-static int stages_for(int nkb, int budget) {
+static int stages_for(int nkb, int budget, int kps, int rbox) {
   using C = tc::Cfg<BN, DUAL>;
-  int st = budget / C::STAGE_BYTES;
+  int st = budget / C::stage_bytes(kps, rbox);
   st = st > tc::kMaxStages ? tc::kMaxStages : st;
   st = st > nkb ? nkb : st;
   return st < 1 ? 1 : st;
@@ -486,7 +521,9 @@ static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tile
   a.splits = p.splits;
   a.stages = p.stages;
   a.region = p.region;
-  a.tx_bytes = p.rbox * 128 * (DUAL ? 2 : 1) + BN * 128;
+  a.kps = p.kps;
+  a.rbox = p.rbox;
+  a.tx_bytes = tc::Cfg<BN, DUAL>::stage_bytes(p.kps, p.rbox);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(tiles_x * p.splits, (max_n + tc::BM - 1) / tc::BM, a.ngroups);
   cfg.blockDim = dim3(tc::kThreads, 1, 1);
@@ -527,48 +564,63 @@ static int feature_tiles(const GemmArgs& a, int max_m, int bn) {
 // cycles, measured on GB300 with back-to-back instructions.
 static int mma_cycles(int bn) { return bn <= 64 ? 50 : bn <= 128 ? 66 : bn <= 192 ? 98 : 129; }
 
-// Estimated time (us) of a plan: the slower of the MMA issue time of a CTA's
-// k-blocks (CTAs sharing an SM share its tensor core) and the load rounds its
-// ring needs (~1.5 us per round of `stages` k-blocks), per wave of resident
-// CTAs, against the feature bytes at HBM speed, plus the split-K tail.
+// TMA cost of one copy on an SM, in cycles: about 300 for any box up to
+// ~32 KB, then about 100 bytes per cycle (measured on GB300).
+static double tma_copy_cycles(double bytes) { return std::max(300.0, bytes / 100.0); }
+
+// Estimated time (us) of a plan: per CTA the slowest of its MMA issue time
+// (CTAs sharing an SM share its tensor core), its TMA copy time, and its
+// ring refill rounds (~1.2 us each); per wave of resident CTAs; against the
+// feature bytes at HBM speed; plus the split-K tail.
 template <int BN, int EPI>
 static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tiles,
                      GemmPlan& best, double& best_t) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = tc::Cfg<BN, DUAL>;
   const int kb_total = a.k_total / tc::BK;
+  const int r_split_kb = a.b_split / tc::BK;
   const long long ftiles = feature_tiles(a, max_m, BN);
   const long long tiles = ftiles * row_tiles;
   const int rows = max_n < tc::BM ? max_n : tc::BM;
-  const int rbox = std::min(tc::BM, (max_n + 7) / 8 * 8);
+  // rows of a row tile: >= 64 so that the MMA's 128-row read stays inside its stage
+  const int rbox = std::max(64, std::min(tc::BM, (max_n + 7) / 8 * 8));
   const int sms = num_sms();
   const double feat_bytes = (double)ftiles * BN * a.k_total * 2.0 * a.ngroups;
-  for (int S = 1; S <= 8; S *= 2) {
-    if (S > 1 && (EPI == kEpiStoreKeys || S > kb_total)) break;
-    const int nkb = (kb_total + S - 1) / S;
-    const long long ctas = tiles * S;
-    const int staging = EPI == kEpiStoreKeys ? 0 : rows * (BN + 4) * 4;
-    for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
-      const int stages = stages_for<BN, DUAL>(nkb, budget);
-      const int region = std::max(stages * C::STAGE_BYTES, staging);
-      const int smem = region + tc::kSmemExtra;
-      if (region > tc::kSmemBudget) continue;
-      long long cap = resident_ctas<BN, EPI>(smem);
-      if (S > 1) {
-        const int nc = resident_clusters<BN, EPI>(smem, S);
-        if (nc <= 0) continue;
-        cap = std::min<long long>(cap, (long long)nc * S);
-      }
-      if (cap <= 0) continue;
-      const long long waves = (ctas + cap - 1) / cap;
-      const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
-      const double t_mma = nkb * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2000.0 * per_sm;
-      const double t_lat = ((nkb + stages - 1) / stages) * 1.5;
-      const double t_tail = S > 1 ? 1.0 + 0.1 * S : 0.3;
-      const double t = std::max(waves * std::max(t_mma, t_lat), feat_bytes / 6.0e6) + t_tail;
-      if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
-        best_t = t;
-        best = GemmPlan{BN, S, stages, 0, tiles, rbox, region};
+  for (int kps = 4; kps >= 1; kps >>= 1) {
+    if (kb_total % kps != 0 || r_split_kb % kps != 0) continue;
+    const int su_total = kb_total / kps;
+    const double stage_tma = tma_copy_cycles((double)kps * BN * 128) +
+                             (DUAL ? 2 : 1) * tma_copy_cycles((double)kps * rbox * 128);
+    for (int S = 1; S <= 8; S *= 2) {
+      if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
+      const int nst = (su_total + S - 1) / S;
+      const long long ctas = tiles * S;
+      const int staging = EPI == kEpiStoreKeys ? 0 : rows * (BN + 4) * 4;
+      for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
+        if (C::stage_bytes(kps, rbox) > budget) continue;
+        const int stages = stages_for<BN, DUAL>(nst, budget, kps, rbox);
+        const int region = std::max(stages * C::stage_bytes(kps, rbox), staging);
+        const int smem = region + tc::kSmemExtra;
+        if (region > tc::kSmemBudget) continue;
+        long long cap = resident_ctas<BN, EPI>(smem);
+        if (S > 1) {
+          const int nc = resident_clusters<BN, EPI>(smem, S);
+          if (nc <= 0) continue;
+          cap = std::min<long long>(cap, (long long)nc * S);
+        }
+        if (cap <= 0) continue;
+        const long long waves = (ctas + cap - 1) / cap;
+        const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
+        const double t_mma = (double)nst * kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2000.0 * per_sm;
+        const double t_tma = nst * stage_tma / 2000.0 * per_sm;
+        const double t_lat = ((nst + stages - 1) / stages) * 1.2;
+        const double t_tail = S > 1 ? 1.0 + 0.1 * S : 0.3;
+        const double t = std::max(waves * std::max(std::max(t_mma, t_tma), t_lat),
+                                  feat_bytes / 6.0e6) + t_tail;
+        if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
+          best_t = t;
+          best = GemmPlan{BN, S, stages, 0, tiles, rbox, region, kps};
+        }
       }
     }
   }
@@ -577,7 +629,7 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
 template <int EPI>
 static GemmPlan plan_epi(const GemmArgs& a, int max_m, int max_n) {
   const long long row_tiles = (long long)(max_n + tc::BM - 1) / tc::BM * a.ngroups;
-  GemmPlan best{256, 1, 2, 0, 1 << 30, 128, 0};
+  GemmPlan best{256, 1, 2, 0, 1 << 30, 128, 0, 1};
   double best_t = 1e30;
   plan_for<256, EPI>(a, max_m, max_n, row_tiles, best, best_t);
   plan_for<128, EPI>(a, max_m, max_n, row_tiles, best, best_t);
@@ -607,8 +659,8 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
   CUtensorMap maps[4];
   const TmaOperand& a1 = A1.base ? A1 : A0;
   const TmaOperand& b1 = B1.base ? B1 : B0;
-  if (!make_map(&maps[0], A0, plan.bn) || !make_map(&maps[1], a1, plan.bn) ||
-      !make_map(&maps[2], B0, plan.rbox) || !make_map(&maps[3], b1, plan.rbox))
+  if (!make_map3(&maps[0], A0, plan.bn, plan.kps) || !make_map3(&maps[1], a1, plan.bn, plan.kps) ||
+      !make_map3(&maps[2], B0, plan.rbox, plan.kps) || !make_map3(&maps[3], b1, plan.rbox, plan.kps))
     return cudaErrorInvalidValue;
   const int tiles_x = feature_tiles(a, max_m, plan.bn);
   switch (epi) {

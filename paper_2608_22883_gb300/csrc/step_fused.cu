@@ -364,7 +364,8 @@ __device__ void mma_issuer(const FusedArgs& a, uint8_t* ring, uint64_t* full, ui
           ok = false;
           break;
         }
-        tc_fence_after();
+        // (no tcgen05 fence per k-block: the stage is published by TMA through
+        // the mbarrier, and a fence would serialise the MMAs)
         uint8_t* stage = ring + st * kStageBytes;
         const uint64_t adesc = sw128_desc(smem_u32(stage));
         const uint64_t adesc_lo = sw128_desc(smem_u32(stage + kRTile));
