@@ -36,10 +36,11 @@ __device__ __forceinline__ void gemm_epilogue(const GemmArgs& a, const GemmGroup
 
 // Epilogue of four consecutive columns m .. m+3 (nv <= 4 of them in range) of
 // output row n: one 8-byte (bf16) or 16-byte (fp32) store per output array
-// where the four are contiguous and aligned, else per element.
+// where the four are contiguous and aligned, else per element.  bias4 holds
+// the four columns' biases (bias epilogues, vector case).
 template <int EPI>
 __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGroup& g, int m, int n,
-                                               const float (&v)[4], int nv) {
+                                               const float (&v)[4], int nv, const float* bias4) {
   typedef __nv_bfloat16 T;
   const long long row = (long long)g.b_row0 + n;
   bool vec = nv == 4;
@@ -57,10 +58,8 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
   } else if constexpr (EPI == kEpiBiasF32) {
     const long long o = row * a.ldc + m;
     if (vec && (o & 3) == 0) {
-      const T* b = static_cast<const T*>(a.bias0) + m;
       *reinterpret_cast<float4*>(static_cast<float*>(a.out0) + o) =
-          make_float4(v[0] + to_f32(b[0]), v[1] + to_f32(b[1]), v[2] + to_f32(b[2]),
-                      v[3] + to_f32(b[3]));
+          make_float4(v[0] + bias4[0], v[1] + bias4[1], v[2] + bias4[2], v[3] + bias4[3]);
       return;
     }
   } else if constexpr (EPI == kEpiStoreHiLo) {
@@ -79,12 +78,10 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
   } else if constexpr (EPI == kEpiBiasSilu) {
     const long long o = row * a.ldc + m;
     if (vec && (o & 3) == 0) {
-      const T* b = m < a.epi_split ? static_cast<const T*>(a.bias0) + m
-                                   : static_cast<const T*>(a.bias1) + (m - a.epi_split);
       T r[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const float z = v[j] + to_f32(b[j]);
+        const float z = v[j] + bias4[j];
         r[j] = from_f32<T>(z * sigmoidf_(z));
       }
       *reinterpret_cast<uint2*>(static_cast<T*>(a.out0) + o) = *reinterpret_cast<const uint2*>(r);

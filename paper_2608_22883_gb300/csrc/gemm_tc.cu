@@ -50,7 +50,7 @@ constexpr int UMMA_K = 16;       // contraction elements per tcgen05.mma (kind::
 constexpr int kThreads = 256;
 constexpr int kSmemBudget = 200 * 1024;   // shared-memory stages, one CTA per SM
 constexpr int kSmemBudgetPair = 100 * 1024;  // two CTAs per SM
-constexpr int kSmemExtra = 1024 /*alignment*/ + 256 /*barriers*/;
+constexpr int kSmemExtra = 1024 /*alignment*/ + 256 /*barriers*/ + 1024 /*tile biases*/;
 constexpr int kMaxStages = 8;
 
 // BN features per tile; DUAL: the row stage holds two tiles (hi and lo parts
@@ -147,6 +147,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* accum = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* bias_s = reinterpret_cast<float*>(smem + args.region + 256);   // [BN] tile biases
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -250,6 +251,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- epilogue: all eight warps.  Warp w reads accumulator lanes (rows)
   // 32 (w % 4) .. +31; warps w and w + 4 take the two halves of the columns.
+  if constexpr (EPI == kEpiBiasSilu || EPI == kEpiBiasF32) {
+    // the tile's biases (weights: independent of the predecessor), fetched by
+    // warps 2-7 while the accumulator is produced
+    typedef __nv_bfloat16 Tb;
+    for (int c = (int)threadIdx.x - 64; c < BN; c += kThreads - 64) {
+      if (c < 0) continue;
+      const int m = m0 + c;
+      float b = 0.0f;
+      if (m < m_end) {
+        if (EPI == kEpiBiasSilu && m >= args.epi_split)
+          b = to_f32(static_cast<const Tb*>(args.bias1)[m - args.epi_split]);
+        else
+          b = to_f32(static_cast<const Tb*>(args.bias0)[m]);
+      }
+      bias_s[c] = b;
+    }
+  }
   pdl_wait();
   __syncwarp();
   bool ok = true;
@@ -364,7 +382,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         if (ok && cc[k] < n_cols) {
           const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
-          gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]));
+          gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
+                              bias_s + cc[k]);
         }
       }
     }
@@ -570,7 +589,8 @@ static double tma_copy_cycles(double bytes) { return std::max(300.0, bytes / 100
 
 // Estimated time (us) of a plan: per CTA the slowest of its MMA issue time
 // (CTAs sharing an SM share its tensor core), its TMA copy time, and its
-// ring refill rounds (~1.2 us each); per wave of resident CTAs; against the
+// ring refills (a stage comes back ~2 us after its copy is issued); per wave
+// of resident CTAs; against the
 // feature bytes at HBM speed; plus the split-K tail.
 template <int BN, int EPI>
 static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tiles,
@@ -613,7 +633,7 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
         const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
         const double t_mma = (double)nst * kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2000.0 * per_sm;
         const double t_tma = nst * stage_tma / 2000.0 * per_sm;
-        const double t_lat = ((nst + stages - 1) / stages) * 1.2;
+        const double t_lat = (double)nst * 2.0 / stages;
         const double t_tail = S > 1 ? 1.0 + 0.1 * S : 0.3;
         const double t = std::max(waves * std::max(std::max(t_mma, t_tma), t_lat),
                                   feat_bytes / 6.0e6) + t_tail;
