@@ -18,12 +18,14 @@
 // tensor memory (lane = row, column = feature) and are read back with
 // tcgen05.ld: each epilogue thread owns one row and its BN features.
 //
-// Roles (128 threads): warp 0 lane 0 issues TMA loads into a ring of shared
-// memory stages, warp 1 owns the tensor-memory allocation and its lane 0
-// issues the MMAs (one elected thread), and all four warps run the epilogue:
-// warp w reads accumulator lanes (rows) 32w..32w+31.  Every mbarrier wait is
-// bounded (~2 s); a wait that gives up sets kErrTimeout in the error word and
-// the CTA unwinds.
+// Roles (256 threads): lanes of warp 0 issue the TMA loads into a ring of
+// shared-memory stages (lane 0 the feature tiles, lane 1 the row tiles, lane
+// 2 the lo row tiles of the scores: the copies one thread issues complete one
+// after another, so each operand gets its own issuing lane), warp 1 owns the
+// tensor-memory allocation and its lane 0 issues the MMAs (one elected
+// thread), and all eight warps run the epilogue: warp w reads accumulator
+// lanes (rows) 32 (w % 4) .. +31.  Every mbarrier wait is bounded (~2 s); a
+// wait that gives up sets kErrTimeout in the error word and the CTA unwinds.
 //
 // Split K: when the output tiles cannot fill the GPU (a 64-row batch against
 // a weight matrix), S <= 8 CTAs share one output tile, each contracting a
@@ -58,9 +60,9 @@ constexpr int kMaxStages = 8;
 // same accumulator.
 //
 // A ring stage holds KPS consecutive k-blocks of 64, loaded with one 3-D TMA
-// box per operand (k within the block, row, k-block), because the TMA engine
-// of an SM costs about the same time per copy for any box up to ~32 KB: few
-// large copies keep the ring fed.  Stage layout: row tiles [KPS][rbox][128 B]
+// box per operand (k within the block, row, k-block), because a copy costs
+// its issuing thread about the same time for any box up to 64 KB: few large
+// copies keep the ring fed.  Stage layout: row tiles [KPS][rbox][128 B]
 // (twice for DUAL: hi, then lo), then feature tiles [KPS][BN][128 B].  The MMA
 // reads 128 rows from each row tile's start; rows past rbox (>= 64, so the
 // read stays inside the stage) only feed accumulator rows that are never
@@ -112,6 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ GemmArgs args) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = Cfg<BN, DUAL>;
+  constexpr int kProducers = DUAL ? 3 : 2;   // TMA-issuing lanes of warp 0
   const int S = args.splits;
   const uint32_t rank = (uint32_t)((int)blockIdx.x % S);
   const GemmGroup& g = args.groups[blockIdx.z];
@@ -152,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int st = 0; st < stages; ++st) {
-      mbar_init(&full[st], 1);
+      mbar_init(&full[st], kProducers);
       mbar_init(&empty[st], 1);
     }
     mbar_init(accum, 1);
@@ -176,15 +179,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int su_hi = (int)((long long)(rank + 1) * su_total / S);
   const int nkb = su_hi - su_lo;                       // stages of this CTA
 
-  if (warp == 0 && lane == 0) {
-    // ---- TMA producer ----
+  if (warp == 0 && lane < kProducers) {
+    // ---- TMA producers: lane 0 loads the feature tiles, lane 1 the row tiles
+    // (lane 2 the lo row tiles of DUAL).  Each lane posts its own bytes on the
+    // stage's full barrier (initialised with one arrival per producer lane).
+    const uint32_t f_bytes = (uint32_t)(KPS * f_tile);
+    const uint32_t r_lane_bytes = (uint32_t)(KPS * r_tile);
     const CUtensorMap* mapF = f_second ? &tmF1 : &tmF0;
     const int fy = f_second ? m0 - split : g.a_row0 + m0;
     const int ry = g.b_row0 + n0;
     // weights / keys of the first stages: independent of the previous kernel
-    const int pre = nkb < stages ? nkb : stages;
+    const int pre = lane == 0 ? (nkb < stages ? nkb : stages) : 0;
     for (int i = 0; i < pre; ++i) {
-      mbar_expect_tx(&full[i], (uint32_t)args.tx_bytes);
+      mbar_expect_tx(&full[i], f_bytes);
       tma_load_3d(smem + i * stage_bytes + r_bytes, mapF, &full[i], 0, fy, (su_lo + i) * KPS);
     }
     pdl_wait();
@@ -200,16 +207,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           *abort_flag = 1;
           break;
         }
-        mbar_expect_tx(&full[st], (uint32_t)args.tx_bytes);
-        tma_load_3d(stg + r_bytes, mapF, &full[st], 0, fy, kb);
-      }
-      if constexpr (DUAL) {
-        tma_load_3d(stg, &tmR0, &full[st], 0, ry, kb);
-        tma_load_3d(stg + KPS * r_tile, &tmR1, &full[st], 0, ry, kb);
-      } else {
-        const bool r_second = kb >= r_split_kb;
-        tma_load_3d(stg, r_second ? &tmR1 : &tmR0, &full[st], 0, ry,
-                    r_second ? kb - r_split_kb : kb);
+        if (lane == 0) {
+          mbar_expect_tx(&full[st], f_bytes);
+          tma_load_3d(stg + r_bytes, mapF, &full[st], 0, fy, kb);
+        } else {
+          mbar_expect_tx(&full[st], r_lane_bytes);
+          if constexpr (DUAL) {
+            if (lane == 1)
+              tma_load_3d(stg, &tmR0, &full[st], 0, ry, kb);
+            else
+              tma_load_3d(stg + KPS * r_tile, &tmR1, &full[st], 0, ry, kb);
+          } else {
+            const bool r_second = kb >= r_split_kb;
+            tma_load_3d(stg, r_second ? &tmR1 : &tmR0, &full[st], 0, ry,
+                        r_second ? kb - r_split_kb : kb);
+          }
+        }
       }
       ++issued;
     }
@@ -583,15 +596,35 @@ static int feature_tiles(const GemmArgs& a, int max_m, int bn) {
 // cycles, measured on GB300 with back-to-back instructions.
 static int mma_cycles(int bn) { return bn <= 64 ? 50 : bn <= 128 ? 66 : bn <= 192 ? 98 : 129; }
 
-// TMA cost of one copy on an SM, in cycles: about 300 for any box up to
-// ~32 KB, then about 100 bytes per cycle (measured on GB300).
-static double tma_copy_cycles(double bytes) { return std::max(300.0, bytes / 100.0); }
+// Estimated time (us) of a plan, fitted to stage timings measured on GB300
+// (per-CTA globaltimer stamps over the draft-step GEMMs, cold L2):
+//   first   the first stage lands: ~0.8 us plus the first stages of all CTAs
+//           at the HBM rate (~7 TB/s);
+//   stage   when the feature operand streams from HBM (one row tile per
+//           group: every feature byte is read once), a ring stage costs
+//           ~0.45 us plus ~7.5 ns per KB (a producer lane lands about one
+//           copy at a time from HBM); when row tiles share the feature
+//           operand through L2, ~0.31 us plus the stage at ~200 KB/us.  At
+//           least the MMAs it feeds and the feature bytes of all CTAs'
+//           stages at the HBM rate; with a one-stage ring the copies and the
+//           MMAs do not overlap;
+//   tail    epilogue: ~2 us, plus the cluster reduction for split K
+//           (~2.4 us + 0.25 us per CTA of the cluster);
+// per wave of resident CTAs.
+static double plan_cost_us(bool streaming, double stage_kb, double stage_f_bytes, double mma_us,
+                           int stages, int nst, long long ctas_resident, int per_sm, long long waves,
+                           int S) {
+  const double hbm = 7.0e6;                        // bytes per us
+  const double all_f = (double)ctas_resident * stage_f_bytes / hbm;
+  const double t_copy = streaming ? 0.45 + 0.0075 * stage_kb : 0.31 + stage_kb / 200.0;
+  double t_stage = std::max(t_copy, mma_us) * per_sm;
+  if (stages == 1) t_stage += mma_us;
+  t_stage = std::max(t_stage, all_f);
+  const double t_first = 0.8 + all_f;
+  const double t_tail = S == 1 ? 2.0 : 2.4 + 0.25 * S;
+  return waves * (t_first + nst * t_stage) + t_tail;
+}
 
-// Estimated time (us) of a plan: per CTA the slowest of its MMA issue time
-// (CTAs sharing an SM share its tensor core), its TMA copy time, and its
-// ring refills (a stage comes back ~2 us after its copy is issued); per wave
-// of resident CTAs; against the
-// feature bytes at HBM speed; plus the split-K tail.
 template <int BN, int EPI>
 static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tiles,
                      GemmPlan& best, double& best_t) {
@@ -605,12 +638,12 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
   // rows of a row tile: >= 64 so that the MMA's 128-row read stays inside its stage
   const int rbox = std::max(64, std::min(tc::BM, (max_n + 7) / 8 * 8));
   const int sms = num_sms();
-  const double feat_bytes = (double)ftiles * BN * a.k_total * 2.0 * a.ngroups;
+  const bool streaming = max_n <= tc::BM;             // one row tile per group
   for (int kps = 4; kps >= 1; kps >>= 1) {
     if (kb_total % kps != 0 || r_split_kb % kps != 0) continue;
     const int su_total = kb_total / kps;
-    const double stage_tma = tma_copy_cycles((double)kps * BN * 128) +
-                             (DUAL ? 2 : 1) * tma_copy_cycles((double)kps * rbox * 128);
+    const double stage_f = (double)kps * BN * 128;
+    const double stage_mma_us = (double)kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2070.0;
     for (int S = 1; S <= 8; S *= 2) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
       const int nst = (su_total + S - 1) / S;
@@ -631,12 +664,9 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
         if (cap <= 0) continue;
         const long long waves = (ctas + cap - 1) / cap;
         const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
-        const double t_mma = (double)nst * kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2000.0 * per_sm;
-        const double t_tma = nst * stage_tma / 2000.0 * per_sm;
-        const double t_lat = (double)nst * 2.0 / stages;
-        const double t_tail = S > 1 ? 1.0 + 0.1 * S : 0.3;
-        const double t = std::max(waves * std::max(std::max(t_mma, t_tma), t_lat),
-                                  feat_bytes / 6.0e6) + t_tail;
+        const double t = plan_cost_us(streaming, C::stage_bytes(kps, rbox) / 1024.0, stage_f,
+                                      stage_mma_us, stages, nst, std::min(ctas, cap), (int)per_sm,
+                                      waves, S);
         if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
           best_t = t;
           best = GemmPlan{BN, S, stages, 0, tiles, rbox, region, kps};
