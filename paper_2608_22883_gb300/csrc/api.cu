@@ -124,6 +124,14 @@ struct fovea_memory {
   int32_t* orig_index = nullptr;     // [total]
   int* err = nullptr;                // device error word
   int refined = 0;                   // key elements re-rounded exactly at build
+  // bf16: the values projected through the r-half of the first fusion layer,
+  // p_i = [W_f1 ; W_g1][:, d:2d] u_i  ([total, 2H]), and the weights they
+  // were built with (a call with other W_f1 / W_g1 pointers or H does not
+  // use them)
+  void* proj = nullptr;
+  const void* proj_wf1 = nullptr;
+  const void* proj_wg1 = nullptr;
+  int proj_h = 0;
 };
 
 static size_t esize(int dtype) { return dtype == FOVEA_BF16 ? 2 : 4; }
@@ -195,6 +203,7 @@ static void free_memory(fovea_memory* m) {
   if (m == nullptr) return;
   cudaFree(m->keys);
   cudaFree(m->values);
+  cudaFree(m->proj);
   cudaFree(m->orig_index);
   cudaFree(m->err);
   delete m;
@@ -211,6 +220,7 @@ static cudaError_t run_gemm(int dtype, int epi, const GemmArgs& a, const TmaOper
 static void init_args(GemmArgs& a) {
   memset(&a, 0, sizeof(a));
   a.a_split = 0x7fffffff;
+  a.a_split2 = 0x7fffffff;
   a.epi_split = 0x7fffffff;
   a.scale = 1.0f;
 }
@@ -360,6 +370,35 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
         if (err == cudaSuccess) err = cudaStreamSynchronize(s);
         if (err != cudaSuccess) return cuda_fail(err, "refine_keys");
       }
+      // bf16 with the fusion weights given: p_i = [W_f1 ; W_g1]_r u_i, the
+      // first fusion layer's r-half applied to every value once per image
+      const int H = p->mlp_hidden;
+      if (bf && p->W_f1 != nullptr && p->W_g1 != nullptr && H > 0 && H % 128 == 0 &&
+          H <= FOVEA_MAX_H && aligned16(p->W_f1) && aligned16(p->W_g1)) {
+        fovea_status ps = alloc_dev(&m->proj, (size_t)total * 2 * H * 2, "projected values");
+        if (ps != FOVEA_OK) return ps;
+        const __nv_bfloat16* wf1r = static_cast<const __nv_bfloat16*>(p->W_f1) + d;
+        const __nv_bfloat16* wg1r = static_cast<const __nv_bfloat16*>(p->W_g1) + d;
+        GemmArgs pa;
+        init_args(pa);
+        pa.k_total = d;
+        pa.a_split = H;
+        pa.b_split = d;
+        pa.B0 = m->values; pa.ldb0 = d;
+        pa.out0 = m->proj; pa.ldc = 2 * H;
+        pa.err = m->err;
+        pa.ngroups = 1;
+        pa.groups[0] = GemmGroup{0, 2 * H, 0, total, 0};
+        { KernelTimer t("memory_proj_fusion", s);
+          err = launch_gemm_tc(kEpiStore, pa, TmaOperand{wf1r, H, d, 2 * d},
+                               TmaOperand{wg1r, H, d, 2 * d}, TmaOperand{m->values, total, d, d},
+                               TmaOperand{nullptr, 0, 0, 0}, 2 * H, total, s); }
+        if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+        if (err != cudaSuccess) return cuda_fail(err, "fusion projection of the values");
+        m->proj_wf1 = p->W_f1;
+        m->proj_wg1 = p->W_g1;
+        m->proj_h = H;
+      }
       return FOVEA_OK;
     };
     st = run();
@@ -415,7 +454,7 @@ constexpr size_t kWsSyncOffset = 128;
 constexpr long long kTileSyncTiles = (kWsHeaderBytes - 256) / 8;
 
 struct WsLayout {
-  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, partials, total;
+  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, partials, total;
   long long partial_floats;
 };
 
@@ -428,6 +467,7 @@ long long step_partial_floats(int dtype, int d, int H, int N, int ngroups, int m
     memset(a, 0, sizeof(GemmArgs));
     a->k_total = k_total;
     a->a_split = a_split;
+    a->a_split2 = 0x7fffffff;
     a->ngroups = groups;
     return plan_gemm_tc(epi, *a, mm, mn).partial_floats;
   };
@@ -475,6 +515,7 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
   L.r_lo = take((size_t)N * d * es);
   L.act = take((size_t)N * 2 * H * es);
   L.c = take((size_t)N * d * 4);
+  L.gh = take(dtype == FOVEA_BF16 ? (size_t)N * 2 * H * 4 : 0);   // [W_f1 ; W_g1]_h h, fp32
   L.partials = take((size_t)partial_floats * 4);
   L.partial_floats = partial_floats;
   L.total = off;
@@ -627,6 +668,7 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   void* r_lo = ws + L.r_lo;
   void* act = ws + L.act;
   float* cbuf = reinterpret_cast<float*>(ws + L.c);
+  float* gh = reinterpret_cast<float*>(ws + L.gh);
   float* partials = reinterpret_cast<float*>(ws + L.partials);
   int* tile_sync = reinterpret_cast<int*>(ws + L.err + 256);
 
@@ -694,8 +736,14 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if (e != cudaSuccess) return cuda_fail(e, "ln_query");
 
   static thread_local GemmArgs a;
-  // (2) q = W_Q x_h  (bf16 path: stored as q_hi + q_lo)
+  // (2) q = W_Q x_h  (bf16 path: stored as q_hi + q_lo).  With the memory's
+  // projected values valid for these weights, the same launch computes
+  // G_h = [W_f1 ; W_g1]_h h (the h-half of the first fusion layer, fp32):
+  // the r-half then reduces to a weighted sum of projected values (4).
   const bool bf = dt == FOVEA_BF16;
+  const bool use_proj = bf && mem->proj != nullptr && mem->proj_wf1 == p->W_f1 &&
+                        mem->proj_wg1 == p->W_g1 && mem->proj_h == H &&
+                        select_readout_fits(max_m, k_max);
   void* q_lo = bf ? static_cast<void*>(static_cast<uint8_t*>(q) + (size_t)N * d * 2) : nullptr;
   init_args(a);
   a.k_total = d; a.b_split = d;
@@ -706,22 +754,41 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
+  if (use_proj) {
+    a.a_split = d; a.a_split2 = d + H;
+    a.r_by_part = 1;
+    a.epi_split = d;
+    a.out2 = gh; a.ldc2 = 2 * H;
+    a.groups[0] = GemmGroup{0, d + 2 * H, 0, N, 0};
+  }
   if (bf) {
-    // the keys (scores, next), and the values when most will be read
+    // the keys (scores, next), and the projected values and / or the values
+    // when most of their rows will be read
     long long m_sel = 0;
     for (int b = 0; b < mem->B; ++b)
       m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
     a.pf_ptr[a.n_prefetch] = mem->keys;
     a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
     if (2 * m_sel >= mem->total) {
-      a.pf_ptr[a.n_prefetch] = mem->values;
-      a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+      if (use_proj) {
+        a.pf_ptr[a.n_prefetch] = mem->proj;
+        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * 2 * H * 2;
+      }
+      if (!use_proj || readout != nullptr) {
+        a.pf_ptr[a.n_prefetch] = mem->values;
+        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+      }
     }
   }
   { KernelTimer t("query_proj", s);
-    e = run_gemm(dt, bf ? kEpiStoreHiLo : kEpiStore, a, TmaOperand{p->W_Q, d, d, d},
-                 TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
-                 TmaOperand{nullptr, 0, 0, 0}, d, N, s); }
+    if (use_proj)
+      e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{p->W_Q, d, d, d}, TmaOperand{p->W_f1, H, d, 2 * d},
+                         TmaOperand{xh, N, d, d}, TmaOperand{h, N, d, d}, d + 2 * H, N, s,
+                         TmaOperand{p->W_g1, H, d, 2 * d});
+    else
+      e = run_gemm(dt, bf ? kEpiStoreHiLo : kEpiStore, a, TmaOperand{p->W_Q, d, d, d},
+                   TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
+                   TmaOperand{nullptr, 0, 0, 0}, d, N, s); }
   if (e != cudaSuccess) return cuda_fail(e, "query_proj");
 
   // (3) s = q k^T / sqrt(d) (* row_scale), per sequence
@@ -745,14 +812,16 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.ngroups = g;
     a.dual_b = bf ? 1 : 0;
     if (bf) {
-      // the fusion weights, read after selection and readout
-      a.pf_ptr[0] = p->W_f1;
-      a.pf_bytes[0] = (long long)H * 2 * d * 2;
-      a.pf_ptr[1] = p->W_g1;
-      a.pf_bytes[1] = (long long)H * 2 * d * 2;
-      a.pf_ptr[2] = p->W_f2;
-      a.pf_bytes[2] = (long long)d * H * 2;
-      a.n_prefetch = 3;
+      // the fusion weights, read after selection and readout (with the
+      // projected values, only the second correction layer)
+      if (!use_proj) {
+        a.pf_ptr[a.n_prefetch] = p->W_f1;
+        a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
+        a.pf_ptr[a.n_prefetch] = p->W_g1;
+        a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
+      }
+      a.pf_ptr[a.n_prefetch] = p->W_f2;
+      a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
     }
     { KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
@@ -761,37 +830,53 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     if (e != cudaSuccess) return cuda_fail(e, "score");
   }
 
-  // (4) softmax, cumulative-mass cardinality, selected set, renormalised weights
-  { KernelTimer t("select", s);
-    e = launch_select(scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m, counts, indices,
-                      sel_pos, sel_w, sel_cnt, s); }
-  if (e != cudaSuccess) return cuda_fail(e, "select");
+  // (4) softmax, cumulative-mass cardinality, selected set, renormalised weights;
+  // (5) r = sum alpha u; with the projected values, also
+  // (6) [a_f | a_g] = SiLU(G_h + sum alpha p + [b_f1 | b_g1])
+  if (use_proj) {
+    { KernelTimer t("select_fuse", s);
+      e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
+                               counts, indices, mem->values, d, readout, nullptr, mem->proj, H,
+                               gh, p->b_f1, p->b_g1, act, s); }
+    if (e != cudaSuccess) return cuda_fail(e, "select_fuse");
+  } else {
+    if (select_readout_fits(max_m, k_max)) {
+      { KernelTimer t("select_readout", s);
+        e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
+                                 counts, indices, mem->values, d, readout, r_lo, nullptr, H,
+                                 nullptr, nullptr, nullptr, nullptr, s); }
+      if (e != cudaSuccess) return cuda_fail(e, "select_readout");
+    } else {
+      { KernelTimer t("select", s);
+        e = launch_select(scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m, counts, indices,
+                          sel_pos, sel_w, sel_cnt, s); }
+      if (e != cudaSuccess) return cuda_fail(e, "select");
+      { KernelTimer t("readout", s);
+        e = launch_readout(dt, mem->values, sel_cnt, sel_pos, sel_w, N, k_max, d, readout, r_lo, s); }
+      if (e != cudaSuccess) return cuda_fail(e, "readout");
+    }
 
-  // (5) r = sum alpha u
-  { KernelTimer t("readout", s);
-    e = launch_readout(dt, mem->values, sel_cnt, sel_pos, sel_w, N, k_max, d, readout, r_lo, s); }
-  if (e != cudaSuccess) return cuda_fail(e, "readout");
-
-  // (6) [a_f | a_g] = SiLU([h; r] [W_f1 | W_g1]^T + [b_f1 | b_g1])
-  init_args(a);
-  a.k_total = 2 * d;
-  a.a_split = H;
-  a.b_split = d;
-  a.A0 = p->W_f1; a.A1 = p->W_g1; a.lda0 = 2 * d; a.lda1 = 2 * d;
-  a.B0 = h; a.B1 = r_lo; a.ldb0 = d; a.ldb1 = d;
-  a.epi_split = H;
-  a.out0 = act; a.ldc = 2 * H;
-  a.bias0 = p->b_f1; a.bias1 = p->b_g1;
-  a.err = err;
-  a.partials = partials; a.partials_floats = L.partial_floats;
-  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
-  a.ngroups = 1;
-  a.groups[0] = GemmGroup{0, 2 * H, 0, N, 0};
-  { KernelTimer t("fuse_hidden", s);
-    e = run_gemm(dt, kEpiBiasSilu, a, TmaOperand{p->W_f1, H, 2 * d, 2 * d},
-                 TmaOperand{p->W_g1, H, 2 * d, 2 * d}, TmaOperand{h, N, d, d},
-                 TmaOperand{r_lo, N, d, d}, 2 * H, N, s); }
-  if (e != cudaSuccess) return cuda_fail(e, "fuse_hidden");
+    // (6) [a_f | a_g] = SiLU([h; r] [W_f1 | W_g1]^T + [b_f1 | b_g1])
+    init_args(a);
+    a.k_total = 2 * d;
+    a.a_split = H;
+    a.b_split = d;
+    a.A0 = p->W_f1; a.A1 = p->W_g1; a.lda0 = 2 * d; a.lda1 = 2 * d;
+    a.B0 = h; a.B1 = r_lo; a.ldb0 = d; a.ldb1 = d;
+    a.epi_split = H;
+    a.out0 = act; a.ldc = 2 * H;
+    a.bias0 = p->b_f1; a.bias1 = p->b_g1;
+    a.err = err;
+    a.partials = partials; a.partials_floats = L.partial_floats;
+    a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
+    a.ngroups = 1;
+    a.groups[0] = GemmGroup{0, 2 * H, 0, N, 0};
+    { KernelTimer t("fuse_hidden", s);
+      e = run_gemm(dt, kEpiBiasSilu, a, TmaOperand{p->W_f1, H, 2 * d, 2 * d},
+                   TmaOperand{p->W_g1, H, 2 * d, 2 * d}, TmaOperand{h, N, d, d},
+                   TmaOperand{r_lo, N, d, d}, 2 * H, N, s); }
+    if (e != cudaSuccess) return cuda_fail(e, "fuse_hidden");
+  }
 
   // (7) c = a_f W_f2^T + b_f2
   init_args(a);

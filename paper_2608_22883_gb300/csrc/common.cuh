@@ -94,6 +94,8 @@ enum EpiKind : int {
   kEpiStoreHiLo = 4,  // out0 = T(acc), out1 = T(acc - out0): acc carried as two stored values
   kEpiStoreKeys = 5,  // kEpiStore, and columns < epi_split whose acc lies near a bf16
                       // rounding midpoint are listed for an exact recomputation
+  kEpiQueryH = 6,     // columns < epi_split as kEpiStoreHiLo; columns >= epi_split:
+                      // out2 (fp32)[row * ldc2 + col - epi_split] = acc
 };
 
 struct KeyFix {       // one listed key element: memory row, feature
@@ -103,6 +105,8 @@ struct KeyFix {       // one listed key element: memory row, feature
 struct GemmArgs {
   int k_total;        // contraction length (multiple of 64)
   int a_split;        // A rows >= a_split come from A1 (row - a_split)
+  int a_split2;       // tensor-core path: A rows >= a_split2 come from A2 (row - a_split2)
+  int r_by_part;      // tensor-core path: output columns from A1 / A2 read B1 at every k
   int b_split;        // contraction index >= b_split comes from B1 (k - b_split)
   int dual_b;         // tensor-core scores: B0 and B1 are the hi / lo parts of one
                       // operand, both multiplied by the same A tile
@@ -112,6 +116,7 @@ struct GemmArgs {
   // epilogue
   int epi_split;
   void* out0; void* out1; long long ldc;
+  void* out2; long long ldc2;                      // kEpiQueryH
   const void* bias0; const void* bias1;
   const float* row_scale; float scale;
   KeyFix* fix_list; int* fix_count; int fix_cap;   // kEpiStoreKeys
@@ -192,6 +197,17 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
 cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, const int32_t* sel_pos,
                            const float* sel_w, int N, int k_max, int d, float* r_out, void* r_lo,
                            cudaStream_t s);
+// Selection fused with the gathers that consume it (select.cu), for rows of
+// at most 2048 valid entries and k_max <= 256 (select_readout_fits): the
+// readout r (r_out fp32 and / or r_lo, either may be null; U unused when
+// both are) and, when P is given, act = SiLU(Gh + sum_t alpha_t P[pi(t)] +
+// [b_f1 ; b_g1]) over 2H columns.
+bool select_readout_fits(int max_m, int k_max);
+cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable& tab, int N,
+                                 const int32_t* orig_index, float rho, int k_min, int k_max,
+                                 int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
+                                 float* r_out, void* r_lo, const void* P, int H, const float* Gh,
+                                 const void* b_f1, const void* b_g1, void* act, cudaStream_t s);
 // Exact rounding of listed key elements: k = sum_l x[row, l] W[col, l]
 // evaluated in double-float, rounded once to bf16.  list == nullptr refines
 // every element of the [rows, d] key matrix.
@@ -226,8 +242,9 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n);
 // elements), 128-byte swizzle, box = 64 columns x box_rows rows.
 bool encode_bf16_map(CUtensorMap* m, const void* base, long long rows, long long cols,
                      long long ld, int box_rows);
+// A2 (optional): the feature operand of output columns >= a_split2.
 cudaError_t launch_gemm_tc(int epi, const GemmArgs& a, const TmaOperand& A0, const TmaOperand& A1,
                            const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
-                           cudaStream_t s);
+                           cudaStream_t s, const TmaOperand& A2 = TmaOperand{nullptr, 0, 0, 0});
 
 }  // namespace fovea

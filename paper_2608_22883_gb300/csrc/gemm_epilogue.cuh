@@ -23,8 +23,12 @@ __device__ __forceinline__ void gemm_epilogue(const GemmArgs& a, const GemmGroup
                                        : to_f32(static_cast<const T*>(a.bias1)[m - a.epi_split]);
     const float z = acc + bias;
     static_cast<T*>(a.out0)[row * a.ldc + m] = from_f32<T>(z * sigmoidf_(z));
-  } else if constexpr (EPI == kEpiStoreHiLo) {
+  } else if constexpr (EPI == kEpiStoreHiLo || EPI == kEpiQueryH) {
     const long long row = (long long)g.b_row0 + n;
+    if (EPI == kEpiQueryH && m >= a.epi_split) {
+      static_cast<float*>(a.out2)[row * a.ldc2 + (m - a.epi_split)] = acc;
+      return;
+    }
     const T hi = from_f32<T>(acc);
     static_cast<T*>(a.out0)[row * a.ldc + m] = hi;
     static_cast<T*>(a.out1)[row * a.ldc + m] = from_f32<T>(acc - to_f32(hi));
@@ -62,9 +66,16 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
           make_float4(v[0] + bias4[0], v[1] + bias4[1], v[2] + bias4[2], v[3] + bias4[3]);
       return;
     }
-  } else if constexpr (EPI == kEpiStoreHiLo) {
+  } else if constexpr (EPI == kEpiStoreHiLo || EPI == kEpiQueryH) {
+    if (EPI == kEpiQueryH && m >= a.epi_split) {
+      const long long o = row * a.ldc2 + (m - a.epi_split);
+      if (vec && (o & 3) == 0) {
+        *reinterpret_cast<float4*>(static_cast<float*>(a.out2) + o) = make_float4(v[0], v[1], v[2], v[3]);
+        return;
+      }
+    }
     const long long o = row * a.ldc + m;
-    if (vec && (o & 3) == 0) {
+    if (vec && (o & 3) == 0 && (EPI != kEpiQueryH || m + 3 < a.epi_split)) {
       T hi[4], lo[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {

@@ -32,8 +32,8 @@
 // slice of K.  The S CTAs of a tile form a thread-block cluster: each stages
 // its fp32 partial tile row-major in its own shared memory (over the idle
 // stage ring), the cluster synchronises, and CTA r sums the S partials of
-// columns [r BN/S, (r+1) BN/S) in rank order through distributed shared
-// memory (so the result does not depend on timing) and runs the epilogue for
+// column quads [r Q/S, (r+1) Q/S) (Q = BN/4) in rank order through
+// distributed shared memory (so the result does not depend on timing) and runs the epilogue for
 // them; a second cluster barrier keeps every partial alive until it is read.
 //
 // Launch overlap: kernels are launched with programmatic dependent launch.
@@ -110,26 +110,28 @@ __device__ __forceinline__ void store_key(const GemmArgs& a, const GemmGroup& g,
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmF0, const __grid_constant__ CUtensorMap tmF1,
-                   const __grid_constant__ CUtensorMap tmR0, const __grid_constant__ CUtensorMap tmR1,
-                   const __grid_constant__ GemmArgs args) {
+                   const __grid_constant__ CUtensorMap tmF2, const __grid_constant__ CUtensorMap tmR0,
+                   const __grid_constant__ CUtensorMap tmR1, const __grid_constant__ GemmArgs args) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = Cfg<BN, DUAL>;
   constexpr int kProducers = DUAL ? 3 : 2;   // TMA-issuing lanes of warp 0
   const int S = args.splits;
   const uint32_t rank = (uint32_t)((int)blockIdx.x % S);
   const GemmGroup& g = args.groups[blockIdx.z];
-  // Output columns (features) [0, a_split) come from F0 and [a_split, m) from
-  // F1; each part is tiled on its own so no tile straddles the two operands.
-  // A group smaller than the grid leaves its extra tiles idle.  The S CTAs of a
-  // tile share these decisions, so a tile's CTAs exit together.
-  const int split = args.a_split;
-  const bool has_second = split < g.m;
-  const int tiles0 = has_second ? (split + BN - 1) / BN : (g.m + BN - 1) / BN;
+  // Output columns (features) [0, a_split) come from F0, [a_split, a_split2)
+  // from F1 and [a_split2, m) from F2; each part is tiled on its own so no
+  // tile straddles two operands.  A group smaller than the grid leaves its
+  // extra tiles idle.  The S CTAs of a tile share these decisions, so a
+  // tile's CTAs exit together.
+  const int s1 = min(args.a_split, g.m);
+  const int s2 = max(s1, min(args.a_split2, g.m));
+  const int t0 = (s1 + BN - 1) / BN, t1 = (s2 - s1 + BN - 1) / BN, t2 = (g.m - s2 + BN - 1) / BN;
   const int tx = (int)blockIdx.x / S;
-  if (!has_second && tx >= tiles0) return;
-  const bool f_second = has_second && tx >= tiles0;
-  const int m0 = f_second ? split + (tx - tiles0) * BN : tx * BN;
-  const int m_end = f_second ? g.m : min(g.m, split);
+  if (tx >= t0 + t1 + t2) return;
+  const int part = tx < t0 ? 0 : (tx < t0 + t1 ? 1 : 2);
+  const int pbeg = part == 0 ? 0 : (part == 1 ? s1 : s2);
+  const int m0 = pbeg + (tx - (part == 0 ? 0 : (part == 1 ? t0 : t0 + t1))) * BN;
+  const int m_end = part == 0 ? s1 : (part == 1 ? s2 : g.m);
   const int n0 = blockIdx.y * BM;
   if (m0 >= m_end || n0 >= g.n) return;
 
@@ -161,7 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(accum, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    prefetch_tmap(&tmF0);
+    prefetch_tmap(part == 0 ? &tmF0 : (part == 1 ? &tmF1 : &tmF2));
     prefetch_tmap(&tmR0);
   }
   if (warp == 1) {
@@ -185,8 +187,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // stage's full barrier (initialised with one arrival per producer lane).
     const uint32_t f_bytes = (uint32_t)(KPS * f_tile);
     const uint32_t r_lane_bytes = (uint32_t)(KPS * r_tile);
-    const CUtensorMap* mapF = f_second ? &tmF1 : &tmF0;
-    const int fy = f_second ? m0 - split : g.a_row0 + m0;
+    const CUtensorMap* mapF = part == 0 ? &tmF0 : (part == 1 ? &tmF1 : &tmF2);
+    const int fy = part == 0 ? g.a_row0 + m0 : m0 - pbeg;
     const int ry = g.b_row0 + n0;
     // weights / keys of the first stages: independent of the previous kernel
     const int pre = lane == 0 ? (nkb < stages ? nkb : stages) : 0;
@@ -218,9 +220,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             else
               tma_load_3d(stg + KPS * r_tile, &tmR1, &full[st], 0, ry, kb);
           } else {
-            const bool r_second = kb >= r_split_kb;
+            // the row operand: by contraction index (B1 from b_split on),
+            // or by feature part (B1 for the columns of F1 and F2)
+            const bool r_second = args.r_by_part ? part != 0 : kb >= r_split_kb;
             tma_load_3d(stg, r_second ? &tmR1 : &tmR0, &full[st], 0, ry,
-                        r_second ? kb - r_split_kb : kb);
+                        (r_second && !args.r_by_part) ? kb - r_split_kb : kb);
           }
         }
       }
@@ -356,8 +360,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
     if (S > 1) cluster_sync(); else __syncthreads();
-    const int cpo = BN / S;
-    const int q4 = cpo >> 2;
+    // CTA `rank` owns the column quads [qlo, qhi) of the tile
+    const int qlo = (int)rank * (BN / 4) / S, qhi = ((int)rank + 1) * (BN / 4) / S;
+    const int q4 = qhi - qlo;
     const int items = rows_real * q4;
     // two items per thread and round, all their loads in flight together
     for (int it0 = threadIdx.x; it0 < items; it0 += 2 * kThreads) {
@@ -369,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         rr[k] = -1;
         if (it < items) {
           rr[k] = it / q4;
-          cc[k] = (int)rank * cpo + (it - rr[k] * q4) * 4;
+          cc[k] = (qlo + (it - rr[k] * q4)) * 4;
           const float* src = part + rr[k] * ldp + cc[k];
           if (S == 1) {
             t[k][0] = *reinterpret_cast<const float4*>(src);
@@ -521,8 +526,8 @@ static int resident_ctas(int smem) {
 // Clusters of S CTAs of this kernel resident on the GPU at once.
 template <int BN, int EPI>
 static int resident_clusters(int smem, int S) {
-  static int cache[64][4];   // by smem / 4 KB, log2 S
-  const int mi = (smem >> 12) & 63, si = S == 2 ? 1 : S == 4 ? 2 : 3;
+  static int cache[64][9];   // by smem / 4 KB, S
+  const int mi = (smem >> 12) & 63, si = S & 7 ? S : 8;
   if (cache[mi][si] != 0) return cache[mi][si];
   auto kern = tc_kernel<BN, EPI>();
   cudaLaunchConfig_t cfg = {};
@@ -574,7 +579,7 @@ static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tile
     attr[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
   }
-  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], a);
+  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], maps[4], a);
 }
 
 template <int EPI>
@@ -587,9 +592,11 @@ static cudaError_t launch_tc_epi(GemmArgs& a, const CUtensorMap* maps, const Gem
   }
 }
 
+// Feature tiles of the widest group: each operand part is tiled on its own.
 static int feature_tiles(const GemmArgs& a, int max_m, int bn) {
-  return a.a_split >= max_m ? (max_m + bn - 1) / bn
-                            : (a.a_split + bn - 1) / bn + (max_m - a.a_split + bn - 1) / bn;
+  const int s1 = std::min(a.a_split, max_m);
+  const int s2 = std::max(s1, std::min(a.a_split2, max_m));
+  return (s1 + bn - 1) / bn + (s2 - s1 + bn - 1) / bn + (max_m - s2 + bn - 1) / bn;
 }
 
 // Issue time of one tcgen05.mma (M = 128, K = 16) by feature-tile width, in
@@ -644,7 +651,7 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
     const int su_total = kb_total / kps;
     const double stage_f = (double)kps * BN * 128;
     const double stage_mma_us = (double)kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2070.0;
-    for (int S = 1; S <= 8; S *= 2) {
+    for (int S = 1; S <= 8; ++S) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
       const int nst = (su_total + S - 1) / S;
       const long long ctas = tiles * S;
@@ -694,23 +701,26 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
     case kEpiBiasSilu: return plan_epi<kEpiBiasSilu>(a, max_m, max_n);
     case kEpiStoreHiLo: return plan_epi<kEpiStoreHiLo>(a, max_m, max_n);
     case kEpiStoreKeys: return plan_epi<kEpiStoreKeys>(a, max_m, max_n);
+    case kEpiQueryH: return plan_epi<kEpiQueryH>(a, max_m, max_n);
     default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
   }
 }
 
 cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, const TmaOperand& A1,
                            const TmaOperand& B0, const TmaOperand& B1, int max_m, int max_n,
-                           cudaStream_t s) {
+                           cudaStream_t s, const TmaOperand& A2) {
   if (max_m <= 0 || max_n <= 0 || args.ngroups <= 0) return cudaSuccess;
   static thread_local GemmArgs a;
   a = args;
   const GemmPlan plan = plan_gemm_tc(epi, a, max_m, max_n);
   if (plan.region <= 0) return cudaErrorInvalidConfiguration;
-  CUtensorMap maps[4];
+  CUtensorMap maps[5];            // F0, F1, F2, R0, R1
   const TmaOperand& a1 = A1.base ? A1 : A0;
+  const TmaOperand& a2 = A2.base ? A2 : a1;
   const TmaOperand& b1 = B1.base ? B1 : B0;
   if (!make_map3(&maps[0], A0, plan.bn, plan.kps) || !make_map3(&maps[1], a1, plan.bn, plan.kps) ||
-      !make_map3(&maps[2], B0, plan.rbox, plan.kps) || !make_map3(&maps[3], b1, plan.rbox, plan.kps))
+      !make_map3(&maps[2], a2, plan.bn, plan.kps) || !make_map3(&maps[3], B0, plan.rbox, plan.kps) ||
+      !make_map3(&maps[4], b1, plan.rbox, plan.kps))
     return cudaErrorInvalidValue;
   const int tiles_x = feature_tiles(a, max_m, plan.bn);
   switch (epi) {
@@ -719,6 +729,7 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
     case kEpiBiasSilu: return launch_tc_epi<kEpiBiasSilu>(a, maps, plan, tiles_x, max_n, s);
     case kEpiStoreHiLo: return launch_tc_epi<kEpiStoreHiLo>(a, maps, plan, tiles_x, max_n, s);
     case kEpiStoreKeys: return launch_tc_epi<kEpiStoreKeys>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiQueryH: return launch_tc_epi<kEpiQueryH>(a, maps, plan, tiles_x, max_n, s);
     default: return launch_tc_epi<kEpiBiasF32>(a, maps, plan, tiles_x, max_n, s);
   }
 }

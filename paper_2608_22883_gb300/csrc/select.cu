@@ -1,7 +1,12 @@
-// Cumulative-mass selection kernel: one CTA of 256 threads per draft state
-// (the algorithm is in select_core.cuh).  The row's scores are staged in
-// shared memory first.
+// Cumulative-mass selection kernels (the algorithm is in select_core.cuh):
+// the selection alone (one CTA of 256 threads per draft state), and the
+// selection fused with the readout r_n = sum_{t < K} alpha_t u_{pi(t)} (the
+// alpha / r_n equation of the retrieval section).  The row's scores are
+// staged in shared memory first.
+#include <algorithm>
+
 #include "select_core.cuh"
+#include "tc_ptx.cuh"
 
 namespace fovea {
 
@@ -46,8 +51,297 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt};
+  SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt,
+               nullptr, nullptr, nullptr};
   return launch_pdl(select_kernel, dim3(N), dim3(kSelThreads), smem, s, a, tab);
+}
+
+// Selection and the gathers that consume it, in one kernel: one
+// thread-block cluster of C CTAs per draft state n.  CTA rank 0 runs the
+// selection of n into its shared memory; after a cluster barrier the other
+// CTAs copy the selected rows and weights through distributed shared memory,
+// so the selection is computed once and never travels through global memory.
+// CTA y then gathers its column chunks of
+//   the readout     r_n = sum_{t < K} alpha_t u_{pi(t)}          (U, d columns)
+//   the projected readout  sum_t alpha_t p_{pi(t)}, p_i = W_r u_i  (P, 2H columns)
+// whichever the call needs.  The first fusion layer is linear in r_n, so
+// [W_f1 ; W_g1] [h_n ; r_n] = G_h[n] + sum_t alpha_t p_{pi(t)} with
+// G_h = [W_f1 ; W_g1]_h h_n computed beside the query projection; the
+// projected chunk is finished here: act = SiLU(G_h + sum + [b_f1 ; b_g1]).
+// Gathers: the threads own 16-byte column vectors; for a chunk of fewer than
+// 256 vectors, G = 256 / vectors groups of threads split the selected entries
+// (group g takes t = g, g + G, ...), eight gathers in flight per thread, and
+// their partial sums are combined in group order (fixed order, fp32).  CTA
+// rank 0 writes counts and indices.
+constexpr int kRoUnroll = 8;
+static inline size_t align_up_sz(size_t x, size_t a) { return (x + a - 1) / a * a; }
+using tc::cluster_sync;
+using tc::ld_dsmem_f4;
+using tc::map_dsmem;
+using tc::smem_u32;
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ int ld_dsmem_s32(uint32_t caddr) {
+  int v;
+  asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(caddr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+struct GatherArgs {
+  // readout: U [rows, d] -> r_out [N, d] fp32 and / or r_lo [N, d] (either may be null)
+  const void* U;
+  int d, chunk_u;
+  float* r_out;
+  void* r_lo;
+  // projected readout: P [rows, HP] -> act [N, HP] = SiLU(Gh + sum + bias) (P null: none)
+  const void* P;
+  int HP, H, chunk_p;
+  const float* Gh;                  // [N, HP] fp32
+  const void* b_f1;                 // [H]: bias of columns < H
+  const void* b_g1;                 // [H]: bias of columns >= H
+  void* act;                        // [N, HP]
+  int red_floats;                   // dynamic shared memory: scores / gather partial sums
+};
+
+// Weighted gather-sum over the selected rows of X [*, ld], columns
+// [c0, c0 + w) (w a multiple of V): out(vector index, sums) once per 16-byte
+// column vector.  Every thread of the CTA calls it (it may synchronise).
+template <class T, class Out>
+__device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, int w, int K,
+                                             const int32_t* pos, const float* wt, float* red,
+                                             int tid, Out out) {
+  constexpr int V = 16 / (int)sizeof(T);
+  const int nvec = w / V;
+  if (nvec <= 0) return;
+  const int G = nvec >= kSelThreads ? 1 : kSelThreads / nvec;
+  for (int vc0 = 0; vc0 < nvec; vc0 += kSelThreads) {
+    const int g = G > 1 ? tid / nvec : 0;
+    const int vc = G > 1 ? tid - g * nvec : vc0 + tid;
+    float acc[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) acc[i] = 0.0f;
+    if (g < G && vc < nvec) {
+      const T* col = X + c0 + (long long)vc * V;
+      int t = g;
+      for (; t + (kRoUnroll - 1) * G < K; t += kRoUnroll * G) {
+        uint4 raw[kRoUnroll];
+#pragma unroll
+        for (int j = 0; j < kRoUnroll; ++j)
+          raw[j] = __ldg(reinterpret_cast<const uint4*>(col + (long long)pos[t + j * G] * ld));
+#pragma unroll
+        for (int j = 0; j < kRoUnroll; ++j) {
+          const float wj = wt[t + j * G];
+          const T* e = reinterpret_cast<const T*>(&raw[j]);
+#pragma unroll
+          for (int i = 0; i < V; ++i) acc[i] = fmaf(wj, to_f32(e[i]), acc[i]);
+        }
+      }
+      for (; t < K; t += G) {
+        const uint4 raw = __ldg(reinterpret_cast<const uint4*>(col + (long long)pos[t] * ld));
+        const float wj = wt[t];
+        const T* e = reinterpret_cast<const T*>(&raw);
+#pragma unroll
+        for (int i = 0; i < V; ++i) acc[i] = fmaf(wj, to_f32(e[i]), acc[i]);
+      }
+    }
+    if (G > 1) {
+      if (g < G)
+#pragma unroll
+        for (int i = 0; i < V; ++i) red[(g * nvec + vc) * V + i] = acc[i];
+      __syncthreads();
+      if (tid < nvec) {
+#pragma unroll
+        for (int i = 0; i < V; ++i) acc[i] = red[tid * V + i];
+        for (int gg = 1; gg < G; ++gg)
+#pragma unroll
+          for (int i = 0; i < V; ++i) acc[i] += red[(gg * nvec + tid) * V + i];
+        out(tid, acc);
+      }
+      __syncthreads();                    // red is free again
+      break;                              // one pass covers the chunk
+    }
+    if (vc < nvec) out(vc, acc);
+  }
+}
+
+template <class T>
+__global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
+    const __grid_constant__ SelectArgs args, const __grid_constant__ SeqTable tab,
+    const __grid_constant__ GatherArgs ga) {
+  constexpr int V = 16 / (int)sizeof(T);                     // elements per 16-byte vector
+  // dynamic: [red_floats] scores, later gather partial sums | [chunk_p] G_h | [chunk_p] bias
+  extern __shared__ __align__(16) float dyn[];
+  __shared__ SelectSmem sm;
+  __shared__ __align__(16) int32_t loc_pos[kRankMax];
+  __shared__ __align__(16) float loc_w[kRankMax];
+  __shared__ int loc_cnt;
+  const int n = blockIdx.x;
+  const int tid = threadIdx.x;
+  const uint32_t rank = cluster_rank();
+  float* s_sc = dyn;
+  float* gh_s = dyn + ga.red_floats;
+  T* bias_s = reinterpret_cast<T*>(gh_s + ga.chunk_p);
+  pdl_wait();
+  pdl_trigger();
+  // G_h and the biases of this CTA's projected chunk: requested now, used last
+  const int cp0 = blockIdx.y * ga.chunk_p;
+  const int wp = ga.P != nullptr ? max(0, min(ga.chunk_p, ga.HP - cp0)) : 0;
+  for (int q = tid; q < wp / 4; q += kSelThreads)
+    cp_async16(gh_s + 4 * q, ga.Gh + (long long)n * ga.HP + cp0 + 4 * q);
+  for (int q = tid; q < wp / V; q += kSelThreads) {
+    const int c = cp0 + q * V;
+    const T* src = c < ga.H ? static_cast<const T*>(ga.b_f1) + c
+                            : static_cast<const T*>(ga.b_g1) + (c - ga.H);
+    cp_async16(bias_s + q * V, src);
+  }
+  if (rank == 0) {
+    SelectArgs a = args;
+    a.loc_pos = loc_pos;
+    a.loc_w = loc_w;
+    a.loc_cnt = &loc_cnt;
+    const int b = seq_of_row(tab, n);
+    const int M = tab.m[b];
+    if (M == 0) {                         // empty valid set: K = 0, r_n = 0
+      select_empty(a, n, tid);
+    } else {
+      const float* src = a.scores + tab.score_off[b] + (long long)(n - tab.row_start[b]) * M;
+      for (int i = tid; i < M; i += kSelThreads) {
+        float v = src[i];
+        if (v == 0.0f) v = 0.0f;          // -0 -> +0 so equal scores get equal keys
+        s_sc[i] = v;
+      }
+      __syncthreads();
+      select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSync{});
+    }
+  }
+  cluster_sync();                         // rank 0's selection is visible to the cluster
+  if (rank != 0) {
+    const int K = ld_dsmem_s32(map_dsmem(smem_u32(&loc_cnt), 0));
+    for (int q = tid; q < (K + 3) / 4; q += kSelThreads) {
+      const float4 p4 = ld_dsmem_f4(map_dsmem(smem_u32(&loc_pos[4 * q]), 0));
+      const float4 w4 = ld_dsmem_f4(map_dsmem(smem_u32(&loc_w[4 * q]), 0));
+      *reinterpret_cast<float4*>(&loc_pos[4 * q]) = p4;
+      *reinterpret_cast<float4*>(&loc_w[4 * q]) = w4;
+    }
+    if (tid == 0) loc_cnt = K;
+  }
+  cluster_arrive();                       // done reading rank 0 (waited for before exit)
+  cp_async_wait_all();
+  __syncthreads();
+  const int K = loc_cnt;
+  float* red = s_sc;
+  // projected readout -> act = SiLU(G_h + sum + bias)
+  if (wp > 0) {
+    T* act = static_cast<T*>(ga.act) + (long long)n * ga.HP + cp0;
+    gather_chunk<T>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, red, tid,
+                    [&](int vc, const float (&acc)[V]) {
+                      T res[V];
+#pragma unroll
+                      for (int i = 0; i < V; ++i) {
+                        const float z = acc[i] + gh_s[vc * V + i] + to_f32(bias_s[vc * V + i]);
+                        res[i] = from_f32<T>(z * sigmoidf_(z));
+                      }
+                      *reinterpret_cast<uint4*>(act + vc * V) = *reinterpret_cast<const uint4*>(res);
+                    });
+  }
+  // readout r_n
+  const int cu0 = blockIdx.y * ga.chunk_u;
+  const int wu = (ga.r_out != nullptr || ga.r_lo != nullptr) ? max(0, min(ga.chunk_u, ga.d - cu0)) : 0;
+  if (wu > 0) {
+    const long long o = (long long)n * ga.d + cu0;
+    gather_chunk<T>(static_cast<const T*>(ga.U), ga.d, cu0, wu, K, loc_pos, loc_w, red, tid,
+                    [&](int vc, const float (&acc)[V]) {
+                      if (ga.r_out != nullptr) {
+#pragma unroll
+                        for (int i = 0; i < V; i += 4)
+                          *reinterpret_cast<float4*>(ga.r_out + o + vc * V + i) =
+                              make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+                      }
+                      if (ga.r_lo != nullptr) {
+                        T res[V];
+#pragma unroll
+                        for (int i = 0; i < V; ++i) res[i] = from_f32<T>(acc[i]);
+                        *reinterpret_cast<uint4*>(static_cast<T*>(ga.r_lo) + o + vc * V) =
+                            *reinterpret_cast<const uint4*>(res);
+                      }
+                    });
+  }
+  cluster_wait();                         // rank 0 stays until every CTA has copied
+}
+
+bool select_readout_fits(int max_m, int k_max) { return max_m <= kFastMaxM && k_max <= kRankMax; }
+
+cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable& tab, int N,
+                                 const int32_t* orig_index, float rho, int k_min, int k_max,
+                                 int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
+                                 float* r_out, void* r_lo, const void* P, int H, const float* Gh,
+                                 const void* b_f1, const void* b_g1, void* act, cudaStream_t s) {
+  if (N == 0) return cudaSuccess;
+  if (!select_readout_fits(max_m, k_max) || d % 64 != 0 || (P != nullptr && H % 64 != 0))
+    return cudaErrorInvalidValue;
+  // CTAs per row (one cluster): about two per SM in one wave, each chunk a
+  // multiple of 64 columns
+  int sms = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
+  if (e != cudaSuccess) return e;
+  const int HP = 2 * H;
+  int nchunk = 1;
+  while (nchunk < 8 && (long long)N * nchunk * 2 <= 2LL * sms && d % (nchunk * 2 * 64) == 0 &&
+         (P == nullptr || HP % (nchunk * 2 * 64) == 0))
+    nchunk *= 2;
+  const int V = dtype == FOVEA_BF16 ? 8 : 4;
+  GatherArgs ga{};
+  ga.U = U;
+  ga.d = d;
+  ga.chunk_u = d / nchunk;
+  ga.r_out = r_out;
+  ga.r_lo = r_lo;
+  ga.P = P;
+  ga.HP = P != nullptr ? HP : 0;
+  ga.H = H;
+  ga.chunk_p = P != nullptr ? HP / nchunk : 0;
+  ga.Gh = Gh;
+  ga.b_f1 = b_f1;
+  ga.b_g1 = b_g1;
+  ga.act = act;
+  ga.red_floats = (int)align_up_sz((size_t)std::max(std::max(max_m, 1), kSelThreads * V), 4);
+  const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
+  const size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
+                      align_up_sz((size_t)ga.chunk_p * es, 16);
+  if (smem > 48 * 1024) return cudaErrorInvalidValue;
+  SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices,
+               nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(N, nchunk);
+  cfg.blockDim = dim3(kSelThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;   // the chunks of one row form a cluster
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = nchunk;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (dtype == FOVEA_BF16)
+    return cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16>, a, tab, ga);
+  return cudaLaunchKernelEx(&cfg, select_gather_kernel<float>, a, tab, ga);
 }
 
 }  // namespace fovea

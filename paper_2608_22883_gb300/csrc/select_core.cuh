@@ -43,9 +43,14 @@ struct SelectArgs {
   int k_min, k_max;
   int32_t* counts;     // [N] or null
   int32_t* indices;    // [N, k_max] or null
-  int32_t* sel_pos;    // [N, k_max] compacted memory row of each selected entry
-  float* sel_w;        // [N, k_max] renormalised weight alpha
-  int32_t* sel_cnt;    // [N]
+  int32_t* sel_pos;    // [N, k_max] compacted memory row of each selected entry, or null
+  float* sel_w;        // [N, k_max] renormalised weight alpha, or null
+  int32_t* sel_cnt;    // [N] or null
+  // the same selection for the calling group alone (shared memory, entry t at
+  // [t]; K <= kRankMax when used), or null
+  int32_t* loc_pos;
+  float* loc_w;
+  int* loc_cnt;
 };
 
 struct SelectSmem {
@@ -289,29 +294,36 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
       const int pos = (int)(0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull));
       const float e = expf(s_sc[pos] - smax);
       const int row = key_off + pos;
-      a.sel_pos[out_row + t] = row;
-      a.sel_w[out_row + t] = e / denom;
+      if (a.sel_pos) a.sel_pos[out_row + t] = row;
+      if (a.sel_w) a.sel_w[out_row + t] = e / denom;
+      if (a.loc_pos) {
+        a.loc_pos[t] = row;
+        a.loc_w[t] = e / denom;
+      }
       if (a.indices) a.indices[out_row + t] = a.orig_index[row];
     } else if (a.indices) {
       a.indices[out_row + t] = -1;
     }
   }
   if (tid == 0) {
-    a.sel_cnt[n] = K;
+    if (a.sel_cnt) a.sel_cnt[n] = K;
+    if (a.loc_cnt) *a.loc_cnt = K;
     if (a.counts) a.counts[n] = K;
   }
 }
 
 // Fast path for rows of at most kFastMaxM entries and K_eff <= kRankMax,
-// with six group barriers: the threads keep their scores in registers; one
-// pass gives the softmax statistics and the minimum score; a 256-bin
-// histogram of s_max - s over [0, s_max - s_min] gives the bin b* holding the
-// K_eff-th largest score (the bin index is monotone in the score, so the top
-// K_eff entries all lie in bins <= b*); the entries of bins <= b* are ranked
-// among themselves by (score desc, position asc), which puts the top K_eff in
-// order; the mass scan then runs one ordered entry per thread.  Returns false,
-// having written nothing, when the candidates exceed kFastMaxCand; the caller
-// then runs the radix path.
+// with six group barriers and short dependency chains between them: the
+// threads keep their scores in registers; (1) the maximum and the minimum
+// score; (2) the softmax denominator (independent exponentials, summed in a
+// fixed tree) and a 256-bin histogram of s_max - s over [0, s_max - s_min],
+// which gives the bin b* holding the K_eff-th largest score (the bin index is
+// monotone in the score, so the top K_eff entries all lie in bins <= b*);
+// (3) the entries of bins <= b* are gathered (one shared-memory atomic per
+// warp) and (4) ranked among themselves by (score desc, position asc), which
+// puts the top K_eff in order; (5, 6) the mass scan runs one ordered entry
+// per thread.  Returns false, having written nothing, when the candidates
+// exceed kFastMaxCand; the caller then runs the radix path.
 constexpr int kFastMaxM = 2048;                   // 8 scores per thread
 constexpr int kFastMaxCand = FOVEA_MAX_K;         // candidates ranked directly
 
@@ -319,47 +331,48 @@ template <class Sync>
 __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, const float* s_sc,
                             SelectSmem& sm, int tid, Sync sync) {
   constexpr int PT = kFastMaxM / kSelThreads;
+  static_assert(PT == 8, "the denominator tree below sums eight terms per thread");
   const int lane = tid & 31, warp = tid >> 5;
   const int k_max = a.k_max;
   const int K_eff = min(k_max, M);
   float v[PT];
-  float lmax = -INFINITY, lsum = 0.0f, lmin = INFINITY;
+  float lmax = -INFINITY, lmin = INFINITY;
 #pragma unroll
   for (int j = 0; j < PT; ++j) {
     const int i = tid + j * kSelThreads;
     v[j] = i < M ? s_sc[i] : -INFINITY;
     if (i < M) {
-      combine_ms(lmax, lsum, v[j], 1.0f);
+      lmax = fmaxf(lmax, v[j]);
       lmin = fminf(lmin, v[j]);
     }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, lmax, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, lsum, o);
-    combine_ms(lmax, lsum, m2, s2);
+    lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, o));
     lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, o));
   }
   for (int i = tid; i < 256; i += kSelThreads) sm.hist[i] = 0;
   if (lane == 0) {
     sm.red_m[warp] = lmax;
-    sm.red_s[warp] = lsum;
     sm.red_lo[warp] = lmin;
   }
   if (tid == 0) sm.sh_cnt_gt = 0;
   sync();                                                     // (1)
-  float smax = sm.red_m[0], sumexp = sm.red_s[0], smin = sm.red_lo[0];
+  float smax = sm.red_m[0], smin = sm.red_lo[0];
+#pragma unroll
   for (int w = 1; w < kSelWarps; ++w) {
-    combine_ms(smax, sumexp, sm.red_m[w], sm.red_s[w]);
+    smax = fmaxf(smax, sm.red_m[w]);
     smin = fminf(smin, sm.red_lo[w]);
   }
-  // ---- histogram of the distance to the maximum ----------------------------
+  // ---- softmax denominator and histogram of the distance to the maximum ----
   const float range = smax - smin;
   const float inv_w = range > 0.0f ? 255.0f / range : 0.0f;
+  float ex[PT];
   int bin[PT];
 #pragma unroll
   for (int j = 0; j < PT; ++j) {
     const int i = tid + j * kSelThreads;
+    ex[j] = i < M ? expf(v[j] - smax) : 0.0f;
     bin[j] = 256;
     if (i < M) {
       const int b = (int)((smax - v[j]) * inv_w);
@@ -367,7 +380,14 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
       atomicAdd(&sm.hist[bin[j]], 1u);
     }
   }
+  float lsum = ((ex[0] + ex[1]) + (ex[2] + ex[3])) + ((ex[4] + ex[5]) + (ex[6] + ex[7]));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+  if (lane == 0) sm.red_s[warp] = lsum;
   sync();                                                     // (2)
+  float sumexp = sm.red_s[0];
+#pragma unroll
+  for (int w = 1; w < kSelWarps; ++w) sumexp += sm.red_s[w];
   // every warp finds b* itself: lane l owns bins 8l .. 8l + 7
   int bstar;
   {
@@ -396,19 +416,28 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
     }
     bstar = __shfl_sync(0xffffffffu, bl, L) - 1;
   }
-  // ---- candidates: the entries of bins <= b* -------------------------------
+  // ---- candidates: the entries of bins <= b*, one atomic per warp ----------
+  {
+    unsigned int bal[PT];
+    int wtot = 0;
 #pragma unroll
-  for (int j = 0; j < PT; ++j) {
-    const int i = tid + j * kSelThreads;
-    const bool take = bin[j] <= bstar;
-    const unsigned int bal = __ballot_sync(0xffffffffu, take);
-    int slot0 = 0;
-    if (lane == 0 && bal) slot0 = atomicAdd(&sm.sh_cnt_gt, __popc(bal));
-    slot0 = __shfl_sync(0xffffffffu, slot0, 0);
-    if (take) {
-      const int slot = slot0 + __popc(bal & ((1u << lane) - 1u));
-      if (slot < kFastMaxCand)
-        sm.cand[slot] = ((unsigned long long)ord_key(v[j]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+    for (int j = 0; j < PT; ++j) {
+      bal[j] = __ballot_sync(0xffffffffu, bin[j] <= bstar);
+      wtot += __popc(bal[j]);
+    }
+    int slot = 0;
+    if (lane == 0 && wtot > 0) slot = atomicAdd(&sm.sh_cnt_gt, wtot);
+    slot = __shfl_sync(0xffffffffu, slot, 0);
+    const unsigned int below = (1u << lane) - 1u;
+#pragma unroll
+    for (int j = 0; j < PT; ++j) {
+      if (bin[j] <= bstar) {
+        const int sj = slot + __popc(bal[j] & below);
+        if (sj < kFastMaxCand)
+          sm.cand[sj] = ((unsigned long long)ord_key(v[j]) << 32) |
+                        (0xFFFFFFFFu - (uint32_t)(tid + j * kSelThreads));
+      }
+      slot += __popc(bal[j]);
     }
   }
   sync();                                                     // (3)
@@ -417,8 +446,16 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
   // ---- rank the candidates: rank = #larger (keys are distinct) -------------
   for (int c = tid; c < C; c += kSelThreads) {
     const unsigned long long me = sm.cand[c];
-    int r = 0;
-    for (int j = 0; j < C; ++j) r += sm.cand[j] > me;
+    int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+    int j = 0;
+    for (; j + 3 < C; j += 4) {
+      r0 += sm.cand[j] > me;
+      r1 += sm.cand[j + 1] > me;
+      r2 += sm.cand[j + 2] > me;
+      r3 += sm.cand[j + 3] > me;
+    }
+    for (; j < C; ++j) r0 += sm.cand[j] > me;
+    const int r = (r0 + r1) + (r2 + r3);
     if (r < K_eff) sm.sorted[r] = me;
   }
   sync();                                                     // (4)
@@ -457,15 +494,20 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
       const int pu = u == t ? pos : (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[u] & 0xFFFFFFFFull));
       const float eu = u == t ? e : expf(s_sc[pu] - smax);
       const int row = key_off + pu;
-      a.sel_pos[out_row + u] = row;
-      a.sel_w[out_row + u] = eu / denom;
+      if (a.sel_pos) a.sel_pos[out_row + u] = row;
+      if (a.sel_w) a.sel_w[out_row + u] = eu / denom;
+      if (a.loc_pos) {
+        a.loc_pos[u] = row;
+        a.loc_w[u] = eu / denom;
+      }
       if (a.indices) a.indices[out_row + u] = a.orig_index[row];
     } else if (a.indices) {
       a.indices[out_row + u] = -1;
     }
   }
   if (tid == 0) {
-    a.sel_cnt[n] = K;
+    if (a.sel_cnt) a.sel_cnt[n] = K;
+    if (a.loc_cnt) *a.loc_cnt = K;
     if (a.counts) a.counts[n] = K;
   }
   return true;
@@ -493,7 +535,8 @@ __device__ __forceinline__ void select_empty(const SelectArgs& a, int n, int tid
   for (int t = tid; t < a.k_max; t += kSelThreads)
     if (a.indices) a.indices[out_row + t] = -1;
   if (tid == 0) {
-    a.sel_cnt[n] = 0;
+    if (a.sel_cnt) a.sel_cnt[n] = 0;
+    if (a.loc_cnt) *a.loc_cnt = 0;
     if (a.counts) a.counts[n] = 0;
   }
 }

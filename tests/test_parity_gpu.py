@@ -63,6 +63,8 @@ SMALL = {
     "bf16-clustered": dict(d=256, m_sizes=[2048], rows=[128], clusters=16, cluster_sigma=0.2,
                            k_max=256),
     "bf16-many-rows": dict(d=256, m_sizes=[130, 500], rows=[300, 4], k_max=64),
+    # rows beyond 2048 entries: selection and readout run as two kernels
+    "bf16-long-rows": dict(d=256, m_sizes=[2500, 300], rows=[12, 5], k_max=64),
     "bf16-hidden-128": dict(d=256, m_sizes=[100], rows=[9], k_max=16, H=128),
     "fp32-ragged": dict(d=256, m_sizes=[64, 130], rows=[4, 11], dtype="fp32", k_max=16),
     "fp32-temperature": dict(d=192, m_sizes=[300, 20], rows=[17, 3], dtype="fp32", k_max=64,
@@ -114,13 +116,20 @@ def test_memory_build_matches_oracle(fovea, name):
 
 
 def test_paths_are_taken(fovea):
-    """AUTO runs the per-stage kernels; FUSED runs the persistent step kernel
-    for a bf16 call and refuses an fp32 one (outside its coverage)."""
+    """AUTO runs the per-stage kernels: for bf16 rows of up to 2048 entries
+    the selection, the projected readout and the first fusion layer's
+    activation in one kernel; beyond that, selection and readout as two
+    kernels and the first fusion layer as a GEMM.  FUSED runs the persistent
+    step kernel for a bf16 call and refuses an fp32 one (outside its
+    coverage)."""
     prev = fovea.step_path(fovea.PATH_AUTO)
     try:
         for path, name, want, absent in (
-                (fovea.PATH_AUTO, "bf16-ragged", {"ln_query", "query_proj", "select", "finalize"},
-                 "fused_step"),
+                (fovea.PATH_AUTO, "bf16-ragged",
+                 {"ln_query", "query_proj", "select_fuse", "fuse_out", "finalize"}, "fuse_hidden"),
+                (fovea.PATH_AUTO, "bf16-long-rows", {"select", "readout", "fuse_hidden"},
+                 "select_fuse"),
+                (fovea.PATH_AUTO, "fp32-ragged", {"select_readout", "fuse_hidden"}, "select_fuse"),
                 (fovea.PATH_FUSED, "bf16-ragged", {"fused_step"}, "query_proj")):
             fovea.step_path(path)
             s = store(small_workload(name))
