@@ -123,6 +123,14 @@ typedef struct fovea_params {
  * Valid entries are compacted in ascending position; the handle keeps each
  * entry's original position, which is what fovea_retrieve_fuse reports as an
  * index.  An image with no valid entry is allowed (its rows select nothing).
+ * bf16 with W_f1 and W_g1 given (and a valid mlp_hidden): the handle also
+ * keeps each value through the r-half of the first fusion layer,
+ * p_i = [W_f1 ; W_g1][:, d:2d] u_i ([2H], bf16).  The fusion of Eq.
+ * hidden_correction is linear in r_n before its SiLU, so a draft step can
+ * form [W_f1 ; W_g1][:, d:2d] r_n = sum_t alpha_t p_{pi(t)} from 2H-wide rows
+ * instead of d-wide ones.  fovea_retrieve_fuse uses them only when it is
+ * given the same W_f1, W_g1 pointers and mlp_hidden; weights changed in
+ * place after the build need a new memory (as W_K, W_U already do).
  * This call allocates the handle's device buffers and synchronises `stream`
  * once (to size them).  B in [1, FOVEA_MAX_SEQ], M_max in [0, ...],
  * per-image valid count <= FOVEA_MAX_ENTRIES.
@@ -192,8 +200,11 @@ FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void*
  * with cumulative global-softmax mass >= rho (|V| if rounding never reaches
  * it); K = min(|V|, k_max, max(k_min, K_raw)); an image with no valid entry
  * gives K = 0 and r = 0.
- * bf16 path: LN(h) + E_dep, q, r (before the fusion) and the SiLU
- * activations are stored as bf16; accumulation is fp32 throughout.
+ * bf16 path: LN(h) + E_dep, q and the SiLU activations are stored as bf16;
+ * r enters the fusion as a bf16 vector, or (memory with projected values for
+ * these weights, rows of <= 2048 entries, k_max <= 256) through the bf16
+ * projected values p_i with the sum kept in fp32; accumulation is fp32
+ * throughout.
  * Errors: INVALID_ARG, UNSUPPORTED (nothing enqueued), CUDA.
  */
 FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_memory* mem,
