@@ -731,8 +731,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
 
   // (1) x_h = LN_h(h) + E_dep[l]
   { KernelTimer t("ln_query", s);
-    e = launch_ln_rows(dt, h, nullptr, N, d, p->ln_h_gamma, p->ln_h_beta, p->ln_eps, p->E_dep,
-                       depth, p->max_depth, err, xh, s); }
+    e = launch_ln_query(dt, h, N, d, p->ln_h_gamma, p->ln_h_beta, p->ln_eps, p->E_dep, depth,
+                        p->max_depth, err, xh, s); }
   if (e != cudaSuccess) return cuda_fail(e, "ln_query");
 
   static thread_local GemmArgs a;

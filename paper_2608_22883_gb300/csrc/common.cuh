@@ -37,6 +37,16 @@ __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// 16-byte asynchronous global -> shared copy (both addresses 16-byte
+// aligned); cp_async_wait_all() waits for the calling thread's copies.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+               "l"(gmem)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 // ---------------------------------------------------------------------------
 // Reductions (fixed order, so results are run-to-run deterministic)
 // ---------------------------------------------------------------------------
@@ -186,6 +196,10 @@ cudaError_t launch_ln_rows(int dtype, const void* x, const int32_t* src_row, int
                            const void* gamma, const void* beta, float eps, const void* E,
                            const int32_t* depth, int max_depth, int* err, void* out,
                            cudaStream_t s);
+// LN of the draft hidden states plus the depth embedding (rowops.cu), fp32.
+cudaError_t launch_ln_query(int dtype, const void* h, int rows, int d, const void* gamma,
+                            const void* beta, float eps, const void* E, const int32_t* depth,
+                            int max_depth, int* err, void* out, cudaStream_t s);
 cudaError_t launch_count_valid(const uint8_t* mask, int B, int M_max, int32_t* counts,
                                cudaStream_t s);
 cudaError_t launch_compact(const uint8_t* mask, int B, int M_max, const int32_t* key_off,

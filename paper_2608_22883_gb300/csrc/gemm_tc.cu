@@ -196,6 +196,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_expect_tx(&full[i], f_bytes);
       tma_load_3d(smem + i * stage_bytes + r_bytes, mapF, &full[i], 0, fy, (su_lo + i) * KPS);
     }
+    if (lane == 0) {
+      // L2 prefetch of data later kernels of the step read (memory entries,
+      // weights: none of it is written by the previous kernel), this CTA's
+      // share of each range, in copies of up to 32 KB
+      const int ncta = (int)(gridDim.x * gridDim.y * gridDim.z);
+      const int cid = (int)(blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z));
+      for (int r = 0; r < args.n_prefetch; ++r) {
+        const long long bytes = args.pf_bytes[r] & ~15ll;
+        const long long share = ((bytes + ncta - 1) / ncta + 15) & ~15ll;
+        const long long beg = (long long)cid * share;
+        const long long len = min(share, bytes - beg);
+        const uint8_t* base = static_cast<const uint8_t*>(args.pf_ptr[r]) + beg;
+        for (long long off = 0; off < len; off += 32768)
+          prefetch_l2_bulk(base + off, (uint32_t)min(32768ll, len - off));
+      }
+    }
     pdl_wait();
     pdl_trigger();
     int issued = 0;

@@ -14,8 +14,12 @@ namespace fovea {
 // and the affine map is evaluated in double-float, so the single rounding to
 // the stored type is taken on an almost exact value (the value a float64
 // evaluation rounds).  16-byte vector loads; the row, gamma, beta and the
-// depth embedding are all requested before any arithmetic.  Optional gather
-// of source rows; an invalid depth sets kErrDepth and uses depth 0.
+// depth embedding are all requested before any arithmetic.  When the depth
+// embedding table fits (<= 64 KB), each thread copies its columns of every
+// row of it into shared memory before griddepcontrol.wait (weights: not
+// written by the previous kernel), so the depth lookup adds no dependent
+// global load.  Optional gather of source rows; an invalid depth sets
+// kErrDepth and uses depth 0.
 // ---------------------------------------------------------------------------
 constexpr int kLnThreads = 512;
 
@@ -31,11 +35,13 @@ template <class T>
 __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
     const T* __restrict__ x, const int32_t* __restrict__ src_row, int d,
     const T* __restrict__ gamma, const T* __restrict__ beta, float eps,
-    const T* __restrict__ E, const int32_t* __restrict__ depth, int max_depth, int* err,
-    T* __restrict__ out) {
+    const T* __restrict__ E, const int32_t* __restrict__ depth, int max_depth, int e_smem,
+    int* err, T* __restrict__ out) {
   constexpr int V = LnVec<T>::N;
   constexpr int kLnMaxVec = LnVec<T>::MAX;
   __shared__ dfloat red[2][kLnThreads / 32];
+  extern __shared__ __align__(16) uint8_t ln_dyn[];
+  T* e_s = reinterpret_cast<T*>(ln_dyn);            // [max_depth + 1, d] when e_smem
   const int row = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nvec = d / V;
@@ -46,6 +52,9 @@ __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
     if (vi < nvec) {
       ln_load<T>(gamma + vi * V, gv[j]);
       ln_load<T>(beta + vi * V, bv[j]);
+      if (E != nullptr && e_smem)
+        for (int r = 0; r <= max_depth; ++r)
+          cp_async16(e_s + (long long)r * d + vi * V, E + (long long)r * d + vi * V);
     }
   }
   pdl_wait();
@@ -60,7 +69,8 @@ __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
     }
   }
   const T* xr = x + src * d;
-  const T* er = E != nullptr ? E + (long long)dep * d : nullptr;
+  const T* er = E != nullptr ? (e_smem ? e_s : E) + (long long)dep * d : nullptr;
+  if (er != nullptr && e_smem) cp_async_wait_all();   // this thread's own copies
 #pragma unroll
   for (int j = 0; j < kLnMaxVec; ++j) {
     const int vi = tid + j * kLnThreads;
@@ -122,20 +132,173 @@ __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
   }
 }
 
+// LN of the draft hidden states plus the depth embedding (query equation:
+// LN(h_n) + E_dep[l_n]), fp32: the mean and the variance in two passes over
+// the register-resident row (sum of x, then sum of (x - mean)^2; fixed-order
+// warp and block reductions), the affine map in fp32, rounded once to the
+// stored type.  Against the float64 evaluation the stored value differs by
+// one unit in the last place only where the exact value lies within fp32
+// rounding of a midpoint of the stored type (for bf16 about one element in
+// 10^4; the query it feeds moves by ~1e-6 of its scale).  Same loads, depth
+// check and shared-memory depth table as ln_rows_kernel; one CTA per row.
+template <class T>
+__global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
+    const T* __restrict__ x, int d, const T* __restrict__ gamma, const T* __restrict__ beta,
+    float eps, const T* __restrict__ E, const int32_t* __restrict__ depth, int max_depth,
+    int e_smem, int* err, T* __restrict__ out) {
+  constexpr int V = LnVec<T>::N;
+  constexpr int kLnMaxVec = LnVec<T>::MAX;
+  constexpr int NW = kLnThreads / 32;
+  __shared__ float red[2][NW];
+  extern __shared__ __align__(16) uint8_t ln_dyn[];
+  T* e_s = reinterpret_cast<T*>(ln_dyn);            // [max_depth + 1, d] when e_smem
+  const int row = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nvec = d / V;
+  float xv[kLnMaxVec][V], gv[kLnMaxVec][V], bv[kLnMaxVec][V], ev[kLnMaxVec][V];
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {      // weights: independent of the predecessor
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      ln_load<T>(gamma + vi * V, gv[j]);
+      ln_load<T>(beta + vi * V, bv[j]);
+      if (e_smem)
+        for (int r = 0; r <= max_depth; ++r)
+          cp_async16(e_s + (long long)r * d + vi * V, E + (long long)r * d + vi * V);
+    }
+  }
+  pdl_wait();
+  pdl_trigger();
+  int dep = depth[row];
+  if (dep < 0 || dep > max_depth) {
+    if (tid == 0) atomicOr(err, kErrDepth);
+    dep = 0;
+  }
+  const T* xr = x + (long long)row * d;
+  const T* er = (e_smem ? e_s : E) + (long long)dep * d;
+  if (e_smem) cp_async_wait_all();          // this thread's own copies
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      ln_load<T>(xr + vi * V, xv[j]);
+      ln_load<T>(er + vi * V, ev[j]);
+    }
+  }
+  // pass 1: mean
+  float s = 0.0f;
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j)
+    if (tid + j * kLnThreads < nvec)
+#pragma unroll
+      for (int i = 0; i < V; ++i) s += xv[j][i];
+  s = warp_sum(s);
+  if (lane == 0) red[0][warp] = s;
+  __syncthreads();
+  float tot = 0.0f;
+#pragma unroll
+  for (int w = 0; w < NW; ++w) tot += red[0][w];
+  const float mean = tot / (float)d;
+  // pass 2: variance about the mean
+  float q = 0.0f;
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j)
+    if (tid + j * kLnThreads < nvec)
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        const float c = xv[j][i] - mean;
+        q = fmaf(c, c, q);
+      }
+  q = warp_sum(q);
+  if (lane == 0) red[1][warp] = q;
+  __syncthreads();
+  float qt = 0.0f;
+#pragma unroll
+  for (int w = 0; w < NW; ++w) qt += red[1][w];
+  const float rstd = 1.0f / sqrtf(qt / (float)d + eps);
+  T* o = out + (long long)row * d;
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) {
+      T res[V];
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        const float y = fmaf((xv[j][i] - mean) * rstd, gv[j][i], bv[j][i]) + ev[j][i];
+        res[i] = from_f32<T>(y);
+      }
+      *reinterpret_cast<uint4*>(o + vi * V) = *reinterpret_cast<const uint4*>(res);
+    }
+  }
+}
+
+cudaError_t launch_ln_query(int dtype, const void* h, int rows, int d, const void* gamma,
+                            const void* beta, float eps, const void* E, const int32_t* depth,
+                            int max_depth, int* err, void* out, cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  constexpr int kESmemMax = 64 * 1024;
+  const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
+  const size_t e_bytes = (size_t)(max_depth + 1) * d * es;
+  const int e_smem = e_bytes <= (size_t)kESmemMax ? 1 : 0;
+  const size_t smem = e_smem ? e_bytes : 0;
+  if (dtype == FOVEA_BF16) {
+    using T = __nv_bfloat16;
+    static bool configured = false;
+    if (!configured) {
+      cudaError_t e = cudaFuncSetAttribute(ln_query_kernel<T>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kESmemMax);
+      if (e != cudaSuccess) return e;
+      configured = true;
+    }
+    return launch_pdl(ln_query_kernel<T>, dim3(rows), dim3(kLnThreads), smem, s, (const T*)h, d,
+                      (const T*)gamma, (const T*)beta, eps, (const T*)E, depth, max_depth, e_smem,
+                      err, (T*)out);
+  }
+  static bool configured_f = false;
+  if (!configured_f) {
+    cudaError_t e = cudaFuncSetAttribute(ln_query_kernel<float>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kESmemMax);
+    if (e != cudaSuccess) return e;
+    configured_f = true;
+  }
+  return launch_pdl(ln_query_kernel<float>, dim3(rows), dim3(kLnThreads), smem, s, (const float*)h,
+                    d, (const float*)gamma, (const float*)beta, eps, (const float*)E, depth,
+                    max_depth, e_smem, err, (float*)out);
+}
+
 cudaError_t launch_ln_rows(int dtype, const void* x, const int32_t* src_row, int rows, int d,
                            const void* gamma, const void* beta, float eps, const void* E,
                            const int32_t* depth, int max_depth, int* err, void* out,
                            cudaStream_t s) {
   if (rows == 0) return cudaSuccess;
+  constexpr int kESmemMax = 64 * 1024;
+  const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
+  const size_t e_bytes = E != nullptr ? (size_t)(max_depth + 1) * d * es : 0;
+  const int e_smem = E != nullptr && e_bytes <= (size_t)kESmemMax ? 1 : 0;
+  const size_t smem = e_smem ? e_bytes : 0;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
-    return launch_pdl(ln_rows_kernel<T>, dim3(rows), dim3(kLnThreads), 0, s, (const T*)x, src_row,
-                      d, (const T*)gamma, (const T*)beta, eps, (const T*)E, depth, max_depth, err,
-                      (T*)out);
+    static bool configured = false;
+    if (!configured) {
+      cudaError_t e = cudaFuncSetAttribute(ln_rows_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           kESmemMax);
+      if (e != cudaSuccess) return e;
+      configured = true;
+    }
+    return launch_pdl(ln_rows_kernel<T>, dim3(rows), dim3(kLnThreads), smem, s, (const T*)x,
+                      src_row, d, (const T*)gamma, (const T*)beta, eps, (const T*)E, depth,
+                      max_depth, e_smem, err, (T*)out);
   }
-  return launch_pdl(ln_rows_kernel<float>, dim3(rows), dim3(kLnThreads), 0, s, (const float*)x,
+  static bool configured_f = false;
+  if (!configured_f) {
+    cudaError_t e = cudaFuncSetAttribute(ln_rows_kernel<float>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kESmemMax);
+    if (e != cudaSuccess) return e;
+    configured_f = true;
+  }
+  return launch_pdl(ln_rows_kernel<float>, dim3(rows), dim3(kLnThreads), smem, s, (const float*)x,
                     src_row, d, (const float*)gamma, (const float*)beta, eps, (const float*)E,
-                    depth, max_depth, err, (float*)out);
+                    depth, max_depth, e_smem, err, (float*)out);
 }
 
 // ---------------------------------------------------------------------------

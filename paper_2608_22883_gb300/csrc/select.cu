@@ -96,10 +96,6 @@ __device__ __forceinline__ int ld_dsmem_s32(uint32_t caddr) {
   asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(caddr) : "memory");
   return v;
 }
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 struct GatherArgs {
   // readout: U [rows, d] -> r_out [N, d] fp32 and / or r_lo [N, d] (either may be null)
@@ -114,43 +110,49 @@ struct GatherArgs {
   const void* b_f1;                 // [H]: bias of columns < H
   const void* b_g1;                 // [H]: bias of columns >= H
   void* act;                        // [N, HP]
-  int red_floats;                   // dynamic shared memory: scores / gather partial sums
+  int red_floats;                   // dynamic shared memory: the row's scores
 };
 
 // Weighted gather-sum over the selected rows of X [*, ld], columns
 // [c0, c0 + w) (w a multiple of V): out(vector index, sums) once per 16-byte
-// column vector.  Every thread of the CTA calls it (it may synchronise).
+// column vector.  A warp covers VPW column vectors with 32 / VPW groups of
+// lanes; group g sums the entries t = g, g + 32 / VPW, ... (eight gathers in
+// flight per lane) and the groups' sums are combined by a fixed shuffle tree,
+// so no shared memory or barrier is involved and the order is deterministic.
 template <class T, class Out>
 __device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, int w, int K,
-                                             const int32_t* pos, const float* wt, float* red,
-                                             int tid, Out out) {
+                                             const int32_t* pos, const float* wt, int tid, Out out) {
   constexpr int V = 16 / (int)sizeof(T);
+  constexpr int kWarps = kSelThreads / 32;
   const int nvec = w / V;
   if (nvec <= 0) return;
-  const int G = nvec >= kSelThreads ? 1 : kSelThreads / nvec;
-  for (int vc0 = 0; vc0 < nvec; vc0 += kSelThreads) {
-    const int g = G > 1 ? tid / nvec : 0;
-    const int vc = G > 1 ? tid - g * nvec : vc0 + tid;
+  int vpw = 1;                            // vectors per warp: a power of two <= 32
+  while (vpw < 32 && vpw * 2 * kWarps <= nvec) vpw *= 2;
+  const int gpw = 32 / vpw;               // lane groups per warp
+  const int lane = tid & 31, warp = tid >> 5;
+  const int g = lane / vpw, v = lane - g * vpw;
+  for (int vbase = 0; vbase < nvec; vbase += kWarps * vpw) {
+    const int vc = vbase + warp * vpw + v;
     float acc[V];
 #pragma unroll
     for (int i = 0; i < V; ++i) acc[i] = 0.0f;
-    if (g < G && vc < nvec) {
+    if (vc < nvec) {
       const T* col = X + c0 + (long long)vc * V;
       int t = g;
-      for (; t + (kRoUnroll - 1) * G < K; t += kRoUnroll * G) {
+      for (; t + (kRoUnroll - 1) * gpw < K; t += kRoUnroll * gpw) {
         uint4 raw[kRoUnroll];
 #pragma unroll
         for (int j = 0; j < kRoUnroll; ++j)
-          raw[j] = __ldg(reinterpret_cast<const uint4*>(col + (long long)pos[t + j * G] * ld));
+          raw[j] = __ldg(reinterpret_cast<const uint4*>(col + (long long)pos[t + j * gpw] * ld));
 #pragma unroll
         for (int j = 0; j < kRoUnroll; ++j) {
-          const float wj = wt[t + j * G];
+          const float wj = wt[t + j * gpw];
           const T* e = reinterpret_cast<const T*>(&raw[j]);
 #pragma unroll
           for (int i = 0; i < V; ++i) acc[i] = fmaf(wj, to_f32(e[i]), acc[i]);
         }
       }
-      for (; t < K; t += G) {
+      for (; t < K; t += gpw) {
         const uint4 raw = __ldg(reinterpret_cast<const uint4*>(col + (long long)pos[t] * ld));
         const float wj = wt[t];
         const T* e = reinterpret_cast<const T*>(&raw);
@@ -158,23 +160,11 @@ __device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, i
         for (int i = 0; i < V; ++i) acc[i] = fmaf(wj, to_f32(e[i]), acc[i]);
       }
     }
-    if (G > 1) {
-      if (g < G)
+    // combine the groups: lanes v, v + vpw, v + 2 vpw, ... (every lane takes part)
+    for (int o = 16; o >= vpw; o >>= 1)
 #pragma unroll
-        for (int i = 0; i < V; ++i) red[(g * nvec + vc) * V + i] = acc[i];
-      __syncthreads();
-      if (tid < nvec) {
-#pragma unroll
-        for (int i = 0; i < V; ++i) acc[i] = red[tid * V + i];
-        for (int gg = 1; gg < G; ++gg)
-#pragma unroll
-          for (int i = 0; i < V; ++i) acc[i] += red[(gg * nvec + tid) * V + i];
-        out(tid, acc);
-      }
-      __syncthreads();                    // red is free again
-      break;                              // one pass covers the chunk
-    }
-    if (vc < nvec) out(vc, acc);
+      for (int i = 0; i < V; ++i) acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], o);
+    if (g == 0 && vc < nvec) out(vc, acc);
   }
 }
 
@@ -183,7 +173,7 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
     const __grid_constant__ SelectArgs args, const __grid_constant__ SeqTable tab,
     const __grid_constant__ GatherArgs ga) {
   constexpr int V = 16 / (int)sizeof(T);                     // elements per 16-byte vector
-  // dynamic: [red_floats] scores, later gather partial sums | [chunk_p] G_h | [chunk_p] bias
+  // dynamic: [red_floats] scores | [chunk_p] G_h | [chunk_p] bias
   extern __shared__ __align__(16) float dyn[];
   __shared__ SelectSmem sm;
   __shared__ __align__(16) int32_t loc_pos[kRankMax];
@@ -243,11 +233,10 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
   cp_async_wait_all();
   __syncthreads();
   const int K = loc_cnt;
-  float* red = s_sc;
   // projected readout -> act = SiLU(G_h + sum + bias)
   if (wp > 0) {
     T* act = static_cast<T*>(ga.act) + (long long)n * ga.HP + cp0;
-    gather_chunk<T>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, red, tid,
+    gather_chunk<T>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid,
                     [&](int vc, const float (&acc)[V]) {
                       T res[V];
 #pragma unroll
@@ -263,7 +252,7 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
   const int wu = (ga.r_out != nullptr || ga.r_lo != nullptr) ? max(0, min(ga.chunk_u, ga.d - cu0)) : 0;
   if (wu > 0) {
     const long long o = (long long)n * ga.d + cu0;
-    gather_chunk<T>(static_cast<const T*>(ga.U), ga.d, cu0, wu, K, loc_pos, loc_w, red, tid,
+    gather_chunk<T>(static_cast<const T*>(ga.U), ga.d, cu0, wu, K, loc_pos, loc_w, tid,
                     [&](int vc, const float (&acc)[V]) {
                       if (ga.r_out != nullptr) {
 #pragma unroll
@@ -303,7 +292,6 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   while (nchunk < 8 && (long long)N * nchunk * 2 <= 2LL * sms && d % (nchunk * 2 * 64) == 0 &&
          (P == nullptr || HP % (nchunk * 2 * 64) == 0))
     nchunk *= 2;
-  const int V = dtype == FOVEA_BF16 ? 8 : 4;
   GatherArgs ga{};
   ga.U = U;
   ga.d = d;
@@ -318,7 +306,7 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   ga.b_f1 = b_f1;
   ga.b_g1 = b_g1;
   ga.act = act;
-  ga.red_floats = (int)align_up_sz((size_t)std::max(std::max(max_m, 1), kSelThreads * V), 4);
+  ga.red_floats = (int)align_up_sz((size_t)std::max(max_m, 1), 4);
   const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
   const size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
                       align_up_sz((size_t)ga.chunk_p * es, 16);
