@@ -54,14 +54,17 @@ def load_peaks():
 # Algorithmic bytes / flops (what the method itself must move and compute)
 # ---------------------------------------------------------------------------
 
-def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray):
+def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, projected: bool):
     """Per-step algorithmic bytes and flops: W_Q, the fusion weights, every
-    valid key of every sequence, the unique selected value rows, row I/O
+    valid key of every sequence, the unique selected memory rows, row I/O
     (h in, h_hat out, counts and indices); scores and hidden activations are
-    intermediates and are not counted."""
+    intermediates and are not counted.  `projected`: the step reads the
+    memory's projected values p_i = [W_f1 ; W_g1]_r u_i (2H wide) instead of
+    the values, and only the h-half of the first fusion layer's weights."""
     d, H, N = w.d, w.params["b_f1"].shape[0], w.N
     es = 2 if w.dtype == "bf16" else 4
-    weights = d * d + 2 * H * 2 * d + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
+    fuse1 = 2 * H * (d if projected else 2 * d)
+    weights = d * d + fuse1 + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
     weights += 2 * d + 2 * d      # LN_h gamma/beta + the E_dep rows touched (bound: 2 rows)
     keys = sum(w.m_sizes) * d
     uniq = 0
@@ -71,22 +74,26 @@ def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray):
         for n in range(lo, hi):
             sel.update(int(x) for x in indices[n, :int(counts[n])])
         uniq += len(sel)
-    values = uniq * d
+    row_w = 2 * H if projected else d
+    values = uniq * row_w
     rows_io = 2 * N * d
     nbytes = es * (weights + keys + values + rows_io) + N * 4 + N * w.k_max * 4
     flops = 2 * N * d * d                                       # query
     rows = [int(w.row_offsets[b + 1] - w.row_offsets[b]) for b in range(w.B)]
     flops += sum(2 * rows[b] * int(w.m_sizes[b]) * d for b in range(w.B))
-    flops += 2 * int(counts.sum()) * d                          # readout
-    flops += 2 * N * (2 * d * 2 * H + H * d + H)                # fusion
+    flops += 2 * int(counts.sum()) * row_w                      # readout (projected or not)
+    flops += 2 * N * (fuse1 + H * d + H)                        # fusion
     return float(nbytes), float(flops), int(uniq)
 
 
-def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int) -> float:
+def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: bool) -> float:
     """HBM bytes one launch of a kernel must move (reads + writes)."""
     d, H, N = w.d, w.params["b_f1"].shape[0], w.N
     es = 2 if w.dtype == "bf16" else 4
+    scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
     if name == "query_proj":
+        if projected:     # W_Q and the h-half of [W_f1 ; W_g1]; x, h in; q_hi, q_lo, G_h out
+            return es * (d * d + 2 * H * d + 2 * N * d + 2 * N * d) + 4 * N * 2 * H
         return es * (d * d + N * d + 2 * N * d)
     if name == "fuse_hidden":
         return es * (2 * H * 2 * d + 2 * N * d + N * 2 * H + 2 * H)
@@ -94,12 +101,14 @@ def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int) -> float:
         return es * (d * H + N * H + d) + 4 * N * d
     if name == "score":
         keys = sum(w.m_sizes) * d * es
-        scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
         return keys + 2 * N * d * es + scores
     if name == "readout":
         return uniq_values * d * es + N * d * (4 + es)
+    if name == "select_fuse":     # scores in; projected rows, G_h, biases in; activations out
+        return scores + uniq_values * 2 * H * es + 4 * N * 2 * H + es * (2 * H + N * 2 * H) + N * 4 + N * w.k_max * 4
+    if name == "select_readout":
+        return scores + uniq_values * d * es + N * d * (4 + es) + N * 4 + N * w.k_max * 4
     if name == "select":
-        scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
         return scores + 3 * N * w.k_max * 4
     if name == "ln_query":
         return es * (2 * N * d + 4 * d)
@@ -423,7 +432,8 @@ def main():
 
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
-    nbytes, flops, uniq = step_cost(w, c_np, i_np)
+    projected = "select_fuse" in per_kernel
+    nbytes, flops, uniq = step_cost(w, c_np, i_np, projected)
     peaks, peak_src = load_peaks()
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
@@ -431,7 +441,7 @@ def main():
     kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
     dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
     # the persistent step kernel moves the whole step's algorithmic bytes
-    dom_bytes = nbytes if dom == "fused_step" else kernel_bytes(dom, w, uniq)
+    dom_bytes = nbytes if dom == "fused_step" else kernel_bytes(dom, w, uniq, projected)
     achieved = dom_bytes / (kern[dom]["ms_avg"] / 1000.0) / 1e9
     launches_per_step = sum(k["launches"] for k in kern.values()) / max(n_kt, 1)
     launches = int(round(launches_per_step * args.steps))
