@@ -433,11 +433,16 @@ def main():
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
     projected = "select_fuse" in per_kernel
-    nbytes, flops, uniq = step_cost(w, c_np, i_np, projected)
+    # the method's algorithmic bytes (full fusion weights, value rows), and
+    # what this path's step moves (projected values: the h-half weights and
+    # 2H-wide memory rows; the projection itself is part of the memory build)
+    nbytes, flops, uniq = step_cost(w, c_np, i_np, False)
+    nbytes_path, flops_path, _ = step_cost(w, c_np, i_np, projected)
     peaks, peak_src = load_peaks()
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
     t_roof = max(t_hbm, t_tc)
+    t_roof_path = max(nbytes_path / (peaks["hbm_gbs"] * 1e9), flops_path / (peaks["bf16_tflops"] * 1e12))
     kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
     dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
     # the persistent step kernel moves the whole step's algorithmic bytes
@@ -479,6 +484,10 @@ def main():
         "step_roofline": {"bytes": nbytes, "flops": flops, "unique_value_rows": uniq,
                           "t_roof_us": 1e6 * t_roof, "bound": "hbm" if t_hbm >= t_tc else "tensor",
                           "frac": t_roof / (ms / 1000.0),
+                          "this_path": {"bytes": nbytes_path, "flops": flops_path,
+                                        "t_roof_us": 1e6 * t_roof_path,
+                                        "frac": t_roof_path / (ms / 1000.0),
+                                        "projected_values": projected},
 
                           "peaks": f"{peak_src}: {peaks['hbm_gbs']} GB/s, {peaks['bf16_tflops']} TF/s"},
         "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"]} for k, v in kern.items()},
