@@ -762,18 +762,14 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.groups[0] = GemmGroup{0, d + 2 * H, 0, N, 0};
   }
   if (bf) {
-    // the keys (scores, next), and the projected values and / or the values
-    // when most of their rows will be read
+    // the keys (scores, next), and the values when most of their rows will
+    // be read by the readout
     long long m_sel = 0;
     for (int b = 0; b < mem->B; ++b)
       m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
     a.pf_ptr[a.n_prefetch] = mem->keys;
     a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
     if (2 * m_sel >= mem->total) {
-      if (use_proj) {
-        a.pf_ptr[a.n_prefetch] = mem->proj;
-        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * 2 * H * 2;
-      }
       if (!use_proj || readout != nullptr) {
         a.pf_ptr[a.n_prefetch] = mem->values;
         a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
@@ -822,6 +818,10 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       }
       a.pf_ptr[a.n_prefetch] = p->W_f2;
       a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
+      if (use_proj) {      // the projected values, gathered right after the scores
+        a.pf_ptr[a.n_prefetch] = mem->proj;
+        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * 2 * H * 2;
+      }
     }
     { KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
@@ -837,14 +837,14 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     { KernelTimer t("select_fuse", s);
       e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
                                counts, indices, mem->values, d, readout, nullptr, mem->proj, H,
-                               gh, p->b_f1, p->b_g1, act, s); }
+                               gh, p->b_f1, p->b_g1, act, err, s); }
     if (e != cudaSuccess) return cuda_fail(e, "select_fuse");
   } else {
     if (select_readout_fits(max_m, k_max)) {
       { KernelTimer t("select_readout", s);
         e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
                                  counts, indices, mem->values, d, readout, r_lo, nullptr, H,
-                                 nullptr, nullptr, nullptr, nullptr, s); }
+                                 nullptr, nullptr, nullptr, nullptr, err, s); }
       if (e != cudaSuccess) return cuda_fail(e, "select_readout");
     } else {
       { KernelTimer t("select", s);

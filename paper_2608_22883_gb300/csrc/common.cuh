@@ -221,7 +221,8 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
                                  const int32_t* orig_index, float rho, int k_min, int k_max,
                                  int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
-                                 const void* b_f1, const void* b_g1, void* act, cudaStream_t s);
+                                 const void* b_f1, const void* b_g1, void* act, int* err,
+                                 cudaStream_t s);
 // Exact rounding of listed key elements: k = sum_l x[row, l] W[col, l]
 // evaluated in double-float, rounded once to bf16.  list == nullptr refines
 // every element of the [rows, d] key matrix.

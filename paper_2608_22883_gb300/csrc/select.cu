@@ -114,16 +114,19 @@ struct GatherArgs {
 };
 
 // Weighted gather-sum over the selected rows of X [*, ld], columns
-// [c0, c0 + w) (w a multiple of V): out(vector index, sums) once per 16-byte
-// column vector.  A warp covers VPW column vectors with 32 / VPW groups of
-// lanes; group g sums the entries t = g, g + 32 / VPW, ... (eight gathers in
-// flight per lane) and the groups' sums are combined by a fixed shuffle tree,
-// so no shared memory or barrier is involved and the order is deterministic.
-template <class T, class Out>
+// [c0, c0 + w) (w a multiple of V): out(vector index, element, sum) once per
+// column.  A warp covers VPW column vectors with 32 / VPW groups of lanes;
+// group g sums the entries t = g, g + 32 / VPW, ... (eight gathers in flight
+// per lane) and the groups' sums are combined by a fixed xor-shuffle tree
+// (every lane of a vector ends with the full sums), so no shared memory or
+// barrier is involved and the order is deterministic; group g then emits
+// elements g, g + 32 / VPW, ... of its vector, so the epilogue work is spread
+// over all lanes.
+template <class T, int NT, class Out>
 __device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, int w, int K,
                                              const int32_t* pos, const float* wt, int tid, Out out) {
   constexpr int V = 16 / (int)sizeof(T);
-  constexpr int kWarps = kSelThreads / 32;
+  constexpr int kWarps = NT / 32;
   const int nvec = w / V;
   if (nvec <= 0) return;
   int vpw = 1;                            // vectors per warp: a power of two <= 32
@@ -164,16 +167,31 @@ __device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, i
     for (int o = 16; o >= vpw; o >>= 1)
 #pragma unroll
       for (int i = 0; i < V; ++i) acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], o);
-    if (g == 0 && vc < nvec) out(vc, acc);
+    if (vc < nvec) {
+#pragma unroll
+      for (int i = 0; i < V; ++i)
+        if (i % gpw == g) out(vc, i, acc[i]);
+    }
   }
 }
 
-template <class T>
-__global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
+// The selection group: the first kSelThreads threads of the CTA, synchronised
+// with a named barrier when the CTA is larger.
+struct SelGroupSync {
+  __device__ __forceinline__ void operator()() const {
+    asm volatile("bar.sync 1, %0;" ::"n"(kSelThreads) : "memory");
+  }
+};
+
+// NT threads per CTA: 256 (chunks of a row over a cluster) or 1024 (one CTA
+// per row: the selection on the first 256 threads, the gathers on all).
+template <class T, int NT>
+__global__ void __launch_bounds__(NT) select_gather_kernel(
     const __grid_constant__ SelectArgs args, const __grid_constant__ SeqTable tab,
     const __grid_constant__ GatherArgs ga) {
   constexpr int V = 16 / (int)sizeof(T);                     // elements per 16-byte vector
-  // dynamic: [red_floats] scores | [chunk_p] G_h | [chunk_p] bias
+  // dynamic: [red_floats] scores | [chunk_p] G_h | [chunk_p] bias | [red_floats] original
+  // positions of the row's sequence (int32)
   extern __shared__ __align__(16) float dyn[];
   __shared__ SelectSmem sm;
   __shared__ __align__(16) int32_t loc_pos[kRankMax];
@@ -187,19 +205,35 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
   T* bias_s = reinterpret_cast<T*>(gh_s + ga.chunk_p);
   pdl_wait();
   pdl_trigger();
-  // G_h and the biases of this CTA's projected chunk: requested now, used last
+  // G_h and the biases of this CTA's projected chunk, and (rank 0) the
+  // original positions of the sequence's entries: requested now, used last
+  int32_t* orig_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(bias_s) +
+                                               ((ga.chunk_p * (int)sizeof(T) + 15) & ~15));
+  if (rank == 0 && args.indices != nullptr) {
+    const int b = seq_of_row(tab, n);
+    const int M = tab.m[b];
+    const int32_t* src = args.orig_index + tab.key_off[b];
+    if ((tab.key_off[b] & 3) == 0) {
+      for (int q = tid; q < M / 4; q += NT) cp_async16(orig_s + 4 * q, src + 4 * q);
+      for (int i = (M / 4) * 4 + tid; i < M; i += NT) orig_s[i] = src[i];
+    } else {
+      for (int i = tid; i < M; i += NT) orig_s[i] = src[i];
+    }
+  }
   const int cp0 = blockIdx.y * ga.chunk_p;
   const int wp = ga.P != nullptr ? max(0, min(ga.chunk_p, ga.HP - cp0)) : 0;
-  for (int q = tid; q < wp / 4; q += kSelThreads)
+  for (int q = tid; q < wp / 4; q += NT)
     cp_async16(gh_s + 4 * q, ga.Gh + (long long)n * ga.HP + cp0 + 4 * q);
-  for (int q = tid; q < wp / V; q += kSelThreads) {
+  for (int q = tid; q < wp / V; q += NT) {
     const int c = cp0 + q * V;
     const T* src = c < ga.H ? static_cast<const T*>(ga.b_f1) + c
                             : static_cast<const T*>(ga.b_g1) + (c - ga.H);
     cp_async16(bias_s + q * V, src);
   }
-  if (rank == 0) {
+  if (rank == 0 && tid < kSelThreads) {
     SelectArgs a = args;
+    a.counts = nullptr;                   // written after the cluster barrier (below), so
+    a.indices = nullptr;                  // the barrier's release has no global writes to wait for
     a.loc_pos = loc_pos;
     a.loc_w = loc_w;
     a.loc_cnt = &loc_cnt;
@@ -214,14 +248,22 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
         if (v == 0.0f) v = 0.0f;          // -0 -> +0 so equal scores get equal keys
         s_sc[i] = v;
       }
-      __syncthreads();
-      select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSync{});
+      if constexpr (NT == kSelThreads) {
+        __syncthreads();
+        select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSync{});
+      } else {
+        SelGroupSync{}();
+        select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, SelGroupSync{});
+      }
     }
   }
-  cluster_sync();                         // rank 0's selection is visible to the cluster
+  // rank 0's selection visible to the cluster (one CTA: a CTA barrier, which
+  // does not wait for the selection's global writes to complete)
+  const bool clustered = gridDim.y > 1;
+  if (clustered) cluster_sync(); else __syncthreads();
   if (rank != 0) {
     const int K = ld_dsmem_s32(map_dsmem(smem_u32(&loc_cnt), 0));
-    for (int q = tid; q < (K + 3) / 4; q += kSelThreads) {
+    for (int q = tid; q < (K + 3) / 4; q += NT) {
       const float4 p4 = ld_dsmem_f4(map_dsmem(smem_u32(&loc_pos[4 * q]), 0));
       const float4 w4 = ld_dsmem_f4(map_dsmem(smem_u32(&loc_w[4 * q]), 0));
       *reinterpret_cast<float4*>(&loc_pos[4 * q]) = p4;
@@ -229,47 +271,41 @@ __global__ void __launch_bounds__(kSelThreads) select_gather_kernel(
     }
     if (tid == 0) loc_cnt = K;
   }
-  cluster_arrive();                       // done reading rank 0 (waited for before exit)
+  if (clustered) cluster_arrive();        // done reading rank 0 (waited for before exit)
   cp_async_wait_all();
   __syncthreads();
   const int K = loc_cnt;
+  if (rank == 0) {                        // counts and indices of row n
+    const long long out_row = (long long)n * args.k_max;
+    if (args.indices != nullptr) {
+      const int key_off = tab.key_off[seq_of_row(tab, n)];
+      for (int t = tid; t < args.k_max; t += NT)
+        args.indices[out_row + t] = t < K ? orig_s[loc_pos[t] - key_off] : -1;
+    }
+    if (args.counts != nullptr && tid == 0) args.counts[n] = K;
+  }
   // projected readout -> act = SiLU(G_h + sum + bias)
   if (wp > 0) {
     T* act = static_cast<T*>(ga.act) + (long long)n * ga.HP + cp0;
-    gather_chunk<T>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid,
-                    [&](int vc, const float (&acc)[V]) {
-                      T res[V];
-#pragma unroll
-                      for (int i = 0; i < V; ++i) {
-                        const float z = acc[i] + gh_s[vc * V + i] + to_f32(bias_s[vc * V + i]);
-                        res[i] = from_f32<T>(z * sigmoidf_(z));
-                      }
-                      *reinterpret_cast<uint4*>(act + vc * V) = *reinterpret_cast<const uint4*>(res);
-                    });
+    auto fin = [&](int vc, int i, float sum) {
+      const int c = vc * V + i;
+      const float z = sum + gh_s[c] + to_f32(bias_s[c]);
+      act[c] = from_f32<T>(z * sigmoidf_(z));
+    };
+    gather_chunk<T, NT>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid, fin);
   }
   // readout r_n
   const int cu0 = blockIdx.y * ga.chunk_u;
   const int wu = (ga.r_out != nullptr || ga.r_lo != nullptr) ? max(0, min(ga.chunk_u, ga.d - cu0)) : 0;
   if (wu > 0) {
     const long long o = (long long)n * ga.d + cu0;
-    gather_chunk<T>(static_cast<const T*>(ga.U), ga.d, cu0, wu, K, loc_pos, loc_w, tid,
-                    [&](int vc, const float (&acc)[V]) {
-                      if (ga.r_out != nullptr) {
-#pragma unroll
-                        for (int i = 0; i < V; i += 4)
-                          *reinterpret_cast<float4*>(ga.r_out + o + vc * V + i) =
-                              make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
-                      }
-                      if (ga.r_lo != nullptr) {
-                        T res[V];
-#pragma unroll
-                        for (int i = 0; i < V; ++i) res[i] = from_f32<T>(acc[i]);
-                        *reinterpret_cast<uint4*>(static_cast<T*>(ga.r_lo) + o + vc * V) =
-                            *reinterpret_cast<const uint4*>(res);
-                      }
-                    });
+    auto fin = [&](int vc, int i, float sum) {
+      if (ga.r_out != nullptr) ga.r_out[o + vc * V + i] = sum;
+      if (ga.r_lo != nullptr) static_cast<T*>(ga.r_lo)[o + vc * V + i] = from_f32<T>(sum);
+    };
+    gather_chunk<T, NT>(static_cast<const T*>(ga.U), ga.d, cu0, wu, K, loc_pos, loc_w, tid, fin);
   }
-  cluster_wait();                         // rank 0 stays until every CTA has copied
+  if (clustered) cluster_wait();          // rank 0 stays until every CTA has copied
 }
 
 bool select_readout_fits(int max_m, int k_max) { return max_m <= kFastMaxM && k_max <= kRankMax; }
@@ -278,7 +314,8 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
                                  const int32_t* orig_index, float rho, int k_min, int k_max,
                                  int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
-                                 const void* b_f1, const void* b_g1, void* act, cudaStream_t s) {
+                                 const void* b_f1, const void* b_g1, void* act, int* err,
+                                 cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   if (!select_readout_fits(max_m, k_max) || d % 64 != 0 || (P != nullptr && H % 64 != 0))
     return cudaErrorInvalidValue;
@@ -288,9 +325,15 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
   if (e != cudaSuccess) return e;
   const int HP = 2 * H;
+  // projected readout: one CTA of 1024 threads per row (the selection on
+  // 256 of them; a cluster barrier costs about a microsecond, more than the
+  // gathers gain from spreading over more SMs); the readout alone: a cluster
+  // of CTAs of 256 threads per row, about two CTAs per SM in one wave, each
+  // chunk a multiple of 64 columns
+  const bool wide = P != nullptr;
   int nchunk = 1;
-  while (nchunk < 8 && (long long)N * nchunk * 2 <= 2LL * sms && d % (nchunk * 2 * 64) == 0 &&
-         (P == nullptr || HP % (nchunk * 2 * 64) == 0))
+  while (!wide && nchunk < 8 && (long long)N * nchunk * 2 <= 2LL * sms &&
+         d % (nchunk * 2 * 64) == 0)
     nchunk *= 2;
   GatherArgs ga{};
   ga.U = U;
@@ -309,13 +352,24 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   ga.red_floats = (int)align_up_sz((size_t)std::max(max_m, 1), 4);
   const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
   const size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
-                      align_up_sz((size_t)ga.chunk_p * es, 16);
-  if (smem > 48 * 1024) return cudaErrorInvalidValue;
+                      align_up_sz((size_t)ga.chunk_p * es, 16) + (size_t)ga.red_floats * 4;
+  if (smem > 64 * 1024) return cudaErrorInvalidValue;
+  static bool configured = false;
+  if (!configured) {
+    for (auto k : {(const void*)select_gather_kernel<__nv_bfloat16, 1024>,
+                   (const void*)select_gather_kernel<__nv_bfloat16, kSelThreads>,
+                   (const void*)select_gather_kernel<float, 1024>,
+                   (const void*)select_gather_kernel<float, kSelThreads>}) {
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+      if (e != cudaSuccess) return e;
+    }
+    configured = true;
+  }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices,
                nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(N, nchunk);
-  cfg.blockDim = dim3(kSelThreads);
+  cfg.blockDim = dim3(wide ? 1024 : kSelThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
@@ -328,8 +382,10 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   if (dtype == FOVEA_BF16)
-    return cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16>, a, tab, ga);
-  return cudaLaunchKernelEx(&cfg, select_gather_kernel<float>, a, tab, ga);
+    return wide ? cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16, 1024>, a, tab, ga)
+                : cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16, kSelThreads>, a, tab, ga);
+  return wide ? cudaLaunchKernelEx(&cfg, select_gather_kernel<float, 1024>, a, tab, ga)
+              : cudaLaunchKernelEx(&cfg, select_gather_kernel<float, kSelThreads>, a, tab, ga);
 }
 
 }  // namespace fovea
