@@ -30,11 +30,13 @@
 // Split K: when the output tiles cannot fill the GPU (a 64-row batch against
 // a weight matrix), S <= 8 CTAs share one output tile, each contracting a
 // slice of K.  The S CTAs of a tile form a thread-block cluster: each stages
-// its fp32 partial tile row-major in its own shared memory (over the idle
-// stage ring), the cluster synchronises, and CTA r sums the S partials of
-// column quads [r Q/S, (r+1) Q/S) (Q = BN/4) in rank order through
-// distributed shared memory (so the result does not depend on timing) and runs the epilogue for
+// its fp32 partial tile in its own shared memory (over the idle stage ring),
+// the cluster synchronises, and CTA r sums the S partials of column quads
+// [r Q/S, (r+1) Q/S) (Q = BN/4) in rank order through distributed shared
+// memory (so the result does not depend on timing) and runs the epilogue for
 // them; a second cluster barrier keeps every partial alive until it is read.
+// (Pushing the partials into the owners' shared memory with remote stores and
+// an mbarrier handshake measured slower: remote stores issue one at a time.)
 //
 // Launch overlap: kernels are launched with programmatic dependent launch.
 // The producer issues the feature-operand (weight / key) loads of the first
@@ -352,77 +354,111 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the tile's cluster meet, and CTA `rank` sums columns [rank cpo,
     // (rank+1) cpo) of the S partial tiles in rank order through distributed
     // shared memory before writing them.
-    float* part = reinterpret_cast<float*>(smem);
-    const int ldp = BN + 4;
     const int rows_real = min(BM, g.n - n0);
     const bool have_acc = ok && nkb > 0;          // warp-uniform
-    if (quarter * 32 < rows_real) {               // warp-uniform
+    if (S == 1) {
+      float* part = reinterpret_cast<float*>(smem);
+      const int ldp = BN + 4;
+      if (quarter * 32 < rows_real) {             // warp-uniform
 #pragma unroll 1
-      for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
-        float v[32];
-        if (have_acc) {
-          tmem_ld32(taddr + (uint32_t)c0, v);     // the whole warp, converged
-        } else {
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+          float v[32];
+          if (have_acc) {
+            tmem_ld32(taddr + (uint32_t)c0, v);   // the whole warp, converged
+          } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = 0.0f;
-        }
-        if (row_in_tile < rows_real) {
+            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+          }
+          if (row_in_tile < rows_real) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            *reinterpret_cast<float4*>(part + row_in_tile * ldp + c0 + 4 * q) =
-                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(part + row_in_tile * ldp + c0 + 4 * q) =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
         }
       }
-    }
-    __syncwarp();
-    if (S > 1) cluster_sync(); else __syncthreads();
-    // CTA `rank` owns the column quads [qlo, qhi) of the tile
-    const int qlo = (int)rank * (BN / 4) / S, qhi = ((int)rank + 1) * (BN / 4) / S;
-    const int q4 = qhi - qlo;
-    const int items = rows_real * q4;
-    // two items per thread and round, all their loads in flight together
-    for (int it0 = threadIdx.x; it0 < items; it0 += 2 * kThreads) {
-      float4 t[2][8];
-      int rr[2], cc[2];
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int it = it0 + k * kThreads;
-        rr[k] = -1;
-        if (it < items) {
-          rr[k] = it / q4;
-          cc[k] = (qlo + (it - rr[k] * q4)) * 4;
-          const float* src = part + rr[k] * ldp + cc[k];
-          if (S == 1) {
-            t[k][0] = *reinterpret_cast<const float4*>(src);
+      __syncthreads();
+      const int q4 = BN / 4;
+      const int items = rows_real * q4;
+      for (int it = threadIdx.x; it < items; it += kThreads) {
+        const int rr = it / q4, cc = (it - rr * q4) * 4;
+        const float4 a4 = *reinterpret_cast<const float4*>(part + rr * ldp + cc);
+        if (ok && cc < n_cols) {
+          const float vals[4] = {a4.x, a4.y, a4.z, a4.w};
+          gemm_epilogue4<EPI>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc), bias_s + cc);
+        }
+      }
+    } else {
+      // Split K: each CTA stages its fp32 partial tile row-major [rows][BN + 4]
+      // over its idle ring (the pitch spreads a warp's 16-byte stores over all
+      // banks); the cluster meets, and CTA `rank` sums the column quads
+      // [qlo, qhi) of the S partial tiles in rank order through distributed
+      // shared memory; a second cluster barrier keeps every partial alive
+      // until it has been read.
+      float* part = reinterpret_cast<float*>(smem);
+      const int ldp = BN + 4;
+      if (quarter * 32 < rows_real) {             // warp-uniform
+#pragma unroll 1
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 32) {
+          float v[32];
+          if (have_acc) {
+            tmem_ld32(taddr + (uint32_t)c0, v);   // the whole warp, converged
           } else {
-            const uint32_t laddr = smem_u32(src);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0.0f;
+          }
+          if (row_in_tile < rows_real) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(part + row_in_tile * ldp + c0 + 4 * q) =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
+        }
+      }
+      __syncwarp();
+      cluster_sync();
+      const int qlo = (int)rank * (BN / 4) / S, qhi = ((int)rank + 1) * (BN / 4) / S;
+      const int q4 = qhi - qlo;
+      const int items = rows_real * q4;
+      // two items per thread and round, all their remote loads in flight together
+      for (int it0 = threadIdx.x; it0 < items; it0 += 2 * kThreads) {
+        float4 t[2][8];
+        int rr[2], cc[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          const int it = it0 + k * kThreads;
+          rr[k] = -1;
+          if (it < items) {
+            rr[k] = it / q4;
+            cc[k] = (qlo + (it - rr[k] * q4)) * 4;
+            const uint32_t laddr = smem_u32(part + rr[k] * ldp + cc[k]);
 #pragma unroll
             for (int sidx = 0; sidx < 8; ++sidx)
               if (sidx < S) t[k][sidx] = ld_dsmem_f4(map_dsmem(laddr, (uint32_t)sidx));
           }
         }
-      }
 #pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        if (rr[k] < 0) continue;
-        float4 acc = t[k][0];
+        for (int k = 0; k < 2; ++k) {
+          if (rr[k] < 0) continue;
+          float4 acc = t[k][0];
 #pragma unroll
-        for (int sidx = 1; sidx < 8; ++sidx)
-          if (sidx < S) {
-            acc.x += t[k][sidx].x;
-            acc.y += t[k][sidx].y;
-            acc.z += t[k][sidx].z;
-            acc.w += t[k][sidx].w;
+          for (int sidx = 1; sidx < 8; ++sidx)
+            if (sidx < S) {
+              acc.x += t[k][sidx].x;
+              acc.y += t[k][sidx].y;
+              acc.z += t[k][sidx].z;
+              acc.w += t[k][sidx].w;
+            }
+          if (ok && cc[k] < n_cols) {
+            const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+            gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
+                                bias_s + cc[k]);
           }
-        if (ok && cc[k] < n_cols) {
-          const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
-          gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
-                              bias_s + cc[k]);
         }
       }
+      __syncwarp();
+      cluster_sync();   // no CTA leaves while another still reads its partial tile
     }
-    __syncwarp();
-    if (S > 1) cluster_sync();   // no CTA leaves while another still reads its partial tile
   }
   tc_fence_before();
   __syncthreads();
