@@ -218,6 +218,17 @@ def cores_used() -> int:
         return os.cpu_count() or 1
 
 
+def max_over_ranks(value: float, dist, device) -> float:
+    """The largest `value` over the ranks of the job (a replica job's step time
+    is its slowest replica's); `dist` is torch.distributed or None (one rank)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_reference(args, w):
     import oracle
     rank = int(os.environ.get("RANK", "0"))
@@ -395,10 +406,7 @@ def main():
     clk = clocks.stop()
     ms = float(np.mean(step_ms))
     fovea.sync_errors(ws)
-    if dist is not None:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dist, dev)
     value = world * N / (ms / 1000.0)
 
     # ---- kernel-timing pass: the same step with an event pair around every
@@ -431,7 +439,7 @@ def main():
         e1.record(stream)
         e1.synchronize()
         e2e_ms_l.append(e0.elapsed_time(e1))
-    e2e_ms = float(np.mean(e2e_ms_l))
+    e2e_ms = max_over_ranks(float(np.mean(e2e_ms_l)), dist, dev)
     h2d = h_host.numel() * h_host.element_size() + depth_host.numel() * 4
     d2h = h_out_host.numel() * h_out_host.element_size() + N * 4 + N * K * 4
     assert torch.equal(h_out_host, h_out.cpu())

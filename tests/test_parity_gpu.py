@@ -115,6 +115,38 @@ def test_memory_build_matches_oracle(fovea, name):
     mem.destroy()
 
 
+def test_plain_fusion_when_weights_differ(fovea):
+    """The memory keeps the values projected through the r-half of the first
+    fusion layer for the W_f1 / W_g1 it was built with.  A bf16 call given
+    other W_f1 / W_g1 pointers (here copies holding the same values) takes the
+    plain path: the readout r, then the first fusion layer as a GEMM over
+    [h; r].  Both paths match the oracle, and each other within the bf16
+    tolerance, with identical selections."""
+    w = small_workload("bf16-ragged")
+    s = store(w)
+    orc, mem = run_oracle(s, mirror=True)
+    params = params_for(s, fovea)
+    fovea.timing_enable(True)
+    proj = run_gpu(s, fovea, params=params)
+    names_proj = set(fovea.timing_read())
+    weights = {n: s.dev[n] for n in workloads.PARAM_NAMES}
+    weights["W_f1"] = weights["W_f1"].clone()
+    weights["W_g1"] = weights["W_g1"].clone()
+    other = fovea.Params(weights, d_model=w.d, mlp_hidden=w.params["b_f1"].shape[0],
+                         max_depth=w.params["E_dep"].shape[0] - 1, dtype=fovea.BF16)
+    fovea.timing_enable(True)              # clears the records
+    plain = run_gpu(s, fovea, params=other, memory=proj["_memory"])
+    names_plain = set(fovea.timing_read())
+    fovea.timing_enable(False)
+    assert "select_fuse" in names_proj and "fuse_hidden" not in names_proj
+    assert "fuse_hidden" in names_plain and "select_fuse" not in names_plain
+    for gpu in (proj, plain):
+        compare(gpu, orc, s, mem=mem, mirror=True)
+    np.testing.assert_array_equal(proj["counts"], plain["counts"])
+    np.testing.assert_array_equal(proj["indices"], plain["indices"])
+    assert rel_err_rows(proj["h_out"].astype(np.float64), plain["h_out"].astype(np.float64)).max() <= 2e-2
+
+
 def test_paths_are_taken(fovea):
     """AUTO runs the per-stage kernels: for bf16 rows of up to 2048 entries
     the selection, the projected readout and the first fusion layer's
