@@ -323,14 +323,27 @@ def main():
 
     N, d, K = w.N, w.d, w.k_max
     ws = fovea.new_workspace(params, mem, w.row_offsets, K)
-    h_out = torch.empty_like(h)
-    counts = torch.empty(N, dtype=torch.int32, device=dev)
-    indices = torch.empty((N, K), dtype=torch.int32, device=dev)
+    # The step's inputs (h, depth) and outputs (h_hat, counts, indices) each
+    # live in one contiguous buffer, so the end-to-end step moves them with
+    # one host-to-device and one device-to-host copy.
+    def packed(parts, device, pin=False):
+        sizes = [int(np.prod(shp)) * torch.empty((), dtype=dt_).element_size() for shp, dt_ in parts]
+        offs = np.cumsum([0] + [(b + 255) // 256 * 256 for b in sizes])
+        buf = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
+        if pin:
+            buf = buf.pin_memory()
+        views = [buf[int(o):int(o) + b].view(dt_).view(shp) for o, b, (shp, dt_) in zip(offs, sizes, parts)]
+        return buf, views
+    out_parts = [((N, d), h.dtype), ((N,), torch.int32), ((N, K), torch.int32)]
+    out_dev, (h_out, counts, indices) = packed(out_parts, dev)
     offs_c = fovea._offsets(w.row_offsets)
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.float32, device=dev)
-    h_in = torch.empty_like(h)          # the step reads its inputs from here
-    depth_in = torch.empty_like(depth)
+    in_parts = [((N, d), h.dtype), ((N,), torch.int32)]
+    in_dev, (h_in, depth_in) = packed(in_parts, dev)         # the step reads its inputs here
+    in_host, (h_in_host, depth_in_host) = packed(in_parts, "cpu", pin=True)
+    h_in_host.copy_(h_host)
+    depth_in_host.copy_(depth_host)
     h_in.copy_(h)
     depth_in.copy_(depth)
 
@@ -358,17 +371,12 @@ def main():
         step()
     # end to end: the host inputs copied in, the step, the results copied
     # back, as one graph (pinned host buffers)
-    h_out_host = torch.empty(h_out.shape, dtype=h_out.dtype).pin_memory()
-    counts_host = torch.empty(N, dtype=torch.int32).pin_memory()
-    idx_host = torch.empty((N, K), dtype=torch.int32).pin_memory()
+    out_host, (h_out_host, counts_host, idx_host) = packed(out_parts, "cpu", pin=True)
     g_e2e = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_e2e, stream=cap):
-        h_in.copy_(h_host, non_blocking=True)
-        depth_in.copy_(depth_host, non_blocking=True)
+        in_dev.copy_(in_host, non_blocking=True)
         step()
-        h_out_host.copy_(h_out, non_blocking=True)
-        counts_host.copy_(counts, non_blocking=True)
-        idx_host.copy_(indices, non_blocking=True)
+        out_host.copy_(out_dev, non_blocking=True)
     fovea.timing_enable(True)            # per-kernel event nodes in the timed graph
     g_timed = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_timed, stream=cap):
@@ -440,8 +448,8 @@ def main():
         e1.synchronize()
         e2e_ms_l.append(e0.elapsed_time(e1))
     e2e_ms = max_over_ranks(float(np.mean(e2e_ms_l)), dist, dev)
-    h2d = h_host.numel() * h_host.element_size() + depth_host.numel() * 4
-    d2h = h_out_host.numel() * h_out_host.element_size() + N * 4 + N * K * 4
+    h2d = in_host.numel()
+    d2h = out_host.numel()
     assert torch.equal(h_out_host, h_out.cpu())
 
     # ---- roofline ----
