@@ -762,13 +762,16 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.groups[0] = GemmGroup{0, d + 2 * H, 0, N, 0};
   }
   if (bf) {
-    // the keys (scores, next), and the values when most of their rows will
-    // be read by the readout
+    // the keys when the score GEMM's own loads before its griddepcontrol.wait
+    // (its first ring stages) cannot cover them, and the values when most of
+    // their rows will be read by the readout
     long long m_sel = 0;
     for (int b = 0; b < mem->B; ++b)
       m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
-    a.pf_ptr[a.n_prefetch] = mem->keys;
-    a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+    if ((long long)mem->total * d * 2 > (8ll << 20)) {
+      a.pf_ptr[a.n_prefetch] = mem->keys;
+      a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+    }
     if (2 * m_sel >= mem->total) {
       if (!use_proj || readout != nullptr) {
         a.pf_ptr[a.n_prefetch] = mem->values;
@@ -807,21 +810,17 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     }
     a.ngroups = g;
     a.dual_b = bf ? 1 : 0;
-    if (bf) {
+    if (bf && !use_proj) {
       // the fusion weights, read after selection and readout (with the
-      // projected values, only the second correction layer)
-      if (!use_proj) {
-        a.pf_ptr[a.n_prefetch] = p->W_f1;
-        a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
-        a.pf_ptr[a.n_prefetch] = p->W_g1;
-        a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
-      }
+      // projected values the selection kernel prefetches them, and the
+      // second correction layer's GEMM loads its weights before its
+      // griddepcontrol.wait)
+      a.pf_ptr[a.n_prefetch] = p->W_f1;
+      a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
+      a.pf_ptr[a.n_prefetch] = p->W_g1;
+      a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
       a.pf_ptr[a.n_prefetch] = p->W_f2;
       a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
-      if (use_proj) {      // the projected values, gathered right after the scores
-        a.pf_ptr[a.n_prefetch] = mem->proj;
-        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * 2 * H * 2;
-      }
     }
     { KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
@@ -837,7 +836,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     { KernelTimer t("select_fuse", s);
       e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
                                counts, indices, mem->values, d, readout, nullptr, mem->proj, H,
-                               gh, p->b_f1, p->b_g1, act, err, s); }
+                               gh, p->b_f1, p->b_g1, act, err, s,
+                               (long long)mem->total * 2 * H * 2); }
     if (e != cudaSuccess) return cuda_fail(e, "select_fuse");
   } else {
     if (select_readout_fits(max_m, k_max)) {

@@ -215,14 +215,15 @@ cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, con
 // at most 2048 valid entries and k_max <= 256 (select_readout_fits): the
 // readout r (r_out fp32 and / or r_lo, either may be null; U unused when
 // both are) and, when P is given, act = SiLU(Gh + sum_t alpha_t P[pi(t)] +
-// [b_f1 ; b_g1]) over 2H columns.
+// [b_f1 ; b_g1]) over 2H columns.  p_prefetch_bytes: the first bytes of P the
+// CTAs prefetch into L2 before waiting for the scores (0: none).
 bool select_readout_fits(int max_m, int k_max);
 cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable& tab, int N,
                                  const int32_t* orig_index, float rho, int k_min, int k_max,
                                  int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
                                  const void* b_f1, const void* b_g1, void* act, int* err,
-                                 cudaStream_t s);
+                                 cudaStream_t s, long long p_prefetch_bytes = 0);
 // Exact rounding of listed key elements: k = sum_l x[row, l] W[col, l]
 // evaluated in double-float, rounded once to bf16.  list == nullptr refines
 // every element of the [rows, d] key matrix.

@@ -110,6 +110,7 @@ struct GatherArgs {
   const void* b_f1;                 // [H]: bias of columns < H
   const void* b_g1;                 // [H]: bias of columns >= H
   void* act;                        // [N, HP]
+  long long p_prefetch;             // bytes of P prefetched into L2 before the wait
   int red_floats;                   // dynamic shared memory: the row's scores
 };
 
@@ -203,6 +204,19 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
   float* s_sc = dyn;
   float* gh_s = dyn + ga.red_floats;
   T* bias_s = reinterpret_cast<T*>(gh_s + ga.chunk_p);
+  if (ga.p_prefetch > 0 && tid == 0) {
+    // the projected values (memory: not written by the previous kernel),
+    // this CTA's share, into L2 while the scores are computed
+    const int ncta = (int)(gridDim.x * gridDim.y);
+    const int cid = (int)(blockIdx.x + gridDim.x * blockIdx.y);
+    const long long bytes = ga.p_prefetch & ~15ll;
+    const long long share = ((bytes + ncta - 1) / ncta + 15) & ~15ll;
+    const long long beg = (long long)cid * share;
+    const long long len = min(share, bytes - beg);
+    const uint8_t* base = static_cast<const uint8_t*>(ga.P) + beg;
+    for (long long off = 0; off < len; off += 32768)
+      tc::prefetch_l2_bulk(base + off, (uint32_t)min(32768ll, len - off));
+  }
   pdl_wait();
   pdl_trigger();
   // G_h and the biases of this CTA's projected chunk, and (rank 0) the
@@ -315,7 +329,7 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
                                  int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
                                  const void* b_f1, const void* b_g1, void* act, int* err,
-                                 cudaStream_t s) {
+                                 cudaStream_t s, long long p_prefetch_bytes) {
   if (N == 0) return cudaSuccess;
   if (!select_readout_fits(max_m, k_max) || d % 64 != 0 || (P != nullptr && H % 64 != 0))
     return cudaErrorInvalidValue;
@@ -349,6 +363,7 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   ga.b_f1 = b_f1;
   ga.b_g1 = b_g1;
   ga.act = act;
+  ga.p_prefetch = P != nullptr ? p_prefetch_bytes : 0;
   ga.red_floats = (int)align_up_sz((size_t)std::max(max_m, 1), 4);
   const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
   const size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
