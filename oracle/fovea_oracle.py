@@ -41,6 +41,13 @@ h_hat (R8).  The query q is not rounded: the bf16 path carries it as a pair
 of bf16 values (about 16 significant bits), so its scores follow the exact
 q.  ``mirror=False`` is exact float64 throughout.
 
+Query folding (``fold=True`` in ``retrieve_fuse``): since q_n . k_i =
+(W_Q x_n) . k_i = x_n . (W_Q^T k_i) with x_n = LN(h_n) + E_dep[l_n], the scores
+may be taken against folded keys kappa_i = W_Q^T k_i formed once per image
+(``fold_keys``).  In exact arithmetic both orders give the same scores; in
+mirror mode kappa_i is rounded to bfloat16 (R9, the folded keys' storage)
+and x_n keeps its R3 rounding, which is what the folded bf16 path stores.
+
 Parity pins: tests/test_oracle_pins.py (bf16 rounding against torch, LN/RMSNorm
 against torch.nn.functional, subset enumeration, closed forms, dense
 attention, fixed top-K against lexsort, gate identities).
@@ -125,6 +132,7 @@ class Memory:
     values: List[np.ndarray]    # per image [|V_b|, d], u_i
     index: List[np.ndarray]     # per image: original position i of each valid entry
     d: int
+    folded: Optional[List[np.ndarray]] = None   # per image [|V_b|, d], kappa_i = W_Q^T k_i
 
 
 def build_memory(p: Dict[str, np.ndarray], v, mask=None, *, mirror=False,
@@ -149,11 +157,22 @@ def build_memory(p: Dict[str, np.ndarray], v, mask=None, *, mirror=False,
 # Retrieval (Sec. "State-conditioned top-K visual evidence retrieval")
 # ----------------------------------------------------------------------------
 
+def query_input(p, h, depth, *, mirror=False, ln_eps=1e-5):
+    """x_n = LN(h_n) + E_dep[l_n], the input of the query projection."""
+    return _maybe(layer_norm(h, p["ln_h_gamma"], p["ln_h_beta"], ln_eps)
+                  + p["E_dep"][np.asarray(depth)], mirror)
+
+
 def query(p, h, depth, *, mirror=False, ln_eps=1e-5):
     """q_n = W_Q (LN(h_n) + E_dep[l_n])."""
-    x = _maybe(layer_norm(h, p["ln_h_gamma"], p["ln_h_beta"], ln_eps)
-               + p["E_dep"][np.asarray(depth)], mirror)
-    return x @ p["W_Q"].T
+    return query_input(p, h, depth, mirror=mirror, ln_eps=ln_eps) @ p["W_Q"].T
+
+
+def fold_keys(p, mem: Memory, *, mirror=False) -> Memory:
+    """Query folding: kappa_i = W_Q^T k_i for every key of every image, so that
+    q_n . k_i = x_n . kappa_i.  Returns the memory with ``folded`` set."""
+    folded = [_maybe(K @ p["W_Q"], mirror) for K in mem.keys]
+    return dataclasses.replace(mem, folded=folded)
 
 
 def scores(q_n, K_b, d, row_scale_n=1.0):
@@ -225,10 +244,12 @@ def fuse(p, h, r, *, mirror=False, rms_eps=1e-6):
 
 def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
                   k_max, *, mirror=False, ln_eps=1e-5, rms_eps=1e-6,
-                  rows=None) -> Dict[str, object]:
+                  rows=None, fold=False) -> Dict[str, object]:
     """Retrieve + fuse for every draft state; rows row_offsets[b] ..
     row_offsets[b+1]-1 query image b.  ``rows`` restricts the computation to a
-    subset of row indices (the rest of the outputs stay zero / -1)."""
+    subset of row indices (the rest of the outputs stay zero / -1).
+    ``fold`` scores x_n against the folded keys (``fold_keys``) instead of
+    q_n against the keys."""
     h = np.asarray(h, dtype=F64)
     N, d = h.shape
     rho = float(np.float32(rho))
@@ -236,8 +257,12 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
     want = np.arange(N) if rows is None else np.asarray(sorted(rows))
     seq_of = np.searchsorted(row_offsets, np.arange(N), side="right") - 1
     q = np.zeros((N, d))
+    x = np.zeros((N, d))
+    if fold and mem.folded is None:
+        mem = fold_keys(p, mem, mirror=mirror)
     if len(want):
-        q[want] = query(p, h[want], np.asarray(depth)[want], mirror=mirror, ln_eps=ln_eps)
+        x[want] = query_input(p, h[want], np.asarray(depth)[want], mirror=mirror, ln_eps=ln_eps)
+        q[want] = x[want] @ p["W_Q"].T
     counts = np.zeros(N, np.int64)
     k_raw = np.zeros(N, np.int64)
     indices = -np.ones((N, k_max), np.int64)
@@ -248,7 +273,7 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
     for n in want:
         b = int(seq_of[n])
         scale = 1.0 if row_scale is None else float(row_scale[n])
-        s = scores(q[n], mem.keys[b], d, scale)
+        s = scores(x[n], mem.folded[b], d, scale) if fold else scores(q[n], mem.keys[b], d, scale)
         S = select(s, rho, k_min, k_max)
         r[n], alphas[n] = readout(s, S.selected, mem.values[b])
         counts[n], k_raw[n] = S.K, S.K_raw

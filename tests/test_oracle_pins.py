@@ -7,6 +7,7 @@ The mutation tests at the end plant a plausible mistake in a copy of an
 oracle function and show that one of the pins catches it.
 """
 
+import dataclasses
 import itertools
 import json
 import math
@@ -378,6 +379,49 @@ def test_mirror_rounds_at_the_storage_points():
     assert rel < 5e-2
 
 
+def test_folded_scores_equal_query_scores():
+    """Query folding: x . (W_Q^T k) against (W_Q x) . k with q formed by
+    torch.nn.functional.linear and the keys by the oracle's build."""
+    p = small_params()
+    v, mask, h, depth, offs = small_step(p, seed=15)
+    mem = oracle.fold_keys(p, oracle.build_memory(p, v, mask))
+    x = oracle.query_input(p, h, depth)
+    q = F.linear(t64(x), t64(p["W_Q"])).numpy()
+    for b in range(len(mem.keys)):
+        for n in range(offs[b], offs[b + 1]):
+            want = mem.keys[b] @ q[n] / 8.0
+            np.testing.assert_allclose(oracle.scores(x[n], mem.folded[b], 64), want,
+                                       rtol=1e-11, atol=1e-11)
+
+
+def test_folded_step_equals_plain_step_in_exact_arithmetic():
+    p = small_params()
+    v, mask, h, depth, offs = small_step(p, seed=16, M=(30, 0, 9), rows=(4, 2, 3))
+    row_scale = np.random.default_rng(17).uniform(0.2, 3.0, h.shape[0])
+    mem = oracle.build_memory(p, v, mask)
+    a = oracle.retrieve_fuse(p, mem, h, depth, offs, row_scale, 0.8, 2, 6)
+    b = oracle.retrieve_fuse(p, mem, h, depth, offs, row_scale, 0.8, 2, 6, fold=True)
+    np.testing.assert_array_equal(a["counts"], b["counts"])
+    np.testing.assert_array_equal(a["indices"], b["indices"])
+    for key in ("readout", "h_out", "gate"):
+        np.testing.assert_allclose(b[key], a[key], rtol=1e-10, atol=1e-12)
+
+
+def test_folded_mirror_rounds_the_folded_keys():
+    p = small_params()
+    v, mask, h, depth, offs = small_step(p, seed=18)
+    mem = oracle.build_memory(p, v, mask, mirror=True)
+    exact = oracle.fold_keys(p, mem)
+    fm = oracle.fold_keys(p, mem, mirror=True)
+    for kf, ke in zip(fm.folded, exact.folded):
+        np.testing.assert_array_equal(kf, oracle.round_bf16(kf))
+        assert np.all(np.abs(kf - ke) <= 2.0 ** -8 * np.abs(ke) + 1e-300)   # half a bf16 ulp
+    out = oracle.retrieve_fuse(p, fm, h, depth, offs, None, 0.9, 1, 8, mirror=True, fold=True)
+    x = oracle.round_bf16(oracle.layer_norm(h, p["ln_h_gamma"], p["ln_h_beta"], 1e-5) + p["E_dep"][depth])
+    for n in range(offs[1]):
+        np.testing.assert_allclose(out["scores"][n], fm.folded[0] @ x[n] / 8.0, rtol=1e-12, atol=1e-12)
+
+
 def test_planted_rows_are_peaked():
     spec = workloads.Spec(0, "planted-small", d=256, B=1, rows_per_seq=12, rho=0.9,
                           k_max=16, k_min=1, dtype="fp32", seed=21, m_fixed=96,
@@ -463,3 +507,15 @@ def test_pins_catch_transposed_query_and_swapped_concat():
     _, _, want = torch_fusion(p, h, r)
     swapped = oracle.fuse(p, r, h)["h_out"]               # [r; h] instead of [h; r]
     assert not np.allclose(swapped, want, rtol=1e-6)
+
+
+def test_pins_catch_a_transposed_fold():
+    p = small_params()
+    v, mask, h, depth, offs = small_step(p, seed=15)
+    mem = oracle.build_memory(p, v, mask)
+    bad = dataclasses.replace(mem, folded=[K @ p["W_Q"].T for K in mem.keys])   # W_Q k, not W_Q^T k
+    x = oracle.query_input(p, h, depth)
+    q = F.linear(t64(x), t64(p["W_Q"])).numpy()
+    n = 0
+    assert not np.allclose(oracle.scores(x[n], bad.folded[0], 64), mem.keys[0] @ q[n] / 8.0,
+                           rtol=1e-6)
