@@ -54,17 +54,20 @@ def load_peaks():
 # Algorithmic bytes / flops (what the method itself must move and compute)
 # ---------------------------------------------------------------------------
 
-def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, projected: bool):
+def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, projected: bool,
+              folded: bool = False):
     """Per-step algorithmic bytes and flops: W_Q, the fusion weights, every
     valid key of every sequence, the unique selected memory rows, row I/O
     (h in, h_hat out, counts and indices); scores and hidden activations are
     intermediates and are not counted.  `projected`: the step reads the
     memory's projected values p_i = [W_f1 ; W_g1]_r u_i (2H wide) instead of
-    the values, and only the h-half of the first fusion layer's weights."""
+    the values, and only the h-half of the first fusion layer's weights.
+    `folded`: the step scores x_h against the memory's folded keys
+    W_Q^T k_i (formed with the memory), so W_Q is not read and q not formed."""
     d, H, N = w.d, w.params["b_f1"].shape[0], w.N
     es = 2 if w.dtype == "bf16" else 4
     fuse1 = 2 * H * (d if projected else 2 * d)
-    weights = d * d + fuse1 + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
+    weights = (0 if folded else d * d) + fuse1 + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
     weights += 2 * d + 2 * d      # LN_h gamma/beta + the E_dep rows touched (bound: 2 rows)
     keys = sum(w.m_sizes) * d
     uniq = 0
@@ -78,7 +81,7 @@ def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, pr
     values = uniq * row_w
     rows_io = 2 * N * d
     nbytes = es * (weights + keys + values + rows_io) + N * 4 + N * w.k_max * 4
-    flops = 2 * N * d * d                                       # query
+    flops = 0 if folded else 2 * N * d * d                      # query
     rows = [int(w.row_offsets[b + 1] - w.row_offsets[b]) for b in range(w.B)]
     flops += sum(2 * rows[b] * int(w.m_sizes[b]) * d for b in range(w.B))
     flops += 2 * int(counts.sum()) * row_w                      # readout (projected or not)
@@ -95,6 +98,12 @@ def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: 
         if projected:     # W_Q and the h-half of [W_f1 ; W_g1]; x, h in; q_hi, q_lo, G_h out
             return es * (d * d + 2 * H * d + 2 * N * d + 2 * N * d) + 4 * N * 2 * H
         return es * (d * d + N * d + 2 * N * d)
+    if name == "fusion_h":        # the h-half of [W_f1 ; W_g1]; h in; G_h out
+        return es * (2 * H * d + N * d) + 4 * N * 2 * H
+    if name == "score_fusion_h":  # folded keys, the h-half of [W_f1 ; W_g1], x_h and h in; scores, G_h out
+        return (sum(w.m_sizes) * d + 2 * H * d + 2 * N * d) * es + scores + 4 * N * 2 * H
+    if name == "score_folded":    # folded keys, x_h in; scores out
+        return sum(w.m_sizes) * d * es + N * d * es + scores
     if name == "fuse_hidden":
         return es * (2 * H * 2 * d + 2 * N * d + N * 2 * H + 2 * H)
     if name == "fuse_out":
@@ -455,11 +464,12 @@ def main():
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
     projected = "select_fuse" in per_kernel
+    folded = "score_folded" in per_kernel
     # the method's algorithmic bytes (full fusion weights, value rows), and
     # what this path's step moves (projected values: the h-half weights and
     # 2H-wide memory rows; the projection itself is part of the memory build)
     nbytes, flops, uniq = step_cost(w, c_np, i_np, False)
-    nbytes_path, flops_path, _ = step_cost(w, c_np, i_np, projected)
+    nbytes_path, flops_path, _ = step_cost(w, c_np, i_np, projected, folded)
     peaks, peak_src = load_peaks()
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
@@ -509,7 +519,8 @@ def main():
                           "this_path": {"bytes": nbytes_path, "flops": flops_path,
                                         "t_roof_us": 1e6 * t_roof_path,
                                         "frac": t_roof_path / (ms / 1000.0),
-                                        "projected_values": projected},
+                                        "projected_values": projected,
+                                        "folded_keys": folded},
 
                           "peaks": f"{peak_src}: {peaks['hbm_gbs']} GB/s, {peaks['bf16_tflops']} TF/s"},
         "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"]} for k, v in kern.items()},

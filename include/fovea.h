@@ -131,6 +131,13 @@ typedef struct fovea_params {
  * instead of d-wide ones.  fovea_retrieve_fuse uses them only when it is
  * given the same W_f1, W_g1 pointers and mlp_hidden; weights changed in
  * place after the build need a new memory (as W_K, W_U already do).
+ * bf16 with W_Q given: the handle also keeps the folded keys
+ * kappa_i = W_Q^T k_i ([d], bf16; query folding).  Since
+ * q_n . k_i = (W_Q x_n) . k_i = x_n . kappa_i with x_n = LN(h_n) + E_dep[l_n],
+ * a draft step given the same W_Q pointer scores x_n against kappa_i and
+ * never streams W_Q.  kappa_i is rounded once from its exact value (elements
+ * whose fp32 sum lies near a bf16 rounding midpoint are recomputed in
+ * double-float).  Pass W_Q = NULL here to keep the unfolded scores.
  * This call allocates the handle's device buffers and synchronises `stream`
  * once (to size them).  B in [1, FOVEA_MAX_SEQ], M_max in [0, ...],
  * per-image valid count <= FOVEA_MAX_ENTRIES.
@@ -157,6 +164,12 @@ FOVEA_API fovea_status fovea_memory_info(const fovea_memory* mem, int* B,
 FOVEA_API fovea_status fovea_memory_tensors(const fovea_memory* mem, const void** keys,
                                             const void** values, const int32_t** index,
                                             int64_t* offsets);
+
+/* The folded keys kappa_i = W_Q^T k_i [total_valid, d] (bf16, device, owned
+ * by the handle) when the memory holds them for this W_Q pointer, else NULL
+ * in *folded: a step given this W_Q scores against them. */
+FOVEA_API fovea_status fovea_memory_folded_keys(const fovea_memory* mem, const void* W_Q,
+                                                const void** folded);
 
 /*
  * Bytes of workspace fovea_retrieve_fuse needs for this memory, these row
@@ -200,7 +213,9 @@ FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void*
  * with cumulative global-softmax mass >= rho (|V| if rounding never reaches
  * it); K = min(|V|, k_max, max(k_min, K_raw)); an image with no valid entry
  * gives K = 0 and r = 0.
- * bf16 path: LN(h) + E_dep, q and the SiLU activations are stored as bf16;
+ * bf16 path: LN(h) + E_dep, q and the SiLU activations are stored as bf16
+ * (with folded keys for this W_Q, q is not formed: the scores are
+ * (x_n . kappa_i) / sqrt(d) * row_scale, x_n the stored bf16 LN(h) + E_dep);
  * r enters the fusion as a bf16 vector, or (memory with projected values for
  * these weights, rows of <= 2048 entries, k_max <= 256) through the bf16
  * projected values p_i with the sum kept in fp32; accumulation is fp32

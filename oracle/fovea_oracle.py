@@ -168,10 +168,13 @@ def query(p, h, depth, *, mirror=False, ln_eps=1e-5):
     return query_input(p, h, depth, mirror=mirror, ln_eps=ln_eps) @ p["W_Q"].T
 
 
-def fold_keys(p, mem: Memory, *, mirror=False) -> Memory:
-    """Query folding: kappa_i = W_Q^T k_i for every key of every image, so that
-    q_n . k_i = x_n . kappa_i.  Returns the memory with ``folded`` set."""
-    folded = [_maybe(K @ p["W_Q"], mirror) for K in mem.keys]
+def fold_keys(p, mem: Memory, *, mirror=False, images=None) -> Memory:
+    """Query folding: kappa_i = W_Q^T k_i for every key of the given images
+    (default all), so that q_n . k_i = x_n . kappa_i.  Returns the memory with
+    ``folded`` set (None for images not folded)."""
+    B = len(mem.keys)
+    images = range(B) if images is None else set(images)
+    folded = [_maybe(mem.keys[b] @ p["W_Q"], mirror) if b in images else None for b in range(B)]
     return dataclasses.replace(mem, folded=folded)
 
 
@@ -259,7 +262,7 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
     q = np.zeros((N, d))
     x = np.zeros((N, d))
     if fold and mem.folded is None:
-        mem = fold_keys(p, mem, mirror=mirror)
+        mem = fold_keys(p, mem, mirror=mirror, images={int(seq_of[n]) for n in want})
     if len(want):
         x[want] = query_input(p, h[want], np.asarray(depth)[want], mirror=mirror, ln_eps=ln_eps)
         q[want] = x[want] @ p["W_Q"].T

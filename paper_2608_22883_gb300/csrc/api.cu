@@ -132,6 +132,12 @@ struct fovea_memory {
   const void* proj_wf1 = nullptr;
   const void* proj_wg1 = nullptr;
   int proj_h = 0;
+  // bf16: the keys folded through the query projection, kappa_i = W_Q^T k_i
+  // ([total, d]), and the W_Q they were built with: q . k_i = x . kappa_i,
+  // so a call with that W_Q scores x = LN(h) + E_dep against them directly
+  void* folded = nullptr;
+  const void* fold_wq = nullptr;
+  int folded_refined = 0;            // folded elements re-rounded exactly at build
 };
 
 static size_t esize(int dtype) { return dtype == FOVEA_BF16 ? 2 : 4; }
@@ -204,6 +210,7 @@ static void free_memory(fovea_memory* m) {
   cudaFree(m->keys);
   cudaFree(m->values);
   cudaFree(m->proj);
+  cudaFree(m->folded);
   cudaFree(m->orig_index);
   cudaFree(m->err);
   delete m;
@@ -370,6 +377,63 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
         if (err == cudaSuccess) err = cudaStreamSynchronize(s);
         if (err != cudaSuccess) return cuda_fail(err, "refine_keys");
       }
+      // bf16 with W_Q given: the folded keys kappa_i = W_Q^T k_i, a GEMM of
+      // W_Q^T (transposed once here) with the stored keys, listed elements
+      // near a bf16 rounding midpoint re-rounded exactly as for the keys
+      if (bf && p->W_Q != nullptr && aligned16(p->W_Q)) {
+        fovea_status fs = alloc_dev(&m->folded, (size_t)total * d * 2, "folded keys");
+        if (fs != FOVEA_OK) return fs;
+        void* wqt = nullptr;
+        if ((fs = alloc_dev(&wqt, (size_t)d * d * 2, "transposed W_Q")) != FOVEA_OK) return fs;
+        auto fold = [&]() -> fovea_status {
+          { KernelTimer t("transpose_wq", s);
+            err = launch_transpose_bf16(p->W_Q, d, d, wqt, s); }
+          if (err != cudaSuccess) return cuda_fail(err, "transpose W_Q");
+          err = cudaMemsetAsync(fix_count, 0, sizeof(int), s);
+          if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+          GemmArgs fa;
+          init_args(fa);
+          fa.k_total = d;
+          fa.b_split = d;
+          fa.B0 = m->keys; fa.ldb0 = d;
+          fa.epi_split = d;
+          fa.out0 = m->folded; fa.ldc = d;
+          fa.err = m->err;
+          fa.fix_list = fix_list; fa.fix_count = fix_count; fa.fix_cap = (int)fix_cap;
+          fa.ngroups = 1;
+          fa.groups[0] = GemmGroup{0, d, 0, total, 0};
+          { KernelTimer t("memory_fold", s);
+            err = launch_gemm_tc(kEpiStoreKeys, fa, TmaOperand{wqt, d, d, d},
+                                 TmaOperand{nullptr, 0, 0, 0}, TmaOperand{m->keys, total, d, d},
+                                 TmaOperand{nullptr, 0, 0, 0}, d, total, s); }
+          if (err != cudaSuccess) return cuda_fail(err, "query folding of the keys");
+          { KernelTimer t("refine_folded", s);
+            err = launch_refine_keys(m->keys, wqt, d, fix_list, fix_count, (int)fix_cap, total,
+                                     m->folded, s); }
+          if (err != cudaSuccess) return cuda_fail(err, "refine_folded");
+          int fe[2] = {0, 0};
+          err = cudaMemcpyAsync(&fe[0], m->err, sizeof(int), cudaMemcpyDeviceToHost, s);
+          if (err == cudaSuccess)
+            err = cudaMemcpyAsync(&fe[1], fix_count, sizeof(int), cudaMemcpyDeviceToHost, s);
+          if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+          if (err != cudaSuccess) return cuda_fail(err, "query folding");
+          if (fe[0] & kErrTimeout)
+            return fail(FOVEA_ERR_TIMEOUT, "a bounded device wait gave up while folding the keys");
+          m->folded_refined = fe[1];
+          if (fe[1] > fix_cap) {           // list overflowed: refine every element
+            { KernelTimer t("refine_folded", s);
+              err = launch_refine_keys(m->keys, wqt, d, nullptr, nullptr, 0, total, m->folded, s); }
+            if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+            if (err != cudaSuccess) return cuda_fail(err, "refine_folded");
+          }
+          return FOVEA_OK;
+        };
+        fs = fold();
+        cudaStreamSynchronize(s);
+        cudaFree(wqt);
+        if (fs != FOVEA_OK) return fs;
+        m->fold_wq = p->W_Q;
+      }
       // bf16 with the fusion weights given: p_i = [W_f1 ; W_g1]_r u_i, the
       // first fusion layer's r-half applied to every value once per image
       const int H = p->mlp_hidden;
@@ -423,6 +487,15 @@ FOVEA_API fovea_status fovea_memory_info(const fovea_memory* mem, int* B, int* t
   if (B) *B = mem->B;
   if (total_valid) *total_valid = mem->total;
   if (valid_counts) memcpy(valid_counts, mem->counts.data(), mem->B * sizeof(int32_t));
+  return FOVEA_OK;
+}
+
+FOVEA_API fovea_status fovea_memory_folded_keys(const fovea_memory* mem, const void* W_Q,
+                                                const void** folded) {
+  g_last_error.clear();
+  if (mem == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "memory is NULL");
+  if (folded == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "folded is NULL");
+  *folded = (mem->folded != nullptr && W_Q != nullptr && mem->fold_wq == W_Q) ? mem->folded : nullptr;
   return FOVEA_OK;
 }
 
@@ -740,10 +813,25 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   // projected values valid for these weights, the same launch computes
   // G_h = [W_f1 ; W_g1]_h h (the h-half of the first fusion layer, fp32):
   // the r-half then reduces to a weighted sum of projected values (4).
+  // With the memory's folded keys valid for this W_Q, q is never formed:
+  // the scores take x_h against the folded keys, and the launch computes
+  // G_h alone (or is skipped without the projected values).
   const bool bf = dt == FOVEA_BF16;
   const bool use_proj = bf && mem->proj != nullptr && mem->proj_wf1 == p->W_f1 &&
                         mem->proj_wg1 == p->W_g1 && mem->proj_h == H &&
                         select_readout_fits(max_m, k_max);
+  const bool use_fold = bf && mem->folded != nullptr && mem->fold_wq == p->W_Q;
+  const void* score_keys = use_fold ? mem->folded : mem->keys;
+  // With folded keys and projected values, G_h does not depend on the query:
+  // when one sequence's keys serve every row (one score group covering all N
+  // rows), the score launch computes it too, as two more feature parts
+  // against h.
+  int gh_seq = -1;
+  if (use_fold && use_proj && ngroups == 1) {
+    for (int b = 0; b < mem->B; ++b)
+      if (row_offsets[b + 1] - row_offsets[b] == N && mem->counts[b] > 0) gh_seq = b;
+  }
+  const bool gh_in_scores = gh_seq >= 0;
   void* q_lo = bf ? static_cast<void*>(static_cast<uint8_t*>(q) + (size_t)N * d * 2) : nullptr;
   init_args(a);
   a.k_total = d; a.b_split = d;
@@ -761,15 +849,17 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.out2 = gh; a.ldc2 = 2 * H;
     a.groups[0] = GemmGroup{0, d + 2 * H, 0, N, 0};
   }
+  // entries selected at most: when they are most of the memory, the value
+  // rows are prefetched
+  long long m_sel = 0;
+  for (int b = 0; b < mem->B; ++b)
+    m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
   if (bf) {
     // the keys when the score GEMM's own loads before its griddepcontrol.wait
     // (its first ring stages) cannot cover them, and the values when most of
     // their rows will be read by the readout
-    long long m_sel = 0;
-    for (int b = 0; b < mem->B; ++b)
-      m_sel += std::min<long long>(mem->counts[b], (long long)(row_offsets[b + 1] - row_offsets[b]) * k_max);
     if ((long long)mem->total * d * 2 > (8ll << 20)) {
-      a.pf_ptr[a.n_prefetch] = mem->keys;
+      a.pf_ptr[a.n_prefetch] = score_keys;
       a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
     }
     if (2 * m_sel >= mem->total) {
@@ -779,6 +869,21 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       }
     }
   }
+  if (use_fold && use_proj && !gh_in_scores) {
+    // G_h only: parts W_f1 and W_g1 (h-halves), both against h, fp32 out
+    a.A0 = p->W_f1; a.lda0 = 2 * d;
+    a.B0 = h;
+    a.a_split = H; a.a_split2 = 0x7fffffff;
+    a.r_by_part = 0;
+    a.epi_split = 0;
+    a.out2 = gh; a.ldc2 = 2 * H;
+    a.groups[0] = GemmGroup{0, 2 * H, 0, N, 0};
+    { KernelTimer t("fusion_h", s);
+      e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{p->W_f1, H, d, 2 * d},
+                         TmaOperand{p->W_g1, H, d, 2 * d}, TmaOperand{h, N, d, d},
+                         TmaOperand{nullptr, 0, 0, 0}, 2 * H, N, s); }
+    if (e != cudaSuccess) return cuda_fail(e, "fusion_h");
+  } else if (!use_fold) {
   { KernelTimer t("query_proj", s);
     if (use_proj)
       e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{p->W_Q, d, d, d}, TmaOperand{p->W_f1, H, d, 2 * d},
@@ -789,13 +894,14 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                    TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
                    TmaOperand{nullptr, 0, 0, 0}, d, N, s); }
   if (e != cudaSuccess) return cuda_fail(e, "query_proj");
+  }
 
   // (3) s = q k^T / sqrt(d) (* row_scale), per sequence
   if (score_elems > 0) {
     init_args(a);
     a.k_total = d; a.b_split = d;
-    a.A0 = mem->keys; a.lda0 = d;
-    a.B0 = q; a.ldb0 = d;
+    a.A0 = score_keys; a.lda0 = d;
+    a.B0 = use_fold ? xh : q; a.ldb0 = d;
     a.out0 = scores;
     a.row_scale = row_scale;
     a.scale = (float)(1.0 / sqrt((double)d));
@@ -809,7 +915,12 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       a.groups[g++] = GemmGroup{(int)mem->offsets[b], mem->counts[b], row_offsets[b], r, tab.score_off[b]};
     }
     a.ngroups = g;
-    a.dual_b = bf ? 1 : 0;
+    a.dual_b = bf && !use_fold ? 1 : 0;
+    if (use_fold && !use_proj && 2 * m_sel >= mem->total) {
+      // no query launch carries the value prefetch on this path
+      a.pf_ptr[a.n_prefetch] = mem->values;
+      a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+    }
     if (bf && !use_proj) {
       // the fusion weights, read after selection and readout (with the
       // projected values the selection kernel prefetches them, and the
@@ -822,10 +933,34 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       a.pf_ptr[a.n_prefetch] = p->W_f2;
       a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
     }
-    { KernelTimer t("score", s);
+    if (gh_in_scores) {
+      // one group: the sequence's folded keys (scores, against x_h), then the
+      // h-halves of W_f1 and W_g1 (G_h, against h)
+      const int M = mem->counts[gh_seq];
+      a.groups[0] = GemmGroup{(int)mem->offsets[gh_seq], M + 2 * H, 0, N, 0};
+      a.a_split = M; a.a_split2 = M + H;
+      a.r_by_part = 1;
+      a.epi_split = M;
+      a.out2 = gh; a.ldc2 = 2 * H;
+      if (readout != nullptr && 2 * m_sel >= mem->total) {
+        a.pf_ptr[a.n_prefetch] = mem->values;
+        a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+      }
+      KernelTimer t("score_fusion_h", s);
+      e = launch_gemm_tc(kEpiScoresFolded, a, TmaOperand{mem->folded, mem->total, d, d},
+                         TmaOperand{p->W_f1, H, d, 2 * d}, TmaOperand{xh, N, d, d},
+                         TmaOperand{h, N, d, d}, M + 2 * H, N, s, TmaOperand{p->W_g1, H, d, 2 * d});
+    } else if (use_fold) {
+      KernelTimer t("score_folded", s);
+      e = launch_gemm_tc(kEpiScoresFolded, a, TmaOperand{mem->folded, mem->total, d, d},
+                         TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
+                         TmaOperand{nullptr, 0, 0, 0}, max_m, max_r, s);
+    } else {
+      KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
                    TmaOperand{nullptr, 0, 0, 0}, TmaOperand{q, N, d, d},
-                   TmaOperand{q_lo, N, d, d}, max_m, max_r, s); }
+                   TmaOperand{q_lo, N, d, d}, max_m, max_r, s);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "score");
   }
 

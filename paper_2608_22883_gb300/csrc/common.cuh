@@ -106,6 +106,10 @@ enum EpiKind : int {
                       // rounding midpoint are listed for an exact recomputation
   kEpiQueryH = 6,     // columns < epi_split as kEpiStoreHiLo; columns >= epi_split:
                       // out2 (fp32)[row * ldc2 + col - epi_split] = acc
+  kEpiScoresFolded = 7,  // kEpiScores with one row operand (x_h against folded keys)
+                         // instead of the hi / lo pair, for columns < epi_split (row
+                         // stride min(m, epi_split)); columns >= epi_split:
+                         // out2 (fp32)[row * ldc2 + col - epi_split] = acc
 };
 
 struct KeyFix {       // one listed key element: memory row, feature
@@ -227,6 +231,10 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
 // Exact rounding of listed key elements: k = sum_l x[row, l] W[col, l]
 // evaluated in double-float, rounded once to bf16.  list == nullptr refines
 // every element of the [rows, d] key matrix.
+// out[c * rows + r] = in[r * cols + c] for a bf16 [rows, cols] matrix, rows
+// and cols multiples of 32 (the query folding's W_Q^T, once per memory build).
+cudaError_t launch_transpose_bf16(const void* in, int rows, int cols, void* out, cudaStream_t s);
+
 cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
                                const int* count, int cap, int rows, void* K, cudaStream_t s);
 cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,

@@ -14,9 +14,14 @@ __device__ __forceinline__ void gemm_epilogue(const GemmArgs& a, const GemmGroup
       static_cast<T*>(a.out0)[row * a.ldc + m] = from_f32<T>(acc);
     else
       static_cast<T*>(a.out1)[row * a.ldc + (m - a.epi_split)] = from_f32<T>(acc);
-  } else if constexpr (EPI == kEpiScores) {
+  } else if constexpr (EPI == kEpiScores || EPI == kEpiScoresFolded) {
+    if (EPI == kEpiScoresFolded && m >= a.epi_split) {
+      static_cast<float*>(a.out2)[((long long)g.b_row0 + n) * a.ldc2 + (m - a.epi_split)] = acc;
+      return;
+    }
+    const int stride = EPI == kEpiScoresFolded ? min(g.m, a.epi_split) : g.m;
     const float rs = a.row_scale ? a.row_scale[g.b_row0 + n] : 1.0f;
-    static_cast<float*>(a.out0)[g.c_off + (long long)n * g.m + m] = acc * a.scale * rs;
+    static_cast<float*>(a.out0)[g.c_off + (long long)n * stride + m] = acc * a.scale * rs;
   } else if constexpr (EPI == kEpiBiasSilu) {
     const long long row = (long long)g.b_row0 + n;
     const float bias = m < a.epi_split ? to_f32(static_cast<const T*>(a.bias0)[m])
@@ -50,9 +55,17 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
   bool vec = nv == 4;
   if constexpr (EPI == kEpiStore || EPI == kEpiBiasSilu)
     vec = vec && (m + 3 < a.epi_split || m >= a.epi_split);
-  if constexpr (EPI == kEpiScores) {
-    const long long o = g.c_off + (long long)n * g.m + m;
-    if (vec && (o & 3) == 0) {
+  if constexpr (EPI == kEpiScores || EPI == kEpiScoresFolded) {
+    if (EPI == kEpiScoresFolded && m >= a.epi_split) {
+      const long long o2 = row * a.ldc2 + (m - a.epi_split);
+      if (vec && (o2 & 3) == 0) {
+        *reinterpret_cast<float4*>(static_cast<float*>(a.out2) + o2) = make_float4(v[0], v[1], v[2], v[3]);
+        return;
+      }
+    }
+    const int stride = EPI == kEpiScoresFolded ? min(g.m, a.epi_split) : g.m;
+    const long long o = g.c_off + (long long)n * stride + m;
+    if (vec && (o & 3) == 0 && (EPI != kEpiScoresFolded || m + 3 < a.epi_split)) {
       const float rs = a.row_scale ? a.row_scale[g.b_row0 + n] : 1.0f;
       *reinterpret_cast<float4*>(static_cast<float*>(a.out0) + o) =
           make_float4(v[0] * a.scale * rs, v[1] * a.scale * rs, v[2] * a.scale * rs,

@@ -420,8 +420,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qlo = (int)rank * (BN / 4) / S, qhi = ((int)rank + 1) * (BN / 4) / S;
       const int q4 = qhi - qlo;
       const int items = rows_real * q4;
-      // two items per thread and round, all their remote loads in flight together
-      for (int it0 = threadIdx.x; it0 < items; it0 += 2 * kThreads) {
+      // two items per thread and round, all their remote loads in flight
+      // together.  The closing cluster barrier is split: each thread arrives
+      // once its last round's remote loads have been summed, before that
+      // round's global stores, so the arrival's release orders no global
+      // write; it waits after the stores.
+      const int rounds = (items + 2 * kThreads - 1) / (2 * kThreads);   // uniform in the CTA
+      for (int rd = 0; rd < rounds; ++rd) {
+        const int it0 = threadIdx.x + rd * 2 * kThreads;
         float4 t[2][8];
         int rr[2], cc[2];
 #pragma unroll
@@ -437,27 +443,39 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (sidx < S) t[k][sidx] = ld_dsmem_f4(map_dsmem(laddr, (uint32_t)sidx));
           }
         }
+        float4 acc[2];
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
           if (rr[k] < 0) continue;
-          float4 acc = t[k][0];
+          acc[k] = t[k][0];
 #pragma unroll
           for (int sidx = 1; sidx < 8; ++sidx)
             if (sidx < S) {
-              acc.x += t[k][sidx].x;
-              acc.y += t[k][sidx].y;
-              acc.z += t[k][sidx].z;
-              acc.w += t[k][sidx].w;
+              acc[k].x += t[k][sidx].x;
+              acc[k].y += t[k][sidx].y;
+              acc[k].z += t[k][sidx].z;
+              acc[k].w += t[k][sidx].w;
             }
+        }
+        if (rd == rounds - 1) {
+          __syncwarp();
+          cluster_arrive();   // this CTA's remote reads are done
+        }
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          if (rr[k] < 0) continue;
           if (ok && cc[k] < n_cols) {
-            const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+            const float vals[4] = {acc[k].x, acc[k].y, acc[k].z, acc[k].w};
             gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
                                 bias_s + cc[k]);
           }
         }
       }
-      __syncwarp();
-      cluster_sync();   // no CTA leaves while another still reads its partial tile
+      if (rounds == 0) {
+        __syncwarp();
+        cluster_arrive();
+      }
+      cluster_wait();   // no CTA leaves while another still reads its partial tile
     }
   }
   tc_fence_before();
@@ -754,6 +772,7 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
     case kEpiStoreHiLo: return plan_epi<kEpiStoreHiLo>(a, max_m, max_n);
     case kEpiStoreKeys: return plan_epi<kEpiStoreKeys>(a, max_m, max_n);
     case kEpiQueryH: return plan_epi<kEpiQueryH>(a, max_m, max_n);
+    case kEpiScoresFolded: return plan_epi<kEpiScoresFolded>(a, max_m, max_n);
     default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
   }
 }
@@ -782,6 +801,7 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
     case kEpiStoreHiLo: return launch_tc_epi<kEpiStoreHiLo>(a, maps, plan, tiles_x, max_n, s);
     case kEpiStoreKeys: return launch_tc_epi<kEpiStoreKeys>(a, maps, plan, tiles_x, max_n, s);
     case kEpiQueryH: return launch_tc_epi<kEpiQueryH>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiScoresFolded: return launch_tc_epi<kEpiScoresFolded>(a, maps, plan, tiles_x, max_n, s);
     default: return launch_tc_epi<kEpiBiasF32>(a, maps, plan, tiles_x, max_n, s);
   }
 }

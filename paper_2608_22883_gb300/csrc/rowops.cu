@@ -516,6 +516,27 @@ __global__ void __launch_bounds__(kRefineThreads) refine_keys_kernel(
   }
 }
 
+// W_Q^T for the query folding: 32 x 32 tiles through shared memory, both the
+// read and the write coalesced along rows.
+__global__ void __launch_bounds__(256) transpose_bf16_kernel(const __nv_bfloat16* __restrict__ in,
+                                                             int rows, int cols,
+                                                             __nv_bfloat16* __restrict__ out) {
+  __shared__ __nv_bfloat16 t[32][34];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int j = ty; j < 32; j += 8) t[j][tx] = in[(long long)(r0 + j) * cols + c0 + tx];
+  __syncthreads();
+  for (int j = ty; j < 32; j += 8) out[(long long)(c0 + j) * rows + r0 + tx] = t[tx][j];
+}
+
+cudaError_t launch_transpose_bf16(const void* in, int rows, int cols, void* out, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0) return cudaSuccess;
+  if (rows % 32 != 0 || cols % 32 != 0) return cudaErrorInvalidValue;
+  transpose_bf16_kernel<<<dim3(cols / 32, rows / 32), 256, 0, s>>>(
+      (const __nv_bfloat16*)in, rows, cols, (__nv_bfloat16*)out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
                                const int* count, int cap, int rows, void* K, cudaStream_t s) {
   const long long total = (long long)rows * d;

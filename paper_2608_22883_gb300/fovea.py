@@ -35,7 +35,7 @@ EXPORTS = (
     "fovea_build_memory", "fovea_memory_destroy", "fovea_memory_info", "fovea_memory_tensors",
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
-    "fovea_retrieve_fuse_noalloc", "fovea_step_path",
+    "fovea_retrieve_fuse_noalloc", "fovea_step_path", "fovea_memory_folded_keys",
 )
 NOALLOC_WORKSPACE_BYTES = 32 << 20
 PATH_AUTO, PATH_FUSED, PATH_KERNELS = 0, 1, 2
@@ -73,6 +73,7 @@ def lib() -> ctypes.CDLL:
         L.fovea_memory_info.argtypes = [vp, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int), i32p]
         L.fovea_memory_tensors.argtypes = [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp),
                                            ctypes.POINTER(ctypes.c_int64)]
+        L.fovea_memory_folded_keys.argtypes = [vp, vp, ctypes.POINTER(vp)]
         L.fovea_workspace_size.argtypes = [ctypes.POINTER(CParams), vp, i32p, ctypes.c_int,
                                            ctypes.POINTER(ctypes.c_size_t)]
         L.fovea_workspace_init.argtypes = [vp, ctypes.c_size_t, vp]
@@ -94,6 +95,7 @@ def lib() -> ctypes.CDLL:
         L.fovea_step_path.argtypes = [ctypes.c_int]
         L.fovea_step_path.restype = ctypes.c_int
         for name in ("fovea_build_memory", "fovea_memory_info", "fovea_memory_tensors",
+                     "fovea_memory_folded_keys",
                      "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse",
                      "fovea_sync_errors", "fovea_timing_enable"):
             getattr(L, name).restype = ctypes.c_int
@@ -188,6 +190,19 @@ class Memory:
             return t.view(torch.bfloat16) if self.dtype == BF16 else t
         index = torch.as_tensor(_CudaView(idx.value, (self.total,), "<i4"), device="cuda")
         return view(k.value), view(u.value), index, list(offs)
+
+    def folded_keys(self, params: Params) -> Optional[torch.Tensor]:
+        """The folded keys kappa = W_Q^T k [total, d] (bf16 view of the handle's
+        memory) when the memory holds them for params' W_Q, else None; a step
+        with these params then scores against them."""
+        f = ctypes.c_void_p()
+        _check(lib().fovea_memory_folded_keys(self.handle, params.c.W_Q, ctypes.byref(f)))
+        if not f.value:
+            return None
+        if self.total == 0:
+            return torch.empty((0, self.d), dtype=torch.bfloat16, device="cuda")
+        return torch.as_tensor(_CudaView(f.value, (self.total, self.d), "<i2"),
+                               device="cuda").view(torch.bfloat16)
 
     def destroy(self):
         if self.handle:

@@ -199,14 +199,21 @@ def run_gpu(s: Stored, fovea, params=None, memory=None):
            for k, v in out.items() if v is not None and k != "workspace"}
     res["_memory"] = mem
     res["_params"] = params
+    res["_folded"] = step_is_folded(fovea, params, mem)
     return res
 
 
-def run_oracle(s: Stored, mirror: bool, rows=None):
+def step_is_folded(fovea, params, mem) -> bool:
+    """True when a per-stage step with these params scores against the
+    memory's folded keys (the persistent step kernel never does)."""
+    return fovea.step_path() != fovea.PATH_FUSED and mem.folded_keys(params) is not None
+
+
+def run_oracle(s: Stored, mirror: bool, rows=None, fold: bool = False):
     w = s.w
     p = oracle_params(s)
     mem = oracle.build_memory(p, s.f64["v"], s.f64.get("mask"), mirror=mirror, ln_eps=LN_EPS)
     out = oracle.retrieve_fuse(p, mem, s.f64["h"], s.f64["depth"], w.row_offsets,
                                s.f64.get("row_scale"), w.rho, w.k_min, w.k_max, mirror=mirror,
-                               rows=rows, ln_eps=LN_EPS, rms_eps=RMS_EPS)
+                               rows=rows, ln_eps=LN_EPS, rms_eps=RMS_EPS, fold=fold)
     return out, mem

@@ -132,6 +132,8 @@ def test_injected_allocation_failure():
 def test_memory_queries_reject_null(L):
     assert L.fovea_memory_info(None, None, None, None) == fovea.ERR_INVALID_ARG
     assert L.fovea_memory_tensors(None, None, None, None, None) == fovea.ERR_INVALID_ARG
+    f = ctypes.c_void_p()
+    assert L.fovea_memory_folded_keys(None, None, ctypes.byref(f)) == fovea.ERR_INVALID_ARG
     n = ctypes.c_size_t()
     c = dummy_params()
     assert L.fovea_workspace_size(ctypes.byref(c), None, None, 16, ctypes.byref(n)) == fovea.ERR_INVALID_ARG

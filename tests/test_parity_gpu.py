@@ -20,7 +20,8 @@ import torch
 
 import oracle
 import workloads
-from parity import compare, params_for, rel_err_rows, run_gpu, run_oracle, store
+from parity import (compare, params_for, rel_err_rows, run_gpu, run_oracle, step_is_folded,
+                    store)
 
 pytestmark = pytest.mark.gpu
 
@@ -54,6 +55,8 @@ SMALL = {
                                      scattered_mask=True, rho=0.8, k_max=32),
     "bf16-empty-and-single": dict(d=256, m_sizes=[0, 1, 70], rows=[3, 4, 9], M_max=80, k_max=8),
     "bf16-kmax-1": dict(d=256, m_sizes=[300], rows=[33], k_max=1),
+    # one score group, after a sequence without rows: its keys start at entry 120
+    "bf16-one-group-offset": dict(d=256, m_sizes=[120, 64], rows=[0, 19], k_max=16),
     "bf16-kmax-beyond-valid": dict(d=256, m_sizes=[45, 3], rows=[10, 6], k_max=256, rho=0.99),
     "bf16-paper-defaults": dict(d=384, m_sizes=[600], rows=[40], rho=0.8, k_min=32, k_max=256),
     "bf16-fixed-top16": dict(d=256, m_sizes=[400, 250], rows=[20, 20], k_min=16, k_max=16),
@@ -83,9 +86,9 @@ def test_small_parity(fovea, path, name):
     skip_fp32_on_fused(path, w.dtype)
     s = store(w)
     gpu = run_gpu(s, fovea)
-    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
+    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"), fold=gpu["_folded"])
     rep = compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"))
-    print(f"{name}: boundary rows {rep['exempt']}, readout err {rep['readout_err']:.2e}, "
+    print(f"{name} (folded: {gpu['_folded']}): boundary rows {rep['exempt']}, readout err {rep['readout_err']:.2e}, "
           f"h_out err {rep['h_out_err']:.2e}")
 
 
@@ -102,12 +105,19 @@ def test_memory_build_matches_oracle(fovea, name):
     assert mem.valid_counts == [len(i) for i in orc.index]
     idx = idx.cpu().numpy()
     tol = 2e-2 if w.dtype == "bf16" else 1e-4
+    kappa = mem.folded_keys(params)
+    assert (kappa is not None) == (w.dtype == "bf16" and mem.total > 0)
+    if kappa is not None:
+        orc = oracle.fold_keys({n: s.f64[n] for n in workloads.PARAM_NAMES}, orc, mirror=True)
     for b in range(w.B):
         lo, hi = offs[b], offs[b + 1]
         np.testing.assert_array_equal(idx[lo:hi], orc.index[b])
         if hi == lo:
             continue
-        for got, ref in ((K, orc.keys[b]), (U, orc.values[b])):
+        pairs = [(K, orc.keys[b]), (U, orc.values[b])]
+        if kappa is not None:
+            pairs.append((kappa, orc.folded[b]))
+        for got, ref in pairs:
             g = got[lo:hi].double().cpu().numpy()
             assert rel_err_rows(g, ref).max() <= tol
             if w.dtype == "bf16":
@@ -124,11 +134,11 @@ def test_plain_fusion_when_weights_differ(fovea):
     tolerance, with identical selections."""
     w = small_workload("bf16-ragged")
     s = store(w)
-    orc, mem = run_oracle(s, mirror=True)
     params = params_for(s, fovea)
     fovea.timing_enable(True)
     proj = run_gpu(s, fovea, params=params)
     names_proj = set(fovea.timing_read())
+    orc, mem = run_oracle(s, mirror=True, fold=proj["_folded"])
     weights = {n: s.dev[n] for n in workloads.PARAM_NAMES}
     weights["W_f1"] = weights["W_f1"].clone()
     weights["W_g1"] = weights["W_g1"].clone()
@@ -140,11 +150,44 @@ def test_plain_fusion_when_weights_differ(fovea):
     fovea.timing_enable(False)
     assert "select_fuse" in names_proj and "fuse_hidden" not in names_proj
     assert "fuse_hidden" in names_plain and "select_fuse" not in names_plain
+    assert proj["_folded"] and plain["_folded"]          # same W_Q: both fold
     for gpu in (proj, plain):
         compare(gpu, orc, s, mem=mem, mirror=True)
     np.testing.assert_array_equal(proj["counts"], plain["counts"])
     np.testing.assert_array_equal(proj["indices"], plain["indices"])
     assert rel_err_rows(proj["h_out"].astype(np.float64), plain["h_out"].astype(np.float64)).max() <= 2e-2
+
+
+def test_unfolded_scores_when_memory_has_no_folded_keys(fovea):
+    """A memory built without W_Q holds no folded keys: the step then forms
+    q = W_Q x_h (hi / lo pair) and scores it against the keys, the paper's
+    own order, and matches the unfolded oracle.  A memory built with W_Q
+    scores x_h against kappa = W_Q^T k and matches the folded oracle; the
+    two agree on every non-boundary row's selection."""
+    w = small_workload("bf16-temperature")
+    s = store(w)
+    params = params_for(s, fovea)
+    no_wq = {n: s.dev[n] for n in workloads.PARAM_NAMES if n != "W_Q"}
+    build_params = fovea.Params(no_wq, d_model=w.d, mlp_hidden=w.params["b_f1"].shape[0],
+                                max_depth=w.params["E_dep"].shape[0] - 1, dtype=fovea.BF16)
+    plain_mem = fovea.build_memory(build_params, s.dev["v"], s.dev.get("mask"))
+    assert plain_mem.folded_keys(params) is None
+    fovea.timing_enable(True)
+    plain = run_gpu(s, fovea, params=params, memory=plain_mem)
+    names_plain = set(fovea.timing_read())
+    fovea.timing_enable(True)
+    folded = run_gpu(s, fovea, params=params)
+    names_folded = set(fovea.timing_read())
+    fovea.timing_enable(False)
+    assert not plain["_folded"] and folded["_folded"]
+    assert {"query_proj", "score"} <= names_plain and "score_folded" not in names_plain
+    assert {"fusion_h", "score_folded"} <= names_folded and "query_proj" not in names_folded
+    orc_p, mem_p = run_oracle(s, mirror=True, fold=False)
+    orc_f, mem_f = run_oracle(s, mirror=True, fold=True)
+    rp = compare(plain, orc_p, s, mem=mem_p, mirror=True)
+    rf = compare(folded, orc_f, s, mem=mem_f, mirror=True)
+    same = [n for n in range(w.N) if n not in rp["exempt"] and n not in rf["exempt"]]
+    np.testing.assert_array_equal(plain["counts"][same], folded["counts"][same])
 
 
 def test_paths_are_taken(fovea):
@@ -158,10 +201,17 @@ def test_paths_are_taken(fovea):
     try:
         for path, name, want, absent in (
                 (fovea.PATH_AUTO, "bf16-ragged",
-                 {"ln_query", "query_proj", "select_fuse", "fuse_out", "finalize"}, "fuse_hidden"),
-                (fovea.PATH_AUTO, "bf16-long-rows", {"select", "readout", "fuse_hidden"},
-                 "select_fuse"),
-                (fovea.PATH_AUTO, "fp32-ragged", {"select_readout", "fuse_hidden"}, "select_fuse"),
+                 {"ln_query", "fusion_h", "score_folded", "select_fuse", "fuse_out", "finalize"},
+                 "fuse_hidden"),
+                (fovea.PATH_AUTO, "bf16-paper-defaults",
+                 {"ln_query", "score_fusion_h", "select_fuse", "fuse_out", "finalize"},
+                 "fusion_h"),
+                (fovea.PATH_AUTO, "bf16-one-group-offset", {"score_fusion_h", "select_fuse"},
+                 "score_folded"),
+                (fovea.PATH_AUTO, "bf16-long-rows",
+                 {"score_folded", "select", "readout", "fuse_hidden"}, "query_proj"),
+                (fovea.PATH_AUTO, "fp32-ragged",
+                 {"query_proj", "score", "select_readout", "fuse_hidden"}, "select_fuse"),
                 (fovea.PATH_FUSED, "bf16-ragged", {"fused_step"}, "query_proj")):
             fovea.step_path(path)
             s = store(small_workload(name))
@@ -199,7 +249,7 @@ def test_planted_rows_select_one_entry(fovea, path):
     gpu = run_gpu(s, fovea)
     for row, entry in w.planted.items():
         assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
-    orc, mem = run_oracle(s, mirror=True)
+    orc, mem = run_oracle(s, mirror=True, fold=gpu["_folded"])
     compare(gpu, orc, s, mem=mem)
 
 
@@ -264,22 +314,29 @@ def test_bad_row_offsets_and_workspace(fovea, path):
 _NAMED = {}
 
 
-def _named(idx):
-    """Inputs and oracle result of a named workload, computed once for both paths."""
+def _named(idx, fold):
+    """Inputs and oracle result of a named workload, computed once per score
+    form (folded keys or the query) for both paths."""
     if idx not in _NAMED:
         w = workloads.generate(workloads.WORKLOADS[idx])
-        s = store(w)
-        orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
-        _NAMED[idx] = (w, s, orc, mem)
-    return _NAMED[idx]
+        _NAMED[idx] = (w, store(w), {})
+    w, s, orcs = _NAMED[idx]
+    if fold not in orcs:
+        orcs[fold] = run_oracle(s, mirror=(w.dtype == "bf16"), fold=fold)
+    orc, mem = orcs[fold]
+    return w, s, orc, mem
 
 
 @pytest.mark.parametrize("idx", [1, 2, 3, 4])
 def test_named_workload_parity(fovea, path, idx):
     if path == "fused" and workloads.WORKLOADS[idx].dtype != "bf16":
         pytest.skip("the persistent step kernel covers bf16 calls only")
-    w, s, orc, mem = _named(idx)
+    w = workloads.generate(workloads.WORKLOADS[idx]) if idx not in _NAMED else _NAMED[idx][0]
+    if idx not in _NAMED:
+        _NAMED[idx] = (w, store(w), {})
+    s = _NAMED[idx][1]
     gpu = run_gpu(s, fovea)
+    w, s, orc, mem = _named(idx, gpu["_folded"])
     mirror = w.dtype == "bf16"
     rep = compare(gpu, orc, s, mem=mem, mirror=mirror)
     print(f"workload {idx} ({path}): {rep}")
@@ -304,6 +361,9 @@ def test_long_memory_sampled_steps(fovea):
     seqs = [0, 3]
     p64 = {n: s0.f64[n] for n in workloads.PARAM_NAMES}
     omem = oracle.build_memory(p64, s0.f64["v"][seqs], None, mirror=True)
+    fold = step_is_folded(fovea, params, mem)
+    if fold:
+        omem = oracle.fold_keys(p64, omem, mirror=True)
     R = spec.rows_per_seq
     rng = np.random.default_rng(5)
     checked = {}
@@ -324,7 +384,7 @@ def test_long_memory_sampled_steps(fovea):
                                  v=w0.v[seqs], mask=None)
         sub = store(hw, device=None)
         orc = oracle.retrieve_fuse(p64, omem, sub.f64["h"], sub.f64["depth"], sub_offsets, None,
-                                   w0.rho, w0.k_min, w0.k_max, mirror=True)
+                                   w0.rho, w0.k_min, w0.k_max, mirror=True, fold=fold)
         g_sub = {k: v[rows] for k, v in gpu.items()}
         rep = compare(g_sub, orc, sub, mem=omem, mirror=True)
         checked[t] = rep
