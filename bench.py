@@ -464,7 +464,7 @@ def main():
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
     projected = "select_fuse" in per_kernel
-    folded = "score_folded" in per_kernel
+    folded = "score_folded" in per_kernel or "score_fusion_h" in per_kernel
     # the method's algorithmic bytes (full fusion weights, value rows), and
     # what this path's step moves (projected values: the h-half weights and
     # 2H-wide memory rows; the projection itself is part of the memory build)
