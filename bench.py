@@ -533,6 +533,11 @@ def main():
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
         "wall_s_timed_region": wall_s,
     }
+    # supplemental points (not the headline): small N and the paper's other
+    # retrieval settings, cold L2, one graph replay per step
+    if args.path != "fused":
+        out["supplemental"] = supplemental(fovea, params, mem, w, h_in, depth_in, row_scale, flush,
+                                           min(args.steps, 300))
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, rows, secs, build_s = time_oracle(w, args.cpu_seconds)
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
@@ -544,6 +549,71 @@ def main():
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def supplemental(fovea, params, mem, w, h, depth, row_scale, flush, n_steps):
+    """Per-step latency of the small-N regime (the root and its K_c = 6
+    depth-1 children of one sequence) and of the paper's other retrieval
+    settings, on the same memory and hidden states.  Each is one CUDA graph of
+    one fovea_retrieve_fuse call, timed like the main step: CUDA events on the
+    launching stream around each replay, L2 flushed before it."""
+    cases = []
+    if w.B == 1 and w.N >= 7:
+        cases.append(("small_n_7", 7, w.rho, w.k_min, w.k_max))
+    cases.append(("paper_defaults_rho0.8_kmin32_kmax256", w.N, 0.8, 32, 256))
+    cases.append(("fixed_top16", w.N, w.rho, 16, 16))
+    m_max = int(max(w.m_sizes))
+    if m_max <= 1024:
+        cases.append((f"dense_k{m_max}", w.N, 1.0, m_max, m_max))
+    stream = torch.cuda.current_stream()
+    fovea.timing_enable(False)           # plain graphs, no per-kernel event nodes
+    out = {}
+    for name, n, rho, kmin, kmax in cases:
+        if n == w.N:
+            offs = list(w.row_offsets)
+        else:
+            offs = [0, n]
+        hn, dn = h[:n].contiguous(), depth[:n].contiguous()
+        rs = row_scale[:n].contiguous() if row_scale is not None else None
+        ws = fovea.new_workspace(params, mem, offs, kmax)
+        h_out = torch.empty_like(hn)
+        counts = torch.empty(n, dtype=torch.int32, device=hn.device)
+        offs_c = fovea._offsets(offs)
+
+        def step():
+            fovea.retrieve_fuse(params, mem, hn, dn, offs, rs, rho, kmin, kmax, h_out, ws,
+                                counts=counts, offsets_c=offs_c)
+        cap = torch.cuda.Stream()
+        cap.wait_stream(stream)
+        with torch.cuda.stream(cap):
+            for _ in range(3):
+                step()
+        stream.wait_stream(cap)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap):
+            step()
+        torch.cuda.synchronize()
+        for i in range(3):
+            flush(i)
+            g.replay()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        ts = []
+        for i in range(n_steps):
+            flush(i)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        fovea.sync_errors(ws)
+        ms = float(np.mean(ts))
+        c = counts.cpu().numpy()
+        out[name] = {"draft_states": n, "rho": rho, "k_min": kmin, "k_max": kmax,
+                     "us_per_step": 1000 * ms, "value": n / (ms / 1000.0), "unit": UNIT,
+                     "mean_count": float(c.mean()), "steps": n_steps}
+    return out
 
 
 def _kernel_sha() -> str:

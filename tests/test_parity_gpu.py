@@ -61,6 +61,9 @@ SMALL = {
     "bf16-paper-defaults": dict(d=384, m_sizes=[600], rows=[40], rho=0.8, k_min=32, k_max=256),
     "bf16-fixed-top16": dict(d=256, m_sizes=[400, 250], rows=[20, 20], k_min=16, k_max=16),
     "bf16-dense": dict(d=256, m_sizes=[180], rows=[21], k_min=180, k_max=180),
+    # dense beyond 256 selected entries: the general selection (bitonic order),
+    # the readout kernel and the first fusion layer as a GEMM
+    "bf16-dense-wide": dict(d=256, m_sizes=[600], rows=[20], rho=1.0, k_min=600, k_max=600),
     "bf16-temperature": dict(d=512, m_sizes=[256, 1024, 700], rows=[32, 32, 17],
                              temperature=(0.1, 10.0), rho=0.8, k_max=128),
     "bf16-clustered": dict(d=256, m_sizes=[2048], rows=[128], clusters=16, cluster_sigma=0.2,
