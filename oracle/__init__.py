@@ -6,5 +6,5 @@ Only tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 
 from .fovea_oracle import (  # noqa: F401
     Memory, Selection, build_memory, fold_keys, fuse, layer_norm, query, query_input, readout,
-    retrieve_fuse, rms_norm, round_bf16, scores, select, sigmoid, silu,
+    lm_head_topk, retrieve_fuse, rms_norm, round_bf16, scores, select, sigmoid, silu,
 )

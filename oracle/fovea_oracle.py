@@ -48,6 +48,10 @@ may be taken against folded keys kappa_i = W_Q^T k_i formed once per image
 mirror mode kappa_i is rounded to bfloat16 (R9, the folded keys' storage)
 and x_n keeps its R3 rounding, which is what the folded bf16 path stores.
 
+The draft logits z_n = W_LM h_hat_n and their K_c largest entries
+(``lm_head_topk``) follow Eq. hidden_correction and the candidate width of
+the experimental setup; the order is by logit, ties by smaller token index.
+
 Parity pins: tests/test_oracle_pins.py (bf16 rounding against torch, LN/RMSNorm
 against torch.nn.functional, subset enumeration, closed forms, dense
 attention, fixed top-K against lexsort, gate identities).
@@ -293,3 +297,26 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
     gate[want] = f["gate"]
     out["gate"] = gate
     return out
+
+
+# ----------------------------------------------------------------------------
+# Draft logits and tree-expansion candidates (Eq. hidden_correction: z = W_LM h_hat;
+# the experimental setup's candidate width K_c)
+# ----------------------------------------------------------------------------
+
+def lm_head_topk(W_LM, h_hat, k_c) -> Dict[str, np.ndarray]:
+    """z_n = W_LM h_hat_n over the vocabulary, and the K_c candidates of each
+    row: the largest logits in descending order, ties broken by the smaller
+    token index.  Returns logits [N, V], top_idx [N, K_c], top_val [N, K_c]."""
+    W_LM = np.asarray(W_LM, dtype=F64)
+    h_hat = np.asarray(h_hat, dtype=F64)
+    z = h_hat @ W_LM.T
+    V = W_LM.shape[0]
+    k = min(int(k_c), V)
+    top_idx = np.zeros((z.shape[0], k), np.int64)
+    for n in range(z.shape[0]):
+        order = np.lexsort((np.arange(V), -z[n]))    # primary: -z ascending; then index
+        top_idx[n] = order[:k]
+    top_val = np.take_along_axis(z, top_idx, axis=1)
+    return dict(logits=z, top_idx=top_idx, top_val=top_val)
+

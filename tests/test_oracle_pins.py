@@ -519,3 +519,49 @@ def test_pins_catch_a_transposed_fold():
     n = 0
     assert not np.allclose(oracle.scores(x[n], bad.folded[0], 64), mem.keys[0] @ q[n] / 8.0,
                            rtol=1e-6)
+
+
+# ----------------------------------------------------------------------------
+# Draft logits and candidates (z = W_LM h_hat, top K_c)
+# ----------------------------------------------------------------------------
+
+def test_lm_head_logits_by_explicit_sums():
+    g = np.random.default_rng(40)
+    V, d, N = 23, 12, 4
+    W, h = g.standard_normal((V, d)), g.standard_normal((N, d))
+    out = oracle.lm_head_topk(W, h, 5)
+    for n in range(N):
+        for j in range(V):
+            want = math.fsum(W[j, i] * h[n, i] for i in range(d))
+            assert abs(out["logits"][n, j] - want) <= 1e-12 * max(1.0, abs(want))
+
+
+def test_lm_head_topk_brute_force_with_ties():
+    g = np.random.default_rng(41)
+    V, d, N, k = 40, 8, 6, 6
+    W = np.round(g.standard_normal((V, d)), 0)        # integer weights: exact ties
+    W[7] = W[3]                                       # duplicated rows tie exactly
+    W[30] = W[3]
+    h = np.round(g.standard_normal((N, d)) * 2.0, 0)
+    h[0] = 0.0                                        # every logit 0: indices 0..k-1
+    out = oracle.lm_head_topk(W, h, k)
+    for n in range(N):
+        z = [sum(W[j, i] * h[n, i] for i in range(d)) for j in range(V)]
+        want = sorted(range(V), key=lambda j: (-z[j], j))[:k]
+        assert list(out["top_idx"][n]) == want
+        assert list(out["top_val"][n]) == [z[j] for j in want]
+    assert list(out["top_idx"][0]) == list(range(k))
+
+
+def test_lm_head_one_hot_rows_closed_form():
+    # W_LM[j] = c_j e_{p(j)}: z_{n,j} = c_j h_{n,p(j)}
+    g = np.random.default_rng(42)
+    V, d = 16, 16
+    p = g.permutation(d)
+    c = np.arange(1, V + 1, dtype=np.float64)
+    W = np.zeros((V, d))
+    W[np.arange(V), p] = c
+    h = np.ones((1, d))
+    out = oracle.lm_head_topk(W, h, 3)
+    assert list(out["top_idx"][0]) == [15, 14, 13]
+    assert list(out["top_val"][0]) == [16.0, 15.0, 14.0]
