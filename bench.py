@@ -538,6 +538,9 @@ def main():
     if args.path != "fused":
         out["supplemental"] = supplemental(fovea, params, mem, w, h_in, depth_in, row_scale, flush,
                                            min(args.steps, 300))
+        if w.dtype == "bf16":
+            out["supplemental"]["lm_head_topk_v32000_k6"] = lm_head_point(
+                fovea, h_out, flush, min(args.steps, 300), peaks)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, rows, secs, build_s = time_oracle(w, args.cpu_seconds)
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
@@ -614,6 +617,54 @@ def supplemental(fovea, params, mem, w, h, depth, row_scale, flush, n_steps):
                      "us_per_step": 1000 * ms, "value": n / (ms / 1000.0), "unit": UNIT,
                      "mean_count": float(c.mean()), "steps": n_steps}
     return out
+
+
+def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=7):
+    """The draft logits and K_c candidates (fovea_lm_head_topk) on the step's
+    own h_hat: a synthetic bf16 W_LM [vocab, d] ~ N(0, 1/d), drawn on the
+    device from a seeded generator; one CUDA graph per call, L2 flushed
+    before each, CUDA events on the launching stream."""
+    N, d = h_hat.shape
+    gen = torch.Generator(device=h_hat.device)
+    gen.manual_seed(seed)
+    W = (torch.randn((vocab, d), generator=gen, device=h_hat.device) / math.sqrt(d)).to(torch.bfloat16)
+    ws = torch.zeros(1 << 14, dtype=torch.uint8, device=h_hat.device)
+    logits = torch.empty((N, vocab), dtype=torch.float32, device=h_hat.device)
+    stream = torch.cuda.current_stream()
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        for _ in range(3):
+            out = fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits)
+    stream.wait_stream(cap)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cap):
+        out = fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits)
+    torch.cuda.synchronize()
+    for i in range(3):
+        flush(i)
+        g.replay()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    ts = []
+    for i in range(n_steps):
+        flush(i)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    fovea.sync_errors(ws)
+    ms = float(np.mean(ts))
+    # algorithmic bytes: W_LM once, h_hat in, the logits out and back in for
+    # the candidate selection, the candidates out
+    nbytes = vocab * d * 2 + N * d * 2 + 2 * N * vocab * 4 + N * k_c * 8
+    gbs = nbytes / (ms / 1000.0) / 1e9
+    del W, logits, out
+    return {"vocab": vocab, "d_model": d, "draft_states": N, "k_c": k_c, "us_per_call": 1000 * ms,
+            "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"],
+            "steps": n_steps, "w_lm": "synthetic N(0, 1/d), bf16"}
 
 
 def _kernel_sha() -> str:

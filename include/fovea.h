@@ -83,6 +83,7 @@ typedef enum { FOVEA_BF16 = 0, FOVEA_FP32 = 1 } fovea_dtype;
 #define FOVEA_MAX_K 1024          /* cap K_max */
 #define FOVEA_MAX_ENTRIES 32768   /* valid entries per image */
 #define FOVEA_MAX_SEQ 512         /* sequences (images) per call */
+#define FOVEA_MAX_KC 32           /* candidate width of fovea_lm_head_topk */
 
 /* Opaque, library-owned, device-resident visual memory of B images. */
 typedef struct fovea_memory fovea_memory;
@@ -262,6 +263,27 @@ FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(const fovea_params* p, const 
                                                    int k_max, void* h_out, int32_t* counts,
                                                    int32_t* indices, float* readout, float* gate,
                                                    void* stream);
+
+/*
+ * Draft logits and tree-expansion candidates (Eq. hidden_correction,
+ * z_n = W_LM h_hat_n; the experimental setup's candidate width K_c, 6 in
+ * the paper): for every row of h_hat, the logits over the vocabulary and the
+ * k_c largest of them in descending order, ties broken by the smaller token
+ * index.
+ *   W_LM      [vocab, d_model] device, dtype, row-major (16-byte aligned)
+ *   h_hat     [N, d_model] device, dtype (e.g. fovea_retrieve_fuse's h_out)
+ *   logits    [N, vocab] device fp32, caller-owned: z (written)
+ *   top_idx   [N, k_c] device int32: token indices (written)
+ *   top_val   [N, k_c] device fp32: their logits (or NULL)
+ *   workspace an initialised step workspace (its error word; >= 16 KB)
+ * bf16 only (fp32 returns UNSUPPORTED); 1 <= k_c <= FOVEA_MAX_KC <= vocab;
+ * accumulation in fp32.  Enqueued on `stream`, no host synchronisation.
+ * Errors: INVALID_ARG, UNSUPPORTED (nothing enqueued), CUDA.
+ */
+FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_model, int dtype,
+                                          const void* h_hat, int N, int k_c, float* logits,
+                                          int32_t* top_idx, float* top_val, void* workspace,
+                                          size_t workspace_bytes, void* stream);
 
 /*
  * Implementation of the draft step (process-wide; the paper has no

@@ -1038,6 +1038,55 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   return FOVEA_OK;
 }
 
+FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_model, int dtype,
+                                          const void* h_hat, int N, int k_c, float* logits,
+                                          int32_t* top_idx, float* top_val, void* workspace,
+                                          size_t workspace_bytes, void* stream) {
+  g_last_error.clear();
+  if (dtype != FOVEA_BF16 && dtype != FOVEA_FP32)
+    return fail(FOVEA_ERR_INVALID_ARG, "dtype %d is neither FOVEA_BF16 nor FOVEA_FP32", dtype);
+  if (d_model <= 0 || d_model % 64 != 0 || d_model > FOVEA_MAX_D)
+    return fail(FOVEA_ERR_INVALID_ARG, "d_model %d must be a positive multiple of 64 (<= %d)",
+                d_model, FOVEA_MAX_D);
+  if (N < 0) return fail(FOVEA_ERR_INVALID_ARG, "N = %d < 0", N);
+  if (k_c < 1 || k_c > FOVEA_MAX_KC)
+    return fail(FOVEA_ERR_INVALID_ARG, "k_c = %d must lie in [1, %d]", k_c, FOVEA_MAX_KC);
+  if (vocab < k_c) return fail(FOVEA_ERR_INVALID_ARG, "vocab %d < k_c %d", vocab, k_c);
+  NEED_PTR(W_LM, "W_LM");
+  NEED_PTR(h_hat, "h_hat");
+  NEED_PTR(logits, "logits");
+  if (top_idx == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "top_idx is NULL");
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return fail(FOVEA_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < kWsHeaderBytes)
+    return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs at least %zu",
+                workspace_bytes, kWsHeaderBytes);
+  if (dtype != FOVEA_BF16)
+    return fail(FOVEA_ERR_UNSUPPORTED, "the LM head runs on bf16 weights and states only");
+  if (N == 0) return FOVEA_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // z = h_hat W_LM^T: W_LM [vocab, d] is the feature operand, streamed once;
+  // every column goes to the fp32 output (the G_h epilogue with its split at 0)
+  static thread_local GemmArgs a;
+  init_args(a);
+  a.k_total = d_model; a.b_split = d_model;
+  a.epi_split = 0;
+  a.out2 = logits; a.ldc2 = vocab;
+  a.err = static_cast<int*>(workspace);
+  a.ngroups = 1;
+  a.groups[0] = GemmGroup{0, vocab, 0, N, 0};
+  cudaError_t e;
+  { KernelTimer t("lm_head", s);
+    e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{W_LM, vocab, d_model, d_model},
+                       TmaOperand{nullptr, 0, 0, 0}, TmaOperand{h_hat, N, d_model, d_model},
+                       TmaOperand{nullptr, 0, 0, 0}, vocab, N, s); }
+  if (e != cudaSuccess) return cuda_fail(e, "lm_head");
+  { KernelTimer t("topk", s);
+    e = launch_topk_rows(logits, N, vocab, k_c, top_idx, top_val, s); }
+  if (e != cudaSuccess) return cuda_fail(e, "topk");
+  return FOVEA_OK;
+}
+
 FOVEA_API int fovea_step_path(int path) {
   if (path == FOVEA_PATH_AUTO || path == FOVEA_PATH_FUSED || path == FOVEA_PATH_KERNELS)
     return g_step_path.exchange(path);

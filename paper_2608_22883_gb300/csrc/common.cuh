@@ -235,6 +235,11 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
 // and cols multiples of 32 (the query folding's W_Q^T, once per memory build).
 cudaError_t launch_transpose_bf16(const void* in, int rows, int cols, void* out, cudaStream_t s);
 
+// Per row of logits [N, V] fp32: the k <= FOVEA_MAX_KC largest in
+// descending order (ties: smaller index first), indices and values.
+cudaError_t launch_topk_rows(const float* logits, int N, long long V, int k, int32_t* top_idx,
+                             float* top_val, cudaStream_t s);
+
 cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
                                const int* count, int cap, int rows, void* K, cudaStream_t s);
 cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,

@@ -36,6 +36,7 @@ EXPORTS = (
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
     "fovea_retrieve_fuse_noalloc", "fovea_step_path", "fovea_memory_folded_keys",
+    "fovea_lm_head_topk",
 )
 NOALLOC_WORKSPACE_BYTES = 32 << 20
 PATH_AUTO, PATH_FUSED, PATH_KERNELS = 0, 1, 2
@@ -74,6 +75,9 @@ def lib() -> ctypes.CDLL:
         L.fovea_memory_tensors.argtypes = [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp),
                                            ctypes.POINTER(ctypes.c_int64)]
         L.fovea_memory_folded_keys.argtypes = [vp, vp, ctypes.POINTER(vp)]
+        L.fovea_lm_head_topk.argtypes = [vp, ctypes.c_int, ctypes.c_int, ctypes.c_int, vp,
+                                         ctypes.c_int, ctypes.c_int, vp, vp, vp, vp,
+                                         ctypes.c_size_t, vp]
         L.fovea_workspace_size.argtypes = [ctypes.POINTER(CParams), vp, i32p, ctypes.c_int,
                                            ctypes.POINTER(ctypes.c_size_t)]
         L.fovea_workspace_init.argtypes = [vp, ctypes.c_size_t, vp]
@@ -95,7 +99,7 @@ def lib() -> ctypes.CDLL:
         L.fovea_step_path.argtypes = [ctypes.c_int]
         L.fovea_step_path.restype = ctypes.c_int
         for name in ("fovea_build_memory", "fovea_memory_info", "fovea_memory_tensors",
-                     "fovea_memory_folded_keys",
+                     "fovea_memory_folded_keys", "fovea_lm_head_topk",
                      "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse",
                      "fovea_sync_errors", "fovea_timing_enable"):
             getattr(L, name).restype = ctypes.c_int
@@ -302,6 +306,24 @@ def retrieve_fuse_noalloc(params: Params, memory: Memory, h: torch.Tensor, depth
 
 def sync_errors(workspace: torch.Tensor, stream=None) -> None:
     _check(lib().fovea_sync_errors(_ptr(workspace), _stream(stream)))
+
+
+def lm_head_topk(W_LM: torch.Tensor, h_hat: torch.Tensor, k_c: int, workspace: torch.Tensor,
+                 logits: Optional[torch.Tensor] = None, stream=None):
+    """fovea_lm_head_topk: z = h_hat W_LM^T [N, V] (fp32) and the k_c largest
+    logits per row (token indices, values), descending, smaller index first
+    on ties.  Returns (top_idx [N, k_c] int32, top_val [N, k_c], logits)."""
+    V, d = W_LM.shape
+    N = h_hat.shape[0]
+    dt = BF16 if W_LM.dtype == torch.bfloat16 else FP32
+    if logits is None:
+        logits = torch.empty((N, V), dtype=torch.float32, device=h_hat.device)
+    idx = torch.empty((N, k_c), dtype=torch.int32, device=h_hat.device)
+    val = torch.empty((N, k_c), dtype=torch.float32, device=h_hat.device)
+    _check(lib().fovea_lm_head_topk(_ptr(W_LM), V, d, dt, _ptr(h_hat), N, k_c, _ptr(logits),
+                                    _ptr(idx), _ptr(val), _ptr(workspace), workspace.numel(),
+                                    _stream(stream)))
+    return idx, val, logits
 
 
 def step_path(path: Optional[int] = None) -> int:

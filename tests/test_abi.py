@@ -147,3 +147,28 @@ def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(fovea, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         fovea.lib()
+
+
+def call_lm_head(L, *, W=0x10000, V=1000, d=256, dtype=fovea.BF16, h=0x10000, N=4, k_c=6,
+                 logits=0x10000, idx=0x10000, ws=0x10000, ws_bytes=1 << 20):
+    return L.fovea_lm_head_topk(W, V, d, dtype, h, N, k_c, logits, idx, None, ws, ws_bytes, None)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(k_c=0), fovea.ERR_INVALID_ARG),
+    (dict(k_c=33), fovea.ERR_INVALID_ARG),
+    (dict(V=5), fovea.ERR_INVALID_ARG),              # vocab < k_c
+    (dict(d=100), fovea.ERR_INVALID_ARG),
+    (dict(N=-1), fovea.ERR_INVALID_ARG),
+    (dict(W=None), fovea.ERR_INVALID_ARG),
+    (dict(h=0x10004), fovea.ERR_INVALID_ARG),        # misaligned
+    (dict(logits=None), fovea.ERR_INVALID_ARG),
+    (dict(idx=None), fovea.ERR_INVALID_ARG),
+    (dict(ws=0x10010), fovea.ERR_INVALID_ARG),       # not 256-byte aligned
+    (dict(ws_bytes=1024), fovea.ERR_INVALID_ARG),
+    (dict(dtype=7), fovea.ERR_INVALID_ARG),
+    (dict(dtype=fovea.FP32), fovea.ERR_UNSUPPORTED),
+])
+def test_lm_head_argument_checks(L, kw, status):
+    assert call_lm_head(L, **kw) == status
+    assert fovea.last_error() != ""

@@ -1,0 +1,88 @@
+"""Draft logits and candidates through the C ABI (fovea_lm_head_topk) against
+the oracle: z = W_LM h_hat (Eq. hidden_correction) and the K_c largest logits
+per row, descending, smaller token index first on ties.
+
+Logits are compared with a bound derived from fp32 accumulation of bf16
+products; candidate lists match the oracle's exactly except where two
+oracle logits lie within that bound of each other (a near-tie), where the
+GPU's entry must lie inside the band around the oracle's."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def fovea():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2608_22883_gb300 import fovea as f
+    f.lib()
+    return f
+
+
+def bf16(x):
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16)
+
+
+def check(fovea, V, d, N, k_c, seed, ties=False):
+    g = np.random.default_rng(seed)
+    W = g.standard_normal((V, d)) / np.sqrt(d)
+    h = g.standard_normal((N, d))
+    if ties:
+        W[V // 2] = W[3]                      # duplicated vocabulary rows tie exactly
+        W[V - 1] = W[3]
+    Wt, ht = bf16(W).cuda(), bf16(h).cuda()
+    W64 = Wt.double().cpu().numpy()
+    h64 = ht.double().cpu().numpy()
+    ws = torch.zeros(1 << 14, dtype=torch.uint8, device="cuda")
+    idx, val, logits = fovea.lm_head_topk(Wt, ht, k_c, ws)
+    torch.cuda.synchronize()
+    fovea.sync_errors(ws)
+    ref = oracle.lm_head_topk(W64, h64, k_c)
+    z_ref = ref["logits"]
+    z = logits.cpu().numpy().astype(np.float64)
+    # fp32 accumulation of d exact bf16 products: |error| <= d * 2^-24 * sum |w h|
+    bound = d * 2.0 ** -24 * (np.abs(h64) @ np.abs(W64).T) + 1e-30
+    assert np.all(np.abs(z - z_ref) <= bound), np.max(np.abs(z - z_ref) / bound)
+    idx = idx.cpu().numpy()
+    val = val.cpu().numpy().astype(np.float64)
+    for n in range(N):
+        band = 2 * bound[n].max()
+        for r in range(k_c):
+            gi, oi = int(idx[n, r]), int(ref["top_idx"][n, r])
+            if gi != oi:
+                assert abs(z_ref[n, gi] - z_ref[n, oi]) <= band, (n, r, gi, oi)
+            assert val[n, r] == np.float32(z[n, gi])
+        assert len(set(idx[n].tolist())) == k_c
+        assert np.all(np.diff(val[n]) <= 0)
+    return idx
+
+
+@pytest.mark.parametrize("V,d,N,k_c,seed", [
+    (1000, 256, 37, 6, 1),       # ragged feature tiles and a ragged row tile
+    (777, 320, 5, 32, 2),        # the widest candidate list
+    (4099, 192, 130, 1, 3),      # argmax; rows over two row tiles
+    (50, 64, 1, 6, 4),           # one row, a vocabulary smaller than a tile
+])
+def test_lm_head_topk_matches_oracle(fovea, V, d, N, k_c, seed):
+    check(fovea, V, d, N, k_c, seed)
+
+
+def test_lm_head_exact_ties_take_the_smaller_index(fovea):
+    # rows 3, V/2 and V-1 of W_LM are equal: whenever one of them is among the
+    # candidates, so are the others in index order (equal logits, equal keys)
+    V, d, N = 600, 128, 24
+    idx = check(fovea, V, d, N, 32, 5, ties=True)
+    for n in range(N):
+        lst = idx[n].tolist()
+        pos = [lst.index(j) for j in (3, V // 2, V - 1) if j in lst]
+        assert pos == sorted(pos)
+
+
+def test_lm_head_vicuna_sized(fovea):
+    # a 32000-token vocabulary over d = 4096, 64 draft states, K_c = 6
+    check(fovea, 32000, 4096, 64, 6, 6)
