@@ -490,7 +490,7 @@ def main():
             with open(tpath) as f:
                 tr = json.load(f)
             ent = tr.get(w.name, {}).get(dom)
-            if ent and ent.get("kernel_sha") == _kernel_sha():
+            if ent and ent.get("kernel_sha") == _kernel_sha(ent.get("files")):
                 traffic = ent["bytes_per_launch"]
         except Exception:
             traffic = None
@@ -667,12 +667,16 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
             "steps": n_steps, "w_lm": "synthetic N(0, 1/d), bf16"}
 
 
-def _kernel_sha() -> str:
+def _kernel_sha(files=None) -> str:
+    """Hash of the sources a kernel is built and launched from (paths relative
+    to the repository root; default: every file of csrc/)."""
     import hashlib
     hsh = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_22883_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, f), "rb") as fh:
+    paths = ([os.path.join(ROOT, f) for f in files] if files
+             else [os.path.join(csrc, f) for f in sorted(os.listdir(csrc))])
+    for path in paths:
+        with open(path, "rb") as fh:
             hsh.update(fh.read())
     return hsh.hexdigest()[:16]
 

@@ -11,6 +11,7 @@ namespace fovea {
 namespace {
 
 constexpr int kTopKThreads = 256;    // registers: up to FOVEA_MAX_KC 64-bit keys per thread
+constexpr int kBatch = 16;           // logits loaded together per thread
 
 // Order-preserving map of a float to an unsigned key (larger float, larger key).
 __device__ __forceinline__ uint32_t logit_key(float f) {
@@ -43,21 +44,34 @@ __global__ void __launch_bounds__(kTopKThreads) topk_rows_kernel(const float* __
   for (int i = 0; i < KC; ++i) loc[i] = 0ull;
   unsigned long long lowest = 0ull;           // the smallest of slots 0 .. k-1
   int low_pos = 0;
-  for (long long j = tid; j < V; j += kTopKThreads) {
-    const unsigned long long key =
-        ((unsigned long long)logit_key(z[j]) << 32) | (0xFFFFFFFFu - (uint32_t)j);
-    if (key <= lowest) continue;
+  // the thread's logits in batches of kBatch, every load of a batch in
+  // flight before the first comparison
+  for (long long j0 = tid; j0 < V; j0 += (long long)kBatch * kTopKThreads) {
+    float v[kBatch];
 #pragma unroll
-    for (int i = 0; i < KC; ++i)
-      if (i == low_pos) loc[i] = key;
-    lowest = loc[0];
-    low_pos = 0;
+    for (int u = 0; u < kBatch; ++u) {
+      const long long j = j0 + (long long)u * kTopKThreads;
+      v[u] = j < V ? z[j] : 0.0f;
+    }
 #pragma unroll
-    for (int i = 1; i < KC; ++i)
-      if (i < k && loc[i] < lowest) {
-        lowest = loc[i];
-        low_pos = i;
-      }
+    for (int u = 0; u < kBatch; ++u) {
+      const long long j = j0 + (long long)u * kTopKThreads;
+      if (j >= V) continue;
+      const unsigned long long key =
+          ((unsigned long long)logit_key(v[u]) << 32) | (0xFFFFFFFFu - (uint32_t)j);
+      if (key <= lowest) continue;
+#pragma unroll
+      for (int i = 0; i < KC; ++i)
+        if (i == low_pos) loc[i] = key;
+      lowest = loc[0];
+      low_pos = 0;
+#pragma unroll
+      for (int i = 1; i < KC; ++i)
+        if (i < k && loc[i] < lowest) {
+          lowest = loc[i];
+          low_pos = i;
+        }
+    }
   }
   for (int r = 0; r < k; ++r) {
     unsigned long long mine = loc[0];
