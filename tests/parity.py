@@ -2,7 +2,8 @@
 and the CPU oracle on the same stored inputs, and compare them under the
 exactness / tolerance rules.
 
-Rules (the spec contract, with the boundary exemption spelled out):
+Rules (exact where the path decides an integer, bounded where it rounds, with
+the boundary exemption spelled out):
 * counts and selected index sets are bit-exact, except rows where the
   oracle's cumulative mass at the decision lies within 1e-4 of rho, or where
   the cut falls inside a score tie band (K-th and (K+1)-th scores within
