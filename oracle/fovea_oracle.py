@@ -48,6 +48,11 @@ may be taken against folded keys kappa_i = W_Q^T k_i formed once per image
 mirror mode kappa_i is rounded to bfloat16 (R9, the folded keys' storage)
 and x_n keeps its R3 rounding, which is what the folded bf16 path stores.
 
+Depth gate (``l_max`` in ``retrieve_fuse``; the experimental setup applies
+the visual correction only to nodes of depth at most 1): a draft state whose
+depth exceeds l_max is not corrected, so its scoring representation is h_n
+itself, with no retrieval (count 0, no indices, r = 0, gate 0).
+
 The draft logits z_n = W_LM h_hat_n and their K_c largest entries
 (``lm_head_topk``) follow Eq. hidden_correction and the candidate width of
 the experimental setup; the order is by logit, ties by smaller token index.
@@ -251,25 +256,30 @@ def fuse(p, h, r, *, mirror=False, rms_eps=1e-6):
 
 def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
                   k_max, *, mirror=False, ln_eps=1e-5, rms_eps=1e-6,
-                  rows=None, fold=False) -> Dict[str, object]:
+                  rows=None, fold=False, l_max=None) -> Dict[str, object]:
     """Retrieve + fuse for every draft state; rows row_offsets[b] ..
     row_offsets[b+1]-1 query image b.  ``rows`` restricts the computation to a
     subset of row indices (the rest of the outputs stay zero / -1).
     ``fold`` scores x_n against the folded keys (``fold_keys``) instead of
-    q_n against the keys."""
+    q_n against the keys.  ``l_max``: rows deeper than l_max are not
+    corrected (h_out = h, no retrieval); None corrects every row."""
     h = np.asarray(h, dtype=F64)
     N, d = h.shape
     rho = float(np.float32(rho))
     row_offsets = np.asarray(row_offsets)
     want = np.arange(N) if rows is None else np.asarray(sorted(rows))
+    gated = np.zeros(N, bool)
+    if l_max is not None:
+        gated = np.asarray(depth) > l_max
+    keep = want[~gated[want]] if len(want) else want
     seq_of = np.searchsorted(row_offsets, np.arange(N), side="right") - 1
     q = np.zeros((N, d))
     x = np.zeros((N, d))
     if fold and mem.folded is None:
-        mem = fold_keys(p, mem, mirror=mirror, images={int(seq_of[n]) for n in want})
-    if len(want):
-        x[want] = query_input(p, h[want], np.asarray(depth)[want], mirror=mirror, ln_eps=ln_eps)
-        q[want] = x[want] @ p["W_Q"].T
+        mem = fold_keys(p, mem, mirror=mirror, images={int(seq_of[n]) for n in keep})
+    if len(keep):
+        x[keep] = query_input(p, h[keep], np.asarray(depth)[keep], mirror=mirror, ln_eps=ln_eps)
+        q[keep] = x[keep] @ p["W_Q"].T
     counts = np.zeros(N, np.int64)
     k_raw = np.zeros(N, np.int64)
     indices = -np.ones((N, k_max), np.int64)
@@ -277,7 +287,7 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
     sel: List[Optional[Selection]] = [None] * N
     sc: List[Optional[np.ndarray]] = [None] * N
     alphas: List[Optional[np.ndarray]] = [None] * N
-    for n in want:
+    for n in keep:
         b = int(seq_of[n])
         scale = 1.0 if row_scale is None else float(row_scale[n])
         s = scores(x[n], mem.folded[b], d, scale) if fold else scores(q[n], mem.keys[b], d, scale)
@@ -287,14 +297,16 @@ def retrieve_fuse(p, mem: Memory, h, depth, row_offsets, row_scale, rho, k_min,
         indices[n, :S.K] = mem.index[b][S.selected]
         sel[n], sc[n] = S, s
     out = dict(q=q, counts=counts, k_raw=k_raw, indices=indices, readout=r,
-               selections=sel, scores=sc, alphas=alphas, seq_of=seq_of)
-    f = fuse(p, h[want], r[want], mirror=mirror, rms_eps=rms_eps)
+               selections=sel, scores=sc, alphas=alphas, seq_of=seq_of, gated=gated)
+    f = fuse(p, h[keep], r[keep], mirror=mirror, rms_eps=rms_eps)
     for key in ("a_f", "a_g", "c", "y", "h_out"):
         full = np.zeros((N,) + f[key].shape[1:])
-        full[want] = f[key]
+        full[keep] = f[key]
         out[key] = full
+    skipped = want[gated[want]] if len(want) else want
+    out["h_out"][skipped] = h[skipped]          # not corrected: h_hat = h
     gate = np.zeros(N)
-    gate[want] = f["gate"]
+    gate[keep] = f["gate"]
     out["gate"] = gate
     return out
 

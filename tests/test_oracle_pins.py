@@ -316,6 +316,30 @@ def test_unit_gate_and_zero_correction():
     np.testing.assert_allclose(out0["h_out"], want, rtol=1e-12, atol=1e-12)
 
 
+def test_depth_gate_leaves_deep_rows_uncorrected():
+    """The experimental setup applies the visual correction to nodes of depth
+    at most 1: with l_max = 1 a deeper row keeps h_n itself as its scoring
+    representation and retrieves nothing, every other row is what the
+    ungated step gives, and l_max = D gates nothing."""
+    p = small_params()
+    v, mask, h, _, offs = small_step(p, seed=21, M=(30, 9), rows=(6, 5))
+    depth = np.array([0, 1, 2, 6, 1, 3, 0, 1, 5, 2, 4])
+    mem = oracle.build_memory(p, v, mask)
+    full = oracle.retrieve_fuse(p, mem, h, depth, offs, None, 0.9, 1, 8)
+    gated = oracle.retrieve_fuse(p, mem, h, depth, offs, None, 0.9, 1, 8, l_max=1)
+    deep = depth > 1
+    np.testing.assert_array_equal(gated["h_out"][deep], h[deep])     # the input itself
+    assert np.all(gated["counts"][deep] == 0) and np.all(gated["indices"][deep] == -1)
+    assert np.all(gated["gate"][deep] == 0.0) and np.all(gated["readout"][deep] == 0.0)
+    np.testing.assert_array_equal(gated["counts"][~deep], full["counts"][~deep])
+    np.testing.assert_array_equal(gated["indices"][~deep], full["indices"][~deep])
+    for key in ("readout", "h_out", "gate"):
+        np.testing.assert_allclose(gated[key][~deep], full[key][~deep], rtol=1e-12, atol=1e-14)
+    same = oracle.retrieve_fuse(p, mem, h, depth, offs, None, 0.9, 1, 8, l_max=6)
+    np.testing.assert_array_equal(same["indices"], full["indices"])
+    np.testing.assert_allclose(same["h_out"], full["h_out"], rtol=1e-12, atol=1e-14)
+
+
 def test_step_matches_composition_of_torch_pieces():
     """The whole step re-derived with torch ops row by row: query, scores with
     row scale, selection (python sort), softmax over the selected, readout, and
