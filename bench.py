@@ -63,13 +63,14 @@ def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, pr
     memory's projected values p_i = [W_f1 ; W_g1]_r u_i (2H wide) instead of
     the values, and only the h-half of the first fusion layer's weights.
     `folded`: the step scores x_h against the memory's folded keys
-    W_Q^T k_i (formed with the memory), so W_Q is not read and q not formed."""
+    W_Q^T k_i (formed with the memory, a hi / lo pair of bf16 values, so
+    twice the key bytes), and W_Q is not read and q not formed."""
     d, H, N = w.d, w.params["b_f1"].shape[0], w.N
     es = 2 if w.dtype == "bf16" else 4
     fuse1 = 2 * H * (d if projected else 2 * d)
     weights = (0 if folded else d * d) + fuse1 + d * H + H + 2 * H + d + H + 1 + d   # W_Q, W_f1/W_g1, W_f2, biases, rms
     weights += 2 * d + 2 * d      # LN_h gamma/beta + the E_dep rows touched (bound: 2 rows)
-    keys = sum(w.m_sizes) * d
+    keys = sum(w.m_sizes) * d * (2 if folded else 1)
     uniq = 0
     for b in range(w.B):
         lo, hi = int(w.row_offsets[b]), int(w.row_offsets[b + 1])
@@ -100,10 +101,10 @@ def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: 
         return es * (d * d + N * d + 2 * N * d)
     if name == "fusion_h":        # the h-half of [W_f1 ; W_g1]; h in; G_h out
         return es * (2 * H * d + N * d) + 4 * N * 2 * H
-    if name == "score_fusion_h":  # folded keys, the h-half of [W_f1 ; W_g1], x_h and h in; scores, G_h out
-        return (sum(w.m_sizes) * d + 2 * H * d + 2 * N * d) * es + scores + 4 * N * 2 * H
-    if name == "score_folded":    # folded keys, x_h in; scores out
-        return sum(w.m_sizes) * d * es + N * d * es + scores
+    if name == "score_fusion_h":  # folded keys (hi, lo), the h-half of [W_f1 ; W_g1], x_h and h in; scores, G_h out
+        return (2 * sum(w.m_sizes) * d + 2 * H * d + 2 * N * d) * es + scores + 4 * N * 2 * H
+    if name == "score_folded":    # folded keys (hi, lo), x_h in; scores out
+        return 2 * sum(w.m_sizes) * d * es + N * d * es + scores
     if name == "fuse_hidden":
         return es * (2 * H * 2 * d + 2 * N * d + N * 2 * H + 2 * H)
     if name == "fuse_out":
@@ -239,6 +240,11 @@ def max_over_ranks(value: float, dist, device) -> float:
 
 
 def run_reference(args, w):
+    """The reference arm: the CPU oracle as it stands, timed on this host's
+    cores on the GPU arm's workload.  A step is an oracle retrieve+fuse over
+    the workload's draft states (the memory is built once, untimed); when
+    --steps such steps would take more than about two minutes, each step
+    covers an evenly strided sample of the rows instead, and the line says so."""
     import oracle
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -248,29 +254,49 @@ def run_reference(args, w):
     mem = oracle.build_memory(p, v, w.mask, mirror=mirror, ln_eps=float(np.float32(1e-5)))
     eps = dict(ln_eps=float(np.float32(1e-5)), rms_eps=float(np.float32(1e-6)))
 
-    def one(i):
-        n = i % w.N
+    def one(rows):
         oracle.retrieve_fuse(p, mem, h, w.depth, w.row_offsets, w.row_scale, w.rho, w.k_min,
-                             w.k_max, mirror=mirror, rows=[n], **eps)
-    for i in range(args.warmup):
-        one(i)
+                             w.k_max, mirror=mirror, rows=rows, **eps)
+    t0 = time.perf_counter()
+    one(None)                                   # first warm-up step: all rows, to size the sample
+    t_full = time.perf_counter() - t0
+    rows_per_step = w.N
+    budget_s = 120.0
+    if t_full * args.steps > budget_s:
+        rows_per_step = max(1, int(w.N * budget_s / (t_full * args.steps)))
+    stride = max(1, w.N // rows_per_step)
+
+    def rows_of(i):
+        if rows_per_step >= w.N:
+            return None
+        return sorted({(i + j * stride) % w.N for j in range(rows_per_step)})
+    for i in range(1, args.warmup):
+        one(rows_of(i))
     t0 = time.perf_counter()
     for i in range(args.steps):
-        one(args.warmup + i)
+        one(rows_of(args.warmup + i))
     el = time.perf_counter() - t0
-    value = args.steps / el
-    sample = f"one draft state per step (cycling the {w.N} rows), memory built once (excluded)"
+    value = rows_per_step * args.steps / el
+    sample = (f"every step the whole {w.N}-row batch" if rows_per_step >= w.N else
+              f"every step {rows_per_step} of the {w.N} rows (strided, rotating), the whole "
+              f"batch taking {t_full:.2f} s")
+    sample += "; memory built once (excluded)"
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": 1000 * el / args.steps, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "impl": "reference",
-           "config": {"workload": w.name, "d_model": w.d, "memory_entries": w.m_sizes,
-                      "draft_states": w.N, "rho": w.rho, "k_max": w.k_max},
+           "config": workload_config(w),
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                             "sample": sample},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
     return 0
+
+
+def workload_config(w: workloads.Workload) -> dict:
+    return {"workload": w.name, "d_model": w.d, "memory_entries": [int(m) for m in w.m_sizes],
+            "draft_states": w.N, "sequences": w.B, "rho": w.rho, "k_min": w.k_min,
+            "k_max": w.k_max, "mlp_hidden": int(w.params["b_f1"].shape[0])}
 
 
 # ---------------------------------------------------------------------------
@@ -286,9 +312,7 @@ def main():
     ap.add_argument("--workload", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--path", default="auto", choices=["auto", "fused", "kernels"],
-                    help="draft-step implementation: the library default (auto), the persistent "
-                         "step kernel (fused) or one kernel per stage (kernels)")
+    ap.add_argument("--no-supplemental", action="store_true")
     args = ap.parse_args()
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
@@ -298,8 +322,6 @@ def main():
         return run_reference(args, w)
 
     from paper_2608_22883_gb300 import fovea
-    fovea.step_path({"auto": fovea.PATH_AUTO, "fused": fovea.PATH_FUSED,
-                     "kernels": fovea.PATH_KERNELS}[args.path])
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -324,11 +346,15 @@ def main():
     depth = depth_host.to(dev)
     row_scale = torch.from_numpy(w.row_scale).to(dev) if w.row_scale is not None else None
 
+    # the memory build (once per image batch), timed with its per-kernel events
     torch.cuda.synchronize()
+    fovea.timing_enable(True)
     t0 = time.perf_counter()
     mem = fovea.build_memory(params, v, mask)
     torch.cuda.synchronize()
     build_ms = 1000 * (time.perf_counter() - t0)
+    build_kernels = {k: {"ms": t, "launches": n} for k, (t, n) in fovea.timing_read().items()}
+    fovea.timing_enable(False)
 
     N, d, K = w.N, w.d, w.k_max
     ws = fovea.new_workspace(params, mem, w.row_offsets, K)
@@ -355,6 +381,7 @@ def main():
     depth_in_host.copy_(depth_host)
     h_in.copy_(h)
     depth_in.copy_(depth)
+    out_host, (h_out_host, counts_host, idx_host) = packed(out_parts, "cpu", pin=True)
 
     def step():
         fovea.retrieve_fuse(params, mem, h_in, depth_in, w.row_offsets, row_scale, w.rho, w.k_min,
@@ -366,64 +393,66 @@ def main():
         flush_w.fill_(i & 0xFF)
         flush_r.sum()
 
-    # The step is replayed from a CUDA graph (one launch per step), the form a
-    # decoding loop uses; the graph holds exactly the kernels of one call.
+    stream = torch.cuda.current_stream()
+    # The step is timed in two forms: one CUDA-graph replay per step (the
+    # form a decoding loop captures), and the plain API call (its kernels
+    # enqueued by fovea_retrieve_fuse itself, the host work overlapping the
+    # L2 flush before it).  The headline takes the plain call.
     cap = torch.cuda.Stream()
-    cap.wait_stream(torch.cuda.current_stream())
+    cap.wait_stream(stream)
     with torch.cuda.stream(cap):
         for _ in range(3):
             step()
-    torch.cuda.current_stream().wait_stream(cap)
+    stream.wait_stream(cap)
     torch.cuda.synchronize()
     g_plain = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_plain, stream=cap):
         step()
-    # end to end: the host inputs copied in, the step, the results copied
-    # back, as one graph (pinned host buffers)
-    out_host, (h_out_host, counts_host, idx_host) = packed(out_parts, "cpu", pin=True)
+    # end to end as a graph: the host inputs copied in, the step, the results
+    # copied back (pinned host buffers)
     g_e2e = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_e2e, stream=cap):
         in_dev.copy_(in_host, non_blocking=True)
         step()
         out_host.copy_(out_dev, non_blocking=True)
-    fovea.timing_enable(True)            # per-kernel event nodes in the timed graph
-    g_timed = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_timed, stream=cap):
-        step()
     torch.cuda.synchronize()
-    stream = torch.cuda.current_stream()
 
-    for i in range(args.warmup):
-        flush(i)
-        g_timed.replay()
-    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+
+    def timed(run, n, seed):
+        ts = []
+        for i in range(n):
+            flush(seed + i)
+            e0.record(stream)
+            run()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return ts
+
+    timed(step, args.warmup, 0)
+    timed(g_plain.replay, args.warmup, 0)
     fovea.sync_errors(ws)
 
-    # ---- timed region: K steps (graph replays), L2 flushed before each ----
+    # ---- timed region: K steps (plain API calls), L2 flushed before each ----
     clocks = ClockSampler(local)
     clocks.start()
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    step_ms = []
     t_wall = time.perf_counter()
-    for i in range(args.steps):
-        flush(i + 7)
-        e0.record(stream)
-        g_plain.replay()
-        e1.record(stream)
-        e1.synchronize()
-        step_ms.append(e0.elapsed_time(e1))
+    step_ms = timed(step, args.steps, 7)
     torch.cuda.synchronize()
     wall_s = time.perf_counter() - t_wall
+    graph_ms_l = timed(g_plain.replay, min(args.steps, 500), 11)
     if dist is not None:
         dist.barrier()
     clk = clocks.stop()
     ms = float(np.mean(step_ms))
     fovea.sync_errors(ws)
     ms = max_over_ranks(ms, dist, dev)
+    graph_ms = max_over_ranks(float(np.mean(graph_ms_l)), dist, dev)
     value = world * N / (ms / 1000.0)
 
     # ---- kernel-timing pass: the same step with an event pair around every
@@ -432,6 +461,11 @@ def main():
     n_kt = min(args.steps, 500)
     per_kernel = {}
     kt_ms = []
+    fovea.timing_enable(True)            # per-kernel event nodes in the timed graph; kept
+    g_timed = torch.cuda.CUDAGraph()     # enabled while the graph is replayed
+    with torch.cuda.graph(g_timed, stream=cap):
+        step()
+    torch.cuda.synchronize()
     for i in range(n_kt):
         flush(i)
         e0.record(stream)
@@ -444,22 +478,37 @@ def main():
             a[0] += tot
             a[1] += n
     ms_hooks = float(np.mean(kt_ms))
-    n_plain = n_kt
 
     # ---- end to end: host buffers in, the step, results back to host (one
     # graph: the copies are memcpy nodes around the step's kernels) ----
-    e2e_ms_l = []
-    for i in range(n_plain):
-        flush(i)
-        e0.record(stream)
-        g_e2e.replay()
-        e1.record(stream)
-        e1.synchronize()
-        e2e_ms_l.append(e0.elapsed_time(e1))
+    fovea.timing_enable(False)
+    e2e_ms_l = timed(g_e2e.replay, n_kt, 3)
     e2e_ms = max_over_ranks(float(np.mean(e2e_ms_l)), dist, dev)
     h2d = in_host.numel()
     d2h = out_host.numel()
     assert torch.equal(h_out_host, h_out.cpu())
+    # ---- the public API call end to end on the host clock: copy the inputs
+    # in, call fovea_retrieve_fuse (argument checks, planning, launches),
+    # copy the outputs back, synchronise; no graph, no L2 flush ----
+    wall_l = []
+    for i in range(min(args.steps, 300) + 3):
+        t0 = time.perf_counter()
+        in_dev.copy_(in_host, non_blocking=True)
+        step()
+        out_host.copy_(out_dev, non_blocking=True)
+        stream.synchronize()
+        if i >= 3:
+            wall_l.append(time.perf_counter() - t0)
+    api_wall_ms = 1000 * float(np.median(wall_l))
+    api_host_l = []
+    for i in range(200):             # host time of the call alone (the GPU catches up after)
+        t0 = time.perf_counter()
+        step()
+        api_host_l.append(time.perf_counter() - t0)
+        if i % 16 == 15:
+            stream.synchronize()
+    stream.synchronize()
+    api_host_us = 1e6 * float(np.median(api_host_l))
 
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
@@ -467,7 +516,7 @@ def main():
     folded = "score_folded" in per_kernel or "score_fusion_h" in per_kernel
     # the method's algorithmic bytes (full fusion weights, value rows), and
     # what this path's step moves (projected values: the h-half weights and
-    # 2H-wide memory rows; the projection itself is part of the memory build)
+    # 2H-wide memory rows; folded keys: no W_Q, hi / lo keys)
     nbytes, flops, uniq = step_cost(w, c_np, i_np, False)
     nbytes_path, flops_path, _ = step_cost(w, c_np, i_np, projected, folded)
     peaks, peak_src = load_peaks()
@@ -477,8 +526,7 @@ def main():
     t_roof_path = max(nbytes_path / (peaks["hbm_gbs"] * 1e9), flops_path / (peaks["bf16_tflops"] * 1e12))
     kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
     dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
-    # the persistent step kernel moves the whole step's algorithmic bytes
-    dom_bytes = nbytes if dom == "fused_step" else kernel_bytes(dom, w, uniq, projected)
+    dom_bytes = kernel_bytes(dom, w, uniq, projected)
     achieved = dom_bytes / (kern[dom]["ms_avg"] / 1000.0) / 1e9
     launches_per_step = sum(k["launches"] for k in kern.values()) / max(n_kt, 1)
     launches = int(round(launches_per_step * args.steps))
@@ -495,19 +543,16 @@ def main():
         except Exception:
             traffic = None
 
+    cfg = workload_config(w)
+    cfg.update({"l2": "flushed before every step outside the per-step events (512 MB write, then a 256 MB read so the evicted lines are clean)",
+                "launch": f"one fovea_retrieve_fuse call per step ({len(kern)} kernels, programmatic "
+                          "dependent launch between them)",
+                "parallelism": f"replicas x{world}"})
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-        "config": {"workload": w.name, "d_model": w.d, "memory_entries": w.m_sizes,
-                   "draft_states": N, "sequences": w.B, "rho": w.rho, "k_min": w.k_min,
-                   "k_max": K, "mlp_hidden": int(w.params["b_f1"].shape[0]),
-                   "l2": "flushed before every step outside the per-step events (512 MB write, then a 256 MB read so the evicted lines are clean)",
-                   "launch": "one CUDA graph replay per step (the kernels of one fovea_retrieve_fuse call: "
-                             + ("one persistent cooperative kernel)" if list(kern) == ["fused_step"]
-                                else f"{len(kern)} kernels)"),
-                   "path": args.path,
-                   "parallelism": f"replicas x{world}"},
+        "config": cfg,
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved,
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
                      "traffic": traffic, "algorithmic_bytes": dom_bytes,
@@ -521,24 +566,35 @@ def main():
                                         "frac": t_roof_path / (ms / 1000.0),
                                         "projected_values": projected,
                                         "folded_keys": folded},
-
                           "peaks": f"{peak_src}: {peaks['hbm_gbs']} GB/s, {peaks['bf16_tflops']} TF/s"},
-        "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"]} for k, v in kern.items()},
+        "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"],
+                        "algorithmic_bytes": kernel_bytes(k, w, uniq, projected),
+                        "gbs": kernel_bytes(k, w, uniq, projected) / (v["ms_avg"] / 1000.0) / 1e9}
+                    for k, v in kern.items()},
+        "ms_per_step_graph_replay": graph_ms,
         "ms_per_step_kernel_timing_pass": ms_hooks,
         "kernel_ms_per_step": total_kernel_ms / max(n_kt, 1),
         "gpu_launches": launches,
         "memory_build_ms": build_ms,
+        "memory_build_kernels": build_kernels,
         "clocks": clk,
         "e2e": {"value": world * N / (e2e_ms / 1000.0), "unit": UNIT, "ms_per_step": e2e_ms,
-                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                "form": "one CUDA graph per step: input copy from pinned host memory, the step, "
+                        "output copy back; CUDA events on the launching stream"},
+        "api_call_host_clock": {"value": world * N / (api_wall_ms / 1000.0), "unit": UNIT,
+                                "ms_per_step": api_wall_ms, "host_us_per_call": api_host_us,
+                                "form": "per step on the host clock: input copy in, "
+                                        "fovea_retrieve_fuse through the Python binding, output "
+                                        "copy back, stream synchronise (median)"},
         "wall_s_timed_region": wall_s,
     }
     # supplemental points (not the headline): small N and the paper's other
-    # retrieval settings, cold L2, one graph replay per step
-    if args.path != "fused":
+    # retrieval settings, cold L2, one plain call per step
+    if not args.no_supplemental:
         out["supplemental"] = supplemental(fovea, params, mem, w, h_in, depth_in, row_scale, flush,
                                            min(args.steps, 300))
-        if w.dtype == "bf16":
+        if w.dtype == "bf16" and w.B == 1:
             out["supplemental"]["lm_head_topk_v32000_k6"] = lm_head_point(
                 fovea, h_out, flush, min(args.steps, 300), peaks)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -554,28 +610,45 @@ def main():
     return 0
 
 
+def _time_calls(call, flush, n_steps, warm=3):
+    """Mean CUDA-event time (ms) of `call` on the current stream, L2 flushed
+    before each, after `warm` untimed calls."""
+    stream = torch.cuda.current_stream()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    for i in range(warm):
+        flush(i)
+        call()
+    ts = []
+    for i in range(n_steps):
+        flush(i)
+        e0.record(stream)
+        call()
+        e1.record(stream)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return float(np.mean(ts))
+
+
 def supplemental(fovea, params, mem, w, h, depth, row_scale, flush, n_steps):
     """Per-step latency of the small-N regime (the root and its K_c = 6
-    depth-1 children of one sequence) and of the paper's other retrieval
-    settings, on the same memory and hidden states.  Each is one CUDA graph of
-    one fovea_retrieve_fuse call, timed like the main step: CUDA events on the
-    launching stream around each replay, L2 flushed before it."""
+    depth-1 children of one sequence), of the depth gate at the paper's
+    l <= 1, and of the paper's other retrieval settings, on the same memory
+    and hidden states.  Each is timed like the headline: CUDA events on the
+    launching stream around one plain call, L2 flushed before it."""
     cases = []
     if w.B == 1 and w.N >= 7:
-        cases.append(("small_n_7", 7, w.rho, w.k_min, w.k_max))
-    cases.append(("paper_defaults_rho0.8_kmin32_kmax256", w.N, 0.8, 32, 256))
-    cases.append(("fixed_top16", w.N, w.rho, 16, 16))
+        cases.append(("small_n_7", 7, w.rho, w.k_min, w.k_max, None))
+    cases.append(("depth_gate_l1", w.N, w.rho, w.k_min, w.k_max, 1))
+    cases.append(("paper_defaults_rho0.8_kmin32_kmax256", w.N, 0.8, 32, 256, None))
+    cases.append(("fixed_top16", w.N, w.rho, 16, 16, None))
     m_max = int(max(w.m_sizes))
     if m_max <= 1024:
-        cases.append((f"dense_k{m_max}", w.N, 1.0, m_max, m_max))
-    stream = torch.cuda.current_stream()
-    fovea.timing_enable(False)           # plain graphs, no per-kernel event nodes
+        cases.append((f"dense_k{m_max}", w.N, 1.0, m_max, m_max, None))
+    fovea.timing_enable(False)
     out = {}
-    for name, n, rho, kmin, kmax in cases:
-        if n == w.N:
-            offs = list(w.row_offsets)
-        else:
-            offs = [0, n]
+    for name, n, rho, kmin, kmax, l_max in cases:
+        offs = list(w.row_offsets) if n == w.N else [0, n]
         hn, dn = h[:n].contiguous(), depth[:n].contiguous()
         rs = row_scale[:n].contiguous() if row_scale is not None else None
         ws = fovea.new_workspace(params, mem, offs, kmax)
@@ -585,44 +658,20 @@ def supplemental(fovea, params, mem, w, h, depth, row_scale, flush, n_steps):
 
         def step():
             fovea.retrieve_fuse(params, mem, hn, dn, offs, rs, rho, kmin, kmax, h_out, ws,
-                                counts=counts, offsets_c=offs_c)
-        cap = torch.cuda.Stream()
-        cap.wait_stream(stream)
-        with torch.cuda.stream(cap):
-            for _ in range(3):
-                step()
-        stream.wait_stream(cap)
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=cap):
-            step()
-        torch.cuda.synchronize()
-        for i in range(3):
-            flush(i)
-            g.replay()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        ts = []
-        for i in range(n_steps):
-            flush(i)
-            e0.record(stream)
-            g.replay()
-            e1.record(stream)
-            e1.synchronize()
-            ts.append(e0.elapsed_time(e1))
+                                counts=counts, offsets_c=offs_c, l_max=l_max)
+        ms = _time_calls(step, flush, n_steps)
         fovea.sync_errors(ws)
-        ms = float(np.mean(ts))
         c = counts.cpu().numpy()
         out[name] = {"draft_states": n, "rho": rho, "k_min": kmin, "k_max": kmax,
-                     "us_per_step": 1000 * ms, "value": n / (ms / 1000.0), "unit": UNIT,
-                     "mean_count": float(c.mean()), "steps": n_steps}
+                     "l_max": l_max, "us_per_step": 1000 * ms, "value": n / (ms / 1000.0),
+                     "unit": UNIT, "mean_count": float(c.mean()), "steps": n_steps}
     return out
 
 
 def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=7):
     """The draft logits and K_c candidates (fovea_lm_head_topk) on the step's
     own h_hat: a synthetic bf16 W_LM [vocab, d] ~ N(0, 1/d), drawn on the
-    device from a seeded generator; one CUDA graph per call, L2 flushed
+    device from a seeded generator; one plain call per step, L2 flushed
     before each, CUDA events on the launching stream."""
     N, d = h_hat.shape
     gen = torch.Generator(device=h_hat.device)
@@ -630,38 +679,13 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
     W = (torch.randn((vocab, d), generator=gen, device=h_hat.device) / math.sqrt(d)).to(torch.bfloat16)
     ws = torch.zeros(1 << 14, dtype=torch.uint8, device=h_hat.device)
     logits = torch.empty((N, vocab), dtype=torch.float32, device=h_hat.device)
-    stream = torch.cuda.current_stream()
-    cap = torch.cuda.Stream()
-    cap.wait_stream(stream)
-    with torch.cuda.stream(cap):
-        for _ in range(3):
-            out = fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits)
-    stream.wait_stream(cap)
-    torch.cuda.synchronize()
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=cap):
-        out = fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits)
-    torch.cuda.synchronize()
-    for i in range(3):
-        flush(i)
-        g.replay()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    ts = []
-    for i in range(n_steps):
-        flush(i)
-        e0.record(stream)
-        g.replay()
-        e1.record(stream)
-        e1.synchronize()
-        ts.append(e0.elapsed_time(e1))
+    ms = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits), flush, n_steps)
     fovea.sync_errors(ws)
-    ms = float(np.mean(ts))
     # algorithmic bytes: W_LM once, h_hat in, the logits out and back in for
     # the candidate selection, the candidates out
     nbytes = vocab * d * 2 + N * d * 2 + 2 * N * vocab * 4 + N * k_c * 8
     gbs = nbytes / (ms / 1000.0) / 1e9
-    del W, logits, out
+    del W, logits
     return {"vocab": vocab, "d_model": d, "draft_states": N, "k_c": k_c, "us_per_call": 1000 * ms,
             "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"],
             "steps": n_steps, "w_lm": "synthetic N(0, 1/d), bf16"}

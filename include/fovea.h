@@ -133,12 +133,14 @@ typedef struct fovea_params {
  * given the same W_f1, W_g1 pointers and mlp_hidden; weights changed in
  * place after the build need a new memory (as W_K, W_U already do).
  * bf16 with W_Q given: the handle also keeps the folded keys
- * kappa_i = W_Q^T k_i ([d], bf16; query folding).  Since
+ * kappa_i = W_Q^T k_i (query folding).  Since
  * q_n . k_i = (W_Q x_n) . k_i = x_n . kappa_i with x_n = LN(h_n) + E_dep[l_n],
  * a draft step given the same W_Q pointer scores x_n against kappa_i and
- * never streams W_Q.  kappa_i is rounded once from its exact value (elements
- * whose fp32 sum lies near a bf16 rounding midpoint are recomputed in
- * double-float).  Pass W_Q = NULL here to keep the unfolded scores.
+ * never streams W_Q.  kappa_i is not rounded to bf16: it is kept as a pair of
+ * bf16 values kappa_hi + kappa_lo (about 16 significant bits, the same
+ * precision the unfolded scores give q = W_Q x_n), so both score forms
+ * follow the paper's q . k to within fp32 accumulation.  Pass W_Q = NULL here
+ * to keep the unfolded scores.
  * This call allocates the handle's device buffers and synchronises `stream`
  * once (to size them).  B in [1, FOVEA_MAX_SEQ], M_max in [0, ...],
  * per-image valid count <= FOVEA_MAX_ENTRIES.
@@ -166,9 +168,10 @@ FOVEA_API fovea_status fovea_memory_tensors(const fovea_memory* mem, const void*
                                             const void** values, const int32_t** index,
                                             int64_t* offsets);
 
-/* The folded keys kappa_i = W_Q^T k_i [total_valid, d] (bf16, device, owned
- * by the handle) when the memory holds them for this W_Q pointer, else NULL
- * in *folded: a step given this W_Q scores against them. */
+/* The folded keys kappa_i = W_Q^T k_i as [total_valid, 2d] bf16 (row i holds
+ * kappa_hi then kappa_lo = bf16(kappa - kappa_hi); device, owned by the
+ * handle) when the memory holds them for this W_Q pointer, else NULL in
+ * *folded: a step given this W_Q scores against them. */
 FOVEA_API fovea_status fovea_memory_folded_keys(const fovea_memory* mem, const void* W_Q,
                                                 const void** folded);
 
@@ -182,10 +185,9 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
                                             const int32_t* row_offsets, int k_max,
                                             size_t* bytes);
 
-/* Zero the workspace's header: the error word and the counters the split-K
- * GEMMs use (enqueued on `stream`).  Kernels leave the counters at zero, so
- * one initialisation serves every later call; re-initialise after a call that
- * reported FOVEA_ERR_TIMEOUT. */
+/* Zero the workspace's header (the sticky error word and reserved words;
+ * enqueued on `stream`).  One initialisation serves every later call;
+ * fovea_sync_errors clears the header again after it reports an error. */
 FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void* stream);
 
 /*
@@ -202,6 +204,11 @@ FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void*
  *               1/sqrt(d_k) per row (NULL = 1, the paper's scores)
  *   rho         mass threshold, 0 < rho <= 1 (paper: 0.8)
  *   k_min,k_max 1 <= k_min <= k_max <= FOVEA_MAX_K (paper: 32, 256)
+ *   l_max       depth gate (the experimental setup corrects nodes at depth
+ *               <= 1): a row with l_n > l_max is not corrected: h_out = h,
+ *               count 0, indices -1, readout 0, gate 0.  l_max >= D corrects
+ *               every row (and reads no depth for the gate).  A depth outside
+ *               [0, D] counts as 0 here, as in the query.
  * Outputs (device, caller-owned):
  *   h_out       [N, d] dtype: h_hat_n = RMSNorm(h_n + g_n c_n)   (required)
  *   counts      [N] int32: K_{r,n}                                (or NULL)
@@ -226,7 +233,7 @@ FOVEA_API fovea_status fovea_workspace_init(void* workspace, size_t bytes, void*
 FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_memory* mem,
                                            const void* h, const int32_t* depth,
                                            const int32_t* row_offsets, const float* row_scale,
-                                           float rho, int k_min, int k_max,
+                                           float rho, int k_min, int k_max, int l_max,
                                            void* h_out, int32_t* counts, int32_t* indices,
                                            float* readout, float* gate,
                                            void* workspace, size_t workspace_bytes,
@@ -252,17 +259,23 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
  *   before any stream capture.
  * - Every call on a device shares the one array: calls that overlap on the GPU
  *   (other streams, other host threads) race and corrupt each other.  Each
- *   call clears the array's error word first; device-side conditions (a bad
- *   depth) are not reported back by this entry point, so validate depths.
+ *   call clears the array's reserved header words, not its error word:
+ *   device-side conditions (a bad depth, a bounded wait that gave up) stay
+ *   in the error word until fovea_noalloc_sync_errors reads and clears it.
+ *   This entry point does not report them itself.
  */
 #define FOVEA_NOALLOC_WORKSPACE_BYTES (32u << 20)
 FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(const fovea_params* p, const fovea_memory* mem,
                                                    const void* h, const int32_t* depth,
                                                    const int32_t* row_offsets,
                                                    const float* row_scale, float rho, int k_min,
-                                                   int k_max, void* h_out, int32_t* counts,
-                                                   int32_t* indices, float* readout, float* gate,
-                                                   void* stream);
+                                                   int k_max, int l_max, void* h_out,
+                                                   int32_t* counts, int32_t* indices,
+                                                   float* readout, float* gate, void* stream);
+/* fovea_sync_errors for the static array of fovea_retrieve_fuse_noalloc on
+ * the current device: synchronise `stream`, read and clear its error word
+ * (FOVEA_OK, FOVEA_ERR_INVALID_ARG for a bad depth, FOVEA_ERR_TIMEOUT). */
+FOVEA_API fovea_status fovea_noalloc_sync_errors(void* stream);
 
 /*
  * Draft logits and tree-expansion candidates (Eq. hidden_correction,
@@ -285,33 +298,22 @@ FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_mod
                                           int32_t* top_idx, float* top_val, void* workspace,
                                           size_t workspace_bytes, void* stream);
 
-/*
- * Implementation of the draft step (process-wide; the paper has no
- * counterpart, both compute the same operator):
- *   FOVEA_PATH_AUTO     the default: currently one kernel per stage, the
- *                       faster implementation on every shape measured so far
- *   FOVEA_PATH_FUSED    the persistent step kernel; it covers bf16 calls with
- *                       <= 64 sequences and <= 3072 valid entries per
- *                       sequence, and any other call returns
- *                       FOVEA_ERR_UNSUPPORTED
- *   FOVEA_PATH_KERNELS  one kernel per stage of the step
- * A workspace sized by fovea_workspace_size serves every path.
- * The persistent kernel is one cooperative launch of one CTA per SM whose
- * phases meet at device-wide barriers kept in the workspace header; it needs
- * the whole GPU, so a concurrent kernel on another stream delays its start.
- * fovea_step_path(path) selects and returns the previous setting; any other
- * value leaves the setting unchanged and returns it.
- */
-#define FOVEA_PATH_AUTO 0
-#define FOVEA_PATH_FUSED 1
-#define FOVEA_PATH_KERNELS 2
-FOVEA_API int fovea_step_path(int path);
-
 /* Synchronise `stream`, read and clear the workspace's sticky error word.
  * Returns FOVEA_OK, FOVEA_ERR_INVALID_ARG (a depth outside [0, D] was seen)
- * or FOVEA_ERR_TIMEOUT (a bounded device wait gave up; the whole workspace
- * header is then cleared, as fovea_workspace_init does), or FOVEA_ERR_CUDA. */
+ * or FOVEA_ERR_TIMEOUT (a bounded device wait gave up), or FOVEA_ERR_CUDA.
+ * After an error the whole header is cleared, as fovea_workspace_init does,
+ * so the workspace serves the next call. */
 FOVEA_API fovea_status fovea_sync_errors(void* workspace, void* stream);
+
+/* Limit of the bounded mbarrier waits in the tensor-core kernels launched
+ * after this call (process-wide; 0 restores the default of about 2 s).  The
+ * paper has no counterpart: it exists so that tests can make a wait give up
+ * and check that the call reports FOVEA_ERR_TIMEOUT (through
+ * fovea_sync_errors) and that the workspace serves the next call.  A wait
+ * that gives up still waits, with fixed limits, for the copies and MMAs its
+ * kernel issued before the kernel exits; the outputs of that call are
+ * undefined. */
+FOVEA_API fovea_status fovea_debug_wait_limit(unsigned long long limit_ns);
 
 /* Message of the last non-OK status returned on this thread ("" if none). */
 FOVEA_API const char* fovea_last_error(void);

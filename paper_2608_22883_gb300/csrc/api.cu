@@ -12,7 +12,6 @@
 #include <atomic>
 
 #include "common.cuh"
-#include "step_fused.h"
 
 using namespace fovea;
 
@@ -46,9 +45,6 @@ static fovea_status cuda_fail(cudaError_t e, const char* where) {
     cudaError_t e_ = (call);                      \
     if (e_ != cudaSuccess) return cuda_fail(e_, where); \
   } while (0)
-
-// Which implementation of the draft step fovea_retrieve_fuse runs.
-static std::atomic<int> g_step_path{FOVEA_PATH_AUTO};
 
 // ---------------------------------------------------------------------------
 // Per-launch timing (CUDA events on the launching stream)
@@ -132,12 +128,13 @@ struct fovea_memory {
   const void* proj_wf1 = nullptr;
   const void* proj_wg1 = nullptr;
   int proj_h = 0;
-  // bf16: the keys folded through the query projection, kappa_i = W_Q^T k_i
-  // ([total, d]), and the W_Q they were built with: q . k_i = x . kappa_i,
-  // so a call with that W_Q scores x = LN(h) + E_dep against them directly
+  // bf16: the keys folded through the query projection, kappa_i = W_Q^T k_i,
+  // as a hi / lo pair of bf16 values ([total, 2d]: row i holds kappa_hi then
+  // kappa_lo = bf16(kappa - kappa_hi), about 16 significant bits), and the
+  // W_Q they were built with: q . k_i = x . kappa_i, so a call with that W_Q
+  // scores x = LN(h) + E_dep against them directly
   void* folded = nullptr;
   const void* fold_wq = nullptr;
-  int folded_refined = 0;            // folded elements re-rounded exactly at build
 };
 
 static size_t esize(int dtype) { return dtype == FOVEA_BF16 ? 2 : 4; }
@@ -236,7 +233,7 @@ extern "C" {
 
 FOVEA_API const char* fovea_last_error(void) { return g_last_error.c_str(); }
 
-FOVEA_API int fovea_version(void) { return 100; }
+FOVEA_API int fovea_version(void) { return 200; }
 
 FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
                                           const uint8_t* mask, int B, int M_max, void* stream,
@@ -378,10 +375,10 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
         if (err != cudaSuccess) return cuda_fail(err, "refine_keys");
       }
       // bf16 with W_Q given: the folded keys kappa_i = W_Q^T k_i, a GEMM of
-      // W_Q^T (transposed once here) with the stored keys, listed elements
-      // near a bf16 rounding midpoint re-rounded exactly as for the keys
+      // W_Q^T (transposed once here) with the stored keys, kept as the hi / lo
+      // pair of its fp32 accumulator (no bf16 rounding of the query map)
       if (bf && p->W_Q != nullptr && aligned16(p->W_Q)) {
-        fovea_status fs = alloc_dev(&m->folded, (size_t)total * d * 2, "folded keys");
+        fovea_status fs = alloc_dev(&m->folded, (size_t)total * 2 * d * 2, "folded keys");
         if (fs != FOVEA_OK) return fs;
         void* wqt = nullptr;
         if ((fs = alloc_dev(&wqt, (size_t)d * d * 2, "transposed W_Q")) != FOVEA_OK) return fs;
@@ -389,43 +386,28 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
           { KernelTimer t("transpose_wq", s);
             err = launch_transpose_bf16(p->W_Q, d, d, wqt, s); }
           if (err != cudaSuccess) return cuda_fail(err, "transpose W_Q");
-          err = cudaMemsetAsync(fix_count, 0, sizeof(int), s);
-          if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
           GemmArgs fa;
           init_args(fa);
           fa.k_total = d;
           fa.b_split = d;
           fa.B0 = m->keys; fa.ldb0 = d;
-          fa.epi_split = d;
-          fa.out0 = m->folded; fa.ldc = d;
+          fa.out0 = m->folded;
+          fa.out1 = static_cast<__nv_bfloat16*>(m->folded) + d;
+          fa.ldc = 2 * d;
           fa.err = m->err;
-          fa.fix_list = fix_list; fa.fix_count = fix_count; fa.fix_cap = (int)fix_cap;
           fa.ngroups = 1;
           fa.groups[0] = GemmGroup{0, d, 0, total, 0};
           { KernelTimer t("memory_fold", s);
-            err = launch_gemm_tc(kEpiStoreKeys, fa, TmaOperand{wqt, d, d, d},
+            err = launch_gemm_tc(kEpiStoreHiLo, fa, TmaOperand{wqt, d, d, d},
                                  TmaOperand{nullptr, 0, 0, 0}, TmaOperand{m->keys, total, d, d},
                                  TmaOperand{nullptr, 0, 0, 0}, d, total, s); }
           if (err != cudaSuccess) return cuda_fail(err, "query folding of the keys");
-          { KernelTimer t("refine_folded", s);
-            err = launch_refine_keys(m->keys, wqt, d, fix_list, fix_count, (int)fix_cap, total,
-                                     m->folded, s); }
-          if (err != cudaSuccess) return cuda_fail(err, "refine_folded");
-          int fe[2] = {0, 0};
-          err = cudaMemcpyAsync(&fe[0], m->err, sizeof(int), cudaMemcpyDeviceToHost, s);
-          if (err == cudaSuccess)
-            err = cudaMemcpyAsync(&fe[1], fix_count, sizeof(int), cudaMemcpyDeviceToHost, s);
+          int fe = 0;
+          err = cudaMemcpyAsync(&fe, m->err, sizeof(int), cudaMemcpyDeviceToHost, s);
           if (err == cudaSuccess) err = cudaStreamSynchronize(s);
           if (err != cudaSuccess) return cuda_fail(err, "query folding");
-          if (fe[0] & kErrTimeout)
+          if (fe & kErrTimeout)
             return fail(FOVEA_ERR_TIMEOUT, "a bounded device wait gave up while folding the keys");
-          m->folded_refined = fe[1];
-          if (fe[1] > fix_cap) {           // list overflowed: refine every element
-            { KernelTimer t("refine_folded", s);
-              err = launch_refine_keys(m->keys, wqt, d, nullptr, nullptr, 0, total, m->folded, s); }
-            if (err == cudaSuccess) err = cudaStreamSynchronize(s);
-            if (err != cudaSuccess) return cuda_fail(err, "refine_folded");
-          }
           return FOVEA_OK;
         };
         fs = fold();
@@ -517,59 +499,11 @@ FOVEA_API fovea_status fovea_memory_tensors(const fovea_memory* mem, const void*
 // Workspace layout (all regions 256-byte aligned)
 // ---------------------------------------------------------------------------
 namespace {
-// Workspace header: the sticky error word (first 256 bytes) and the split-K
-// tile counters (pairs of ints).  Zero when the workspace is initialised; the
-// kernels leave the counters at zero after every launch.
-constexpr size_t kWsHeaderBytes = 16384;
-// Words of the persistent step kernel inside the header's first 256 bytes
-// (bytes 128..175): grid-barrier arrival counters, exit counter, abort word.
-constexpr size_t kWsSyncOffset = 128;
-constexpr long long kTileSyncTiles = (kWsHeaderBytes - 256) / 8;
-
 struct WsLayout {
-  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, partials, total;
-  long long partial_floats;
+  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, total;
 };
 
-// fp32 scratch for the split-K partial tiles of the step's tensor-core GEMMs
-// (they run one after another, so one region serves all of them).
-long long step_partial_floats(int dtype, int d, int H, int N, int ngroups, int max_m, int max_r) {
-  if (dtype != FOVEA_BF16 || N == 0) return 0;
-  GemmArgs* a = new GemmArgs;
-  auto plan = [&](int epi, int k_total, int a_split, int groups, int mm, int mn) {
-    memset(a, 0, sizeof(GemmArgs));
-    a->k_total = k_total;
-    a->a_split = a_split;
-    a->a_split2 = 0x7fffffff;
-    a->ngroups = groups;
-    return plan_gemm_tc(epi, *a, mm, mn).partial_floats;
-  };
-  long long need = plan(kEpiStoreHiLo, d, 0x7fffffff, 1, d, N);
-  if (ngroups > 0) need = std::max(need, plan(kEpiScores, d, 0x7fffffff, ngroups, max_m, max_r));
-  need = std::max(need, plan(kEpiBiasSilu, 2 * d, H, 1, 2 * H, N));
-  need = std::max(need, plan(kEpiBiasF32, H, 0x7fffffff, 1, d, N));
-  delete a;
-  return need;
-}
-
-// The persistent-kernel plan of a call (false: the call's shape is outside it).
-// (Independent of the path setting: a workspace is sized for both paths.)
-bool plan_fused_call(const fovea_params* p, const fovea_memory* mem, const int32_t* row_offsets,
-                     int k_max, FusedPlan* plan) {
-  FusedShape sh;
-  sh.bf16 = p->dtype == FOVEA_BF16;
-  sh.N = row_offsets[mem->B];
-  sh.d = p->d_model;
-  sh.H = p->mlp_hidden;
-  sh.B = mem->B;
-  sh.k_max = k_max;
-  sh.row_offsets = row_offsets;
-  sh.m = mem->counts.data();
-  return fused_plan(sh, plan);
-}
-
-WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems,
-                   long long partial_floats) {
+WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems) {
   WsLayout L;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -578,7 +512,7 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
     return o;
   };
   const size_t es = esize(dtype);
-  L.err = take(kWsHeaderBytes);          // error word, then split-K tile counters
+  L.err = take(kWsHeaderBytes);          // the sticky error word, then reserved words
   L.xh = take((size_t)N * d * es);
   L.q = take((size_t)N * d * es * (dtype == FOVEA_BF16 ? 2 : 1));   // bf16: q_hi | q_lo
   L.scores = take((size_t)score_elems * 4);
@@ -589,8 +523,6 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
   L.act = take((size_t)N * 2 * H * es);
   L.c = take((size_t)N * d * 4);
   L.gh = take(dtype == FOVEA_BF16 ? (size_t)N * 2 * H * 4 : 0);   // [W_f1 ; W_g1]_h h, fp32
-  L.partials = take((size_t)partial_floats * 4);
-  L.partial_floats = partial_floats;
   L.total = off;
   return L;
 }
@@ -637,10 +569,7 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
   int N, mm, mr, ng;
   long long se;
   if ((st = check_rows(mem, row_offsets, &N, &se, &mm, &mr, &ng)) != FOVEA_OK) return st;
-  long long pf = step_partial_floats(p->dtype, p->d_model, p->mlp_hidden, N, ng, mm, mr);
-  static thread_local FusedPlan fp;
-  if (N > 0 && plan_fused_call(p, mem, row_offsets, k_max, &fp)) pf = std::max(pf, fp.partial_floats);
-  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se, pf).total;
+  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se).total;
   return FOVEA_OK;
 }
 
@@ -662,27 +591,30 @@ FOVEA_API fovea_status fovea_sync_errors(void* workspace, void* stream) {
   FOVEA_CUDA(cudaMemcpyAsync(&herr, workspace, sizeof(int), cudaMemcpyDeviceToHost, s),
              "cudaMemcpyAsync");
   FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-  FOVEA_CUDA(cudaMemsetAsync(workspace, 0, sizeof(int), s), "cudaMemsetAsync");
+  // clear the whole header: a kernel that gave up may have left other words set
+  FOVEA_CUDA(cudaMemsetAsync(workspace, 0, herr ? kWsHeaderBytes : sizeof(int), s),
+             "cudaMemsetAsync");
   FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
-  if (herr & kErrTimeout) {
-    // the kernels that gave up may have left barrier counters or the abort
-    // word set: start the next call from a clean header
-    FOVEA_CUDA(cudaMemsetAsync(workspace, 0, kWsHeaderBytes, s), "cudaMemsetAsync");
-    FOVEA_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+  if (herr & kErrTimeout)
     return fail(FOVEA_ERR_TIMEOUT, "a bounded device wait gave up (error word 0x%x)", herr);
-  }
   if (herr & kErrDepth)
     return fail(FOVEA_ERR_INVALID_ARG, "a draft state had a depth outside [0, max_depth]");
+  return FOVEA_OK;
+}
+
+FOVEA_API fovea_status fovea_debug_wait_limit(unsigned long long limit_ns) {
+  g_last_error.clear();
+  set_wait_limit_ns(limit_ns == 0 ? kDefaultWaitLimitNs : limit_ns);
   return FOVEA_OK;
 }
 
 FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_memory* mem,
                                            const void* h, const int32_t* depth,
                                            const int32_t* row_offsets, const float* row_scale,
-                                           float rho, int k_min, int k_max, void* h_out,
-                                           int32_t* counts, int32_t* indices, float* readout,
-                                           float* gate, void* workspace, size_t workspace_bytes,
-                                           void* stream) {
+                                           float rho, int k_min, int k_max, int l_max,
+                                           void* h_out, int32_t* counts, int32_t* indices,
+                                           float* readout, float* gate, void* workspace,
+                                           size_t workspace_bytes, void* stream) {
   g_last_error.clear();
   fovea_status st = check_step_params(p);
   if (st != FOVEA_OK) return st;
@@ -710,22 +642,7 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   const int d = p->d_model, H = p->mlp_hidden, dt = p->dtype;
-  static thread_local FusedPlan fplan;
-  // the persistent kernel runs only when selected; AUTO takes the per-stage
-  // kernels, which are faster on the shapes measured so far
-  const bool want_fused = g_step_path.load() == FOVEA_PATH_FUSED;
-  const bool use_fused = want_fused && plan_fused_call(p, mem, row_offsets, k_max, &fplan);
-  if (!use_fused && want_fused)
-    return fail(FOVEA_ERR_UNSUPPORTED,
-                "the persistent step kernel does not cover this call (bf16, <= %d sequences, "
-                "<= 3072 entries per sequence are required)", fused::kMaxSeq);
-  long long pfloats = step_partial_floats(dt, d, H, N, ngroups, max_m, max_r);
-  {
-    static thread_local FusedPlan fp_any;
-    if (plan_fused_call(p, mem, row_offsets, k_max, &fp_any))
-      pfloats = std::max(pfloats, fp_any.partial_floats);
-  }
-  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems, pfloats);
+  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems);
   if (workspace_bytes < L.total)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);
 
@@ -742,47 +659,10 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   void* act = ws + L.act;
   float* cbuf = reinterpret_cast<float*>(ws + L.c);
   float* gh = reinterpret_cast<float*>(ws + L.gh);
-  float* partials = reinterpret_cast<float*>(ws + L.partials);
-  int* tile_sync = reinterpret_cast<int*>(ws + L.err + 256);
-
-  if (use_fused) {
-    // the whole step as one persistent cooperative kernel (step_fused.cu)
-    static thread_local std::vector<int32_t> key_off;
-    key_off.resize(mem->B);
-    long long m_sel = 0;
-    for (int b = 0; b < mem->B; ++b) {
-      key_off[b] = (int32_t)mem->offsets[b];
-      const long long R = row_offsets[b + 1] - row_offsets[b];
-      m_sel += std::min<long long>(mem->counts[b], R * k_max);
-    }
-    FusedLaunch fl;
-    memset(&fl, 0, sizeof(fl));
-    fl.N = N; fl.d = d; fl.H = H; fl.B = mem->B; fl.k_max = k_max; fl.k_min = k_min;
-    fl.max_depth = p->max_depth; fl.rho = rho; fl.ln_eps = p->ln_eps; fl.rms_eps = p->rms_eps;
-    fl.row_offsets = row_offsets; fl.key_off = key_off.data(); fl.m = mem->counts.data();
-    fl.total_keys = mem->total;
-    fl.prefetch_values = 2 * m_sel >= mem->total;     // most value rows will be read
-    fl.h = h; fl.ln_gamma = p->ln_h_gamma; fl.ln_beta = p->ln_h_beta; fl.E = p->E_dep;
-    fl.W_Q = p->W_Q; fl.keys = mem->keys; fl.values = mem->values;
-    fl.W_f1 = p->W_f1; fl.W_g1 = p->W_g1; fl.W_f2 = p->W_f2;
-    fl.b_f1 = p->b_f1; fl.b_g1 = p->b_g1; fl.b_f2 = p->b_f2; fl.w_g2 = p->w_g2; fl.b_g2 = p->b_g2;
-    fl.rms_gamma = p->rms_gamma;
-    fl.depth = depth; fl.row_scale = row_scale; fl.orig_index = mem->orig_index;
-    fl.x = ws + L.xh; fl.q_hi = ws + L.q; fl.q_lo = ws + L.q + (size_t)N * d * 2;
-    fl.r = ws + L.r_lo; fl.act = ws + L.act;
-    fl.partials = reinterpret_cast<float*>(ws + L.partials);
-    fl.sel_pos = reinterpret_cast<int32_t*>(ws + L.sel_pos);
-    fl.sel_w = reinterpret_cast<float*>(ws + L.sel_w);
-    fl.sel_cnt = reinterpret_cast<int32_t*>(ws + L.sel_cnt);
-    fl.err = reinterpret_cast<int*>(ws + L.err);
-    fl.sync = reinterpret_cast<int*>(ws + L.err + kWsSyncOffset);
-    fl.h_out = h_out; fl.counts = counts; fl.indices = indices; fl.readout = readout; fl.gate = gate;
-    cudaError_t e;
-    { KernelTimer t("fused_step", s);
-      e = launch_fused_step(fplan, fl, s); }
-    if (e != cudaSuccess) return cuda_fail(e, "fused_step");
-    return FOVEA_OK;
-  }
+  // depth gate: rows deeper than l_max are not corrected (their selection is
+  // empty and h_hat = h); with l_max >= D every row is corrected and the gate
+  // reads nothing
+  const DepthGate gate_rows{l_max < p->max_depth ? depth : nullptr, l_max, p->max_depth};
 
   // Per-sequence table (kernel parameter).
   static thread_local SeqTable tab;
@@ -821,6 +701,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                         mem->proj_wg1 == p->W_g1 && mem->proj_h == H &&
                         select_readout_fits(max_m, k_max);
   const bool use_fold = bf && mem->folded != nullptr && mem->fold_wq == p->W_Q;
+  // the folded keys are [total, 2d] (hi | lo per entry)
+  const long long score_key_bytes = (long long)mem->total * d * 2 * (use_fold ? 2 : 1);
   const void* score_keys = use_fold ? mem->folded : mem->keys;
   // With folded keys and projected values, G_h does not depend on the query:
   // when one sequence's keys serve every row (one score group covering all N
@@ -838,8 +720,6 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.A0 = p->W_Q; a.lda0 = d;
   a.B0 = xh; a.ldb0 = d;
   a.out0 = q; a.out1 = q_lo; a.ldc = d; a.err = err;
-  a.partials = partials; a.partials_floats = L.partial_floats;
-  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
   if (use_proj) {
@@ -858,9 +738,9 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     // the keys when the score GEMM's own loads before its griddepcontrol.wait
     // (its first ring stages) cannot cover them, and the values when most of
     // their rows will be read by the readout
-    if ((long long)mem->total * d * 2 > (8ll << 20)) {
+    if (score_key_bytes > (8ll << 20)) {
       a.pf_ptr[a.n_prefetch] = score_keys;
-      a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
+      a.pf_bytes[a.n_prefetch++] = score_key_bytes;
     }
     if (2 * m_sel >= mem->total) {
       if (!use_proj || readout != nullptr) {
@@ -884,7 +764,7 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                          TmaOperand{nullptr, 0, 0, 0}, 2 * H, N, s); }
     if (e != cudaSuccess) return cuda_fail(e, "fusion_h");
   } else if (!use_fold) {
-  { KernelTimer t("query_proj", s);
+    KernelTimer t("query_proj", s);
     if (use_proj)
       e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{p->W_Q, d, d, d}, TmaOperand{p->W_f1, H, d, 2 * d},
                          TmaOperand{xh, N, d, d}, TmaOperand{h, N, d, d}, d + 2 * H, N, s,
@@ -892,22 +772,22 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     else
       e = run_gemm(dt, bf ? kEpiStoreHiLo : kEpiStore, a, TmaOperand{p->W_Q, d, d, d},
                    TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
-                   TmaOperand{nullptr, 0, 0, 0}, d, N, s); }
-  if (e != cudaSuccess) return cuda_fail(e, "query_proj");
+                   TmaOperand{nullptr, 0, 0, 0}, d, N, s);
+    if (e != cudaSuccess) return cuda_fail(e, "query_proj");
   }
 
-  // (3) s = q k^T / sqrt(d) (* row_scale), per sequence
+  // (3) s = q k^T / sqrt(d) (* row_scale), per sequence; folded: x_h against
+  // kappa_hi and kappa_lo
   if (score_elems > 0) {
     init_args(a);
     a.k_total = d; a.b_split = d;
-    a.A0 = score_keys; a.lda0 = d;
+    a.A0 = score_keys; a.lda0 = use_fold ? 2 * d : d;
     a.B0 = use_fold ? xh : q; a.ldb0 = d;
     a.out0 = scores;
     a.row_scale = row_scale;
     a.scale = (float)(1.0 / sqrt((double)d));
     a.err = err;
-  a.partials = partials; a.partials_floats = L.partial_floats;
-  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
+    a.f_lo_kb = use_fold ? d / 64 : 0;
     int g = 0;
     for (int b = 0; b < mem->B; ++b) {
       const int r = row_offsets[b + 1] - row_offsets[b];
@@ -930,9 +810,12 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
       a.pf_ptr[a.n_prefetch] = p->W_g1;
       a.pf_bytes[a.n_prefetch++] = (long long)H * 2 * d * 2;
-      a.pf_ptr[a.n_prefetch] = p->W_f2;
-      a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
+      if (a.n_prefetch < 4) {
+        a.pf_ptr[a.n_prefetch] = p->W_f2;
+        a.pf_bytes[a.n_prefetch++] = (long long)d * H * 2;
+      }
     }
+    const TmaOperand folded_op{mem->folded, mem->total, 2 * d, 2 * d};
     if (gh_in_scores) {
       // one group: the sequence's folded keys (scores, against x_h), then the
       // h-halves of W_f1 and W_g1 (G_h, against h)
@@ -942,19 +825,18 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
       a.r_by_part = 1;
       a.epi_split = M;
       a.out2 = gh; a.ldc2 = 2 * H;
-      if (readout != nullptr && 2 * m_sel >= mem->total) {
+      if (readout != nullptr && 2 * m_sel >= mem->total && a.n_prefetch < 4) {
         a.pf_ptr[a.n_prefetch] = mem->values;
         a.pf_bytes[a.n_prefetch++] = (long long)mem->total * d * 2;
       }
       KernelTimer t("score_fusion_h", s);
-      e = launch_gemm_tc(kEpiScoresFolded, a, TmaOperand{mem->folded, mem->total, d, d},
-                         TmaOperand{p->W_f1, H, d, 2 * d}, TmaOperand{xh, N, d, d},
-                         TmaOperand{h, N, d, d}, M + 2 * H, N, s, TmaOperand{p->W_g1, H, d, 2 * d});
+      e = launch_gemm_tc(kEpiScoresFolded, a, folded_op, TmaOperand{p->W_f1, H, d, 2 * d},
+                         TmaOperand{xh, N, d, d}, TmaOperand{h, N, d, d}, M + 2 * H, N, s,
+                         TmaOperand{p->W_g1, H, d, 2 * d});
     } else if (use_fold) {
       KernelTimer t("score_folded", s);
-      e = launch_gemm_tc(kEpiScoresFolded, a, TmaOperand{mem->folded, mem->total, d, d},
-                         TmaOperand{nullptr, 0, 0, 0}, TmaOperand{xh, N, d, d},
-                         TmaOperand{nullptr, 0, 0, 0}, max_m, max_r, s);
+      e = launch_gemm_tc(kEpiScoresFolded, a, folded_op, TmaOperand{nullptr, 0, 0, 0},
+                         TmaOperand{xh, N, d, d}, TmaOperand{nullptr, 0, 0, 0}, max_m, max_r, s);
     } else {
       KernelTimer t("score", s);
       e = run_gemm(dt, kEpiScores, a, TmaOperand{mem->keys, mem->total, d, d},
@@ -970,21 +852,21 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if (use_proj) {
     { KernelTimer t("select_fuse", s);
       e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
-                               counts, indices, mem->values, d, readout, nullptr, mem->proj, H,
-                               gh, p->b_f1, p->b_g1, act, err, s,
+                               gate_rows, counts, indices, mem->values, d, readout, nullptr,
+                               mem->proj, H, gh, p->b_f1, p->b_g1, act, err, s,
                                (long long)mem->total * 2 * H * 2); }
     if (e != cudaSuccess) return cuda_fail(e, "select_fuse");
   } else {
     if (select_readout_fits(max_m, k_max)) {
       { KernelTimer t("select_readout", s);
         e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
-                                 counts, indices, mem->values, d, readout, r_lo, nullptr, H,
-                                 nullptr, nullptr, nullptr, nullptr, err, s); }
+                                 gate_rows, counts, indices, mem->values, d, readout, r_lo,
+                                 nullptr, H, nullptr, nullptr, nullptr, nullptr, err, s); }
       if (e != cudaSuccess) return cuda_fail(e, "select_readout");
     } else {
       { KernelTimer t("select", s);
-        e = launch_select(scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m, counts, indices,
-                          sel_pos, sel_w, sel_cnt, s); }
+        e = launch_select(scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m, gate_rows,
+                          counts, indices, sel_pos, sel_w, sel_cnt, s); }
       if (e != cudaSuccess) return cuda_fail(e, "select");
       { KernelTimer t("readout", s);
         e = launch_readout(dt, mem->values, sel_cnt, sel_pos, sel_w, N, k_max, d, readout, r_lo, s); }
@@ -1002,8 +884,6 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
     a.out0 = act; a.ldc = 2 * H;
     a.bias0 = p->b_f1; a.bias1 = p->b_g1;
     a.err = err;
-    a.partials = partials; a.partials_floats = L.partial_floats;
-    a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
     a.ngroups = 1;
     a.groups[0] = GemmGroup{0, 2 * H, 0, N, 0};
     { KernelTimer t("fuse_hidden", s);
@@ -1021,8 +901,6 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   a.out0 = cbuf; a.ldc = d;
   a.bias0 = p->b_f2;
   a.err = err;
-  a.partials = partials; a.partials_floats = L.partial_floats;
-  a.tile_sync = tile_sync; a.tile_sync_tiles = kTileSyncTiles;
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, d, 0, N, 0};
   { KernelTimer t("fuse_out", s);
@@ -1030,10 +908,11 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
                  TmaOperand{act, N, H, 2 * H}, TmaOperand{nullptr, 0, 0, 0}, d, N, s); }
   if (e != cudaSuccess) return cuda_fail(e, "fuse_out");
 
-  // (8) g = sigma(a_g w_g2 + b_g2); h_hat = RMSNorm(h + g c)
+  // (8) g = sigma(a_g w_g2 + b_g2); h_hat = RMSNorm(h + g c); rows past the
+  // depth gate: h_hat = h
   { KernelTimer t("finalize", s);
     e = launch_finalize(dt, h, cbuf, act, H, d, p->w_g2, p->b_g2, p->rms_gamma, p->rms_eps, N,
-                        h_out, gate, s); }
+                        gate_rows, h_out, gate, s); }
   if (e != cudaSuccess) return cuda_fail(e, "finalize");
   return FOVEA_OK;
 }
@@ -1085,12 +964,6 @@ FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_mod
     e = launch_topk_rows(logits, N, vocab, k_c, top_idx, top_val, s); }
   if (e != cudaSuccess) return cuda_fail(e, "topk");
   return FOVEA_OK;
-}
-
-FOVEA_API int fovea_step_path(int path) {
-  if (path == FOVEA_PATH_AUTO || path == FOVEA_PATH_FUSED || path == FOVEA_PATH_KERNELS)
-    return g_step_path.exchange(path);
-  return g_step_path.load();
 }
 
 FOVEA_API fovea_status fovea_timing_enable(int enable) {

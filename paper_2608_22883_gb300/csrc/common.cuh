@@ -13,6 +13,33 @@ namespace fovea {
 // Sticky device error bits (workspace / memory error word).
 enum : int { kErrDepth = 1, kErrTimeout = 2 };
 
+// Bytes at the start of a step workspace: the sticky error word and reserved
+// words (fovea_workspace_init zeroes them).
+constexpr size_t kWsHeaderBytes = 4096;
+
+// Limit of a bounded mbarrier wait inside the tensor-core kernels (ns).  A
+// wait that gives up sets kErrTimeout; the kernel then waits for the work it
+// has already issued (copies, MMAs) with fixed limits and unwinds.
+constexpr unsigned long long kDefaultWaitLimitNs = 2000000000ull;
+// Process-wide limit the GEMM launches pass to their kernels
+// (fovea_debug_wait_limit; api.cu).
+void set_wait_limit_ns(unsigned long long ns);
+unsigned long long wait_limit_ns();
+
+// Depth gate of a draft step: rows whose depth l_n (an invalid depth counts
+// as 0, as in the query LN) exceeds l_max are not corrected.  depth == null:
+// every row is corrected.
+struct DepthGate {
+  const int32_t* depth;
+  int l_max, max_depth;
+};
+__device__ __forceinline__ bool row_gated(const DepthGate& g, int n) {
+  if (g.depth == nullptr) return false;
+  int l = g.depth[n];
+  if (l < 0 || l > g.max_depth) l = 0;
+  return l > g.l_max;
+}
+
 // ---------------------------------------------------------------------------
 // Scalar conversions
 // ---------------------------------------------------------------------------
@@ -106,10 +133,10 @@ enum EpiKind : int {
                       // rounding midpoint are listed for an exact recomputation
   kEpiQueryH = 6,     // columns < epi_split as kEpiStoreHiLo; columns >= epi_split:
                       // out2 (fp32)[row * ldc2 + col - epi_split] = acc
-  kEpiScoresFolded = 7,  // kEpiScores with one row operand (x_h against folded keys)
-                         // instead of the hi / lo pair, for columns < epi_split (row
-                         // stride min(m, epi_split)); columns >= epi_split:
-                         // out2 (fp32)[row * ldc2 + col - epi_split] = acc
+  kEpiScoresFolded = 7,  // kEpiScores with one row operand (x_h) against the folded
+                         // keys, a hi / lo pair of feature tiles (f_lo_kb), for columns
+                         // < epi_split (row stride min(m, epi_split)); columns >=
+                         // epi_split: out2 (fp32)[row * ldc2 + col - epi_split] = acc
 };
 
 struct KeyFix {       // one listed key element: memory row, feature
@@ -124,6 +151,9 @@ struct GemmArgs {
   int b_split;        // contraction index >= b_split comes from B1 (k - b_split)
   int dual_b;         // tensor-core scores: B0 and B1 are the hi / lo parts of one
                       // operand, both multiplied by the same A tile
+  int f_lo_kb;        // tensor-core folded scores: the feature operand A0 holds the
+                      // hi / lo parts of the folded keys in each row, lo starting
+                      // f_lo_kb k-blocks after hi (0: one part)
   // raw operands (SIMT path; the tensor-core path uses tensor maps)
   const void* A0; const void* A1; long long lda0, lda1;
   const void* B0; const void* B1; long long ldb0, ldb1;
@@ -140,10 +170,7 @@ struct GemmArgs {
   int kps;            // tensor-core path: k-blocks of 64 per ring stage
   int rbox;           // tensor-core path: rows of a row-operand tile (64 or 128)
   int region;         // tensor-core path: bytes of the ring / partial-tile staging region
-  float* partials;    // tensor-core split K: fp32 partial tiles (scratch)
-  long long partials_floats;
-  int* tile_sync;     // tensor-core split K: per tile {arrivals, departures}, zero between launches
-  long long tile_sync_tiles;
+  unsigned long long wait_ns;   // tensor-core path: limit of a bounded mbarrier wait
   int* err;
   // tensor-core path: byte ranges whose share each CTA prefetches into L2 once
   // it has requested its own operands (data a later kernel of the step reads)
@@ -209,9 +236,9 @@ cudaError_t launch_count_valid(const uint8_t* mask, int B, int M_max, int32_t* c
 cudaError_t launch_compact(const uint8_t* mask, int B, int M_max, const int32_t* key_off,
                            int32_t* orig_index, int32_t* src_row, cudaStream_t s);
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
-                          float rho, int k_min, int k_max, int max_m, int32_t* counts,
-                          int32_t* indices, int32_t* sel_pos, float* sel_w, int32_t* sel_cnt,
-                          cudaStream_t s);
+                          float rho, int k_min, int k_max, int max_m, const DepthGate& gate,
+                          int32_t* counts, int32_t* indices, int32_t* sel_pos, float* sel_w,
+                          int32_t* sel_cnt, cudaStream_t s);
 cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, const int32_t* sel_pos,
                            const float* sel_w, int N, int k_max, int d, float* r_out, void* r_lo,
                            cudaStream_t s);
@@ -224,7 +251,8 @@ cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, con
 bool select_readout_fits(int max_m, int k_max);
 cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable& tab, int N,
                                  const int32_t* orig_index, float rho, int k_min, int k_max,
-                                 int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
+                                 int max_m, const DepthGate& gate, int32_t* counts,
+                                 int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
                                  const void* b_f1, const void* b_g1, void* act, int* err,
                                  cudaStream_t s, long long p_prefetch_bytes = 0);
@@ -242,9 +270,11 @@ cudaError_t launch_topk_rows(const float* logits, int N, long long V, int k, int
 
 cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
                                const int* count, int cap, int rows, void* K, cudaStream_t s);
+// Rows past the depth gate: h_out = h and gate 0.
 cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,
                             const void* w_g2, const void* b_g2, const void* rms_gamma, float eps,
-                            int N, void* h_out, float* gate_out, cudaStream_t s);
+                            int N, const DepthGate& gate, void* h_out, float* gate_out,
+                            cudaStream_t s);
 
 // GEMM C = A . B^T with a chosen epilogue.  `tc` selects the tcgen05 path
 // (bf16 only); otherwise the SIMT path (fp32 and bf16).

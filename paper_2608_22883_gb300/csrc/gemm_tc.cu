@@ -1,9 +1,10 @@
 // tcgen05 GEMM C = A . B^T for the bf16 path (sm_103a): the memory
-// projections k = W_K LN(v), u = W_U LN(v), the query projection W_Q, the
-// scores q . k^T per sequence, and the two fusion layers.  For the scores the
-// query is carried as a bf16 hi/lo pair (q ~= q_hi + q_lo, about 16
-// significant bits) and each key tile meets both parts, so the scores are not
-// limited by a bf16 rounding of q.
+// projections k = W_K LN(v), u = W_U LN(v), the folded keys W_Q^T k, the
+// query projection W_Q, the scores per sequence, and the two fusion layers.
+// Neither score form rounds the query map to bf16: the unfolded scores carry
+// q = W_Q x as a bf16 hi/lo pair (q ~= q_hi + q_lo, about 16 significant
+// bits) and each key tile meets both parts; the folded scores carry the
+// folded keys kappa = W_Q^T k as a hi/lo pair and each x tile meets both.
 //
 // Operand roles.  In the GemmArgs vocabulary A holds the output columns
 // (weights, keys: the "feature" operand) and B the output rows (draft states,
@@ -24,8 +25,11 @@
 // after another, so each operand gets its own issuing lane), warp 1 owns the
 // tensor-memory allocation and its lane 0 issues the MMAs (one elected
 // thread), and all eight warps run the epilogue: warp w reads accumulator
-// lanes (rows) 32 (w % 4) .. +31.  Every mbarrier wait is bounded (~2 s); a
-// wait that gives up sets kErrTimeout in the error word and the CTA unwinds.
+// lanes (rows) 32 (w % 4) .. +31.  Every mbarrier wait is bounded (~2 s, or
+// the limit fovea_debug_wait_limit sets); a wait that gives up sets
+// kErrTimeout in the error word and the CTA unwinds: the producer waits for
+// the copies it issued, the MMA issuer commits what it issued, and the
+// epilogue waits for those MMAs before the tensor memory is freed.
 //
 // Split K: when the output tiles cannot fill the GPU (a 64-row batch against
 // a weight matrix), S <= 8 CTAs share one output tile, each contracting a
@@ -42,6 +46,8 @@
 // The producer issues the feature-operand (weight / key) loads of the first
 // stages before griddepcontrol.wait; those operands never depend on the
 // previous kernel, so the weight stream starts while the predecessor drains.
+#include <atomic>
+
 #include "gemm_epilogue.cuh"
 #include "tc_ptx.cuh"
 
@@ -69,11 +75,14 @@ constexpr int kMaxStages = 8;
 // reads 128 rows from each row tile's start; rows past rbox (>= 64, so the
 // read stays inside the stage) only feed accumulator rows that are never
 // stored.
+// DF (dual feature, the folded scores): the feature stage holds two tiles (hi
+// and lo parts of the folded keys), each multiplied by the same row tile into
+// the same accumulator.
 template <int BN, bool DUAL = false>
 struct Cfg {
   static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
-  __host__ __device__ static constexpr int stage_bytes(int kps, int rbox) {
-    return kps * (rbox * (DUAL ? 2 : 1) + BN) * 128;
+  __host__ __device__ static constexpr int stage_bytes(int kps, int rbox, bool df = false) {
+    return kps * (rbox * (DUAL ? 2 : 1) + BN * (df ? 2 : 1)) * 128;
   }
   // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9
   // = 1), B bf16 (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at
@@ -116,7 +125,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap tmR1, const __grid_constant__ GemmArgs args) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = Cfg<BN, DUAL>;
-  constexpr int kProducers = DUAL ? 3 : 2;   // TMA-issuing lanes of warp 0
   const int S = args.splits;
   const uint32_t rank = (uint32_t)((int)blockIdx.x % S);
   const GemmGroup& g = args.groups[blockIdx.z];
@@ -137,12 +145,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n0 = blockIdx.y * BM;
   if (m0 >= m_end || n0 >= g.n) return;
 
-  const int stages = args.stages;
+  // folded scores: the folded keys (part 0) are a hi / lo pair of bf16 values,
+  // the lo part f_lo_kb k-blocks after the hi part in the same rows
+  const bool dual_f = EPI == kEpiScoresFolded && args.f_lo_kb > 0 && part == 0;
+  const int kProducers = (DUAL || dual_f) ? 3 : 2;   // TMA-issuing lanes of warp 0
   const int KPS = args.kps, rbox = args.rbox;
   const int r_tile = rbox * 128;                       // one k-block of the row operand
   const int r_bytes = KPS * r_tile * (DUAL ? 2 : 1);
   const int f_tile = BN * 128;                         // one k-block of the feature operand
-  const int stage_bytes = C::stage_bytes(KPS, rbox);
+  const int stage_bytes = C::stage_bytes(KPS, rbox, dual_f);
+  const int stages = dual_f ? max(1, min(args.stages, args.region / stage_bytes)) : args.stages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -185,18 +197,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 && lane < kProducers) {
     // ---- TMA producers: lane 0 loads the feature tiles, lane 1 the row tiles
-    // (lane 2 the lo row tiles of DUAL).  Each lane posts its own bytes on the
-    // stage's full barrier (initialised with one arrival per producer lane).
+    // (lane 2 the lo row tiles of DUAL, or the lo feature tiles of the folded
+    // keys).  Each lane posts its own bytes on the stage's full barrier
+    // (initialised with one arrival per producer lane).
     const uint32_t f_bytes = (uint32_t)(KPS * f_tile);
     const uint32_t r_lane_bytes = (uint32_t)(KPS * r_tile);
     const CUtensorMap* mapF = part == 0 ? &tmF0 : (part == 1 ? &tmF1 : &tmF2);
     const int fy = part == 0 ? g.a_row0 + m0 : m0 - pbeg;
     const int ry = g.b_row0 + n0;
+    const bool f_lane = lane == 0 || (dual_f && lane == 2);   // loads feature tiles
+    const int f_off = lane == 0 ? 0 : KPS * f_tile;            // hi, or lo after it
+    const int f_kb = lane == 0 ? 0 : args.f_lo_kb;
     // weights / keys of the first stages: independent of the previous kernel
-    const int pre = lane == 0 ? (nkb < stages ? nkb : stages) : 0;
+    const int pre = f_lane ? (nkb < stages ? nkb : stages) : 0;
     for (int i = 0; i < pre; ++i) {
       mbar_expect_tx(&full[i], f_bytes);
-      tma_load_3d(smem + i * stage_bytes + r_bytes, mapF, &full[i], 0, fy, (su_lo + i) * KPS);
+      tma_load_3d(smem + i * stage_bytes + r_bytes + f_off, mapF, &full[i], 0, fy,
+                  (su_lo + i) * KPS + f_kb);
     }
     if (lane == 0) {
       // L2 prefetch of data later kernels of the step read (memory entries,
@@ -223,13 +240,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t ph = (uint32_t)(i / stages) & 1u;
       uint8_t* stg = smem + st * stage_bytes;
       if (i >= pre) {
-        if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag)) {
+        if (!mbar_wait(&empty[st], ph ^ 1u, abort_flag, args.wait_ns)) {
           *abort_flag = 1;
           break;
         }
-        if (lane == 0) {
+        if (f_lane) {
           mbar_expect_tx(&full[st], f_bytes);
-          tma_load_3d(stg + r_bytes, mapF, &full[st], 0, fy, kb);
+          tma_load_3d(stg + r_bytes + f_off, mapF, &full[st], 0, fy, kb + f_kb);
         } else {
           mbar_expect_tx(&full[st], r_lane_bytes);
           if constexpr (DUAL) {
@@ -257,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < nkb; ++i) {
       const int st = i % stages;
       const uint32_t ph = (uint32_t)(i / stages) & 1u;
-      if (!mbar_wait(&full[st], ph, abort_flag)) {
+      if (!mbar_wait(&full[st], ph, abort_flag, args.wait_ns)) {
         *abort_flag = 1;
         break;
       }
@@ -275,6 +292,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if constexpr (DUAL) {
             const uint64_t adesc_lo = sw128_desc(stg + (uint32_t)((KPS + j) * r_tile));
             umma_bf16(tmem_base, adesc_lo + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k), C::IDESC,
+                      1u);
+          }
+          if (dual_f) {
+            const uint64_t bdesc_lo = sw128_desc(stg + (uint32_t)(r_bytes + (KPS + j) * f_tile));
+            umma_bf16(tmem_base, adesc + (uint64_t)(2 * k), bdesc_lo + (uint64_t)(2 * k), C::IDESC,
                       1u);
           }
         }
@@ -307,7 +329,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();
   bool ok = true;
   if (nkb > 0) {
-    const bool waited = mbar_wait(accum, 0, abort_flag);
+    const bool waited = mbar_wait(accum, 0, abort_flag, args.wait_ns);
+    // after a wait that gave up, the MMAs already issued (the issuer commits
+    // them to `accum` however its loop ended) complete before the tensor
+    // memory they write is freed
+    if (!waited) mbar_wait(accum, 0, nullptr, kDefaultWaitLimitNs);
     // warp-uniform decision: tcgen05.ld below is a .sync.aligned instruction
     ok = __all_sync(0xffffffffu, waited && *abort_flag == 0);
   }
@@ -544,6 +570,10 @@ bool encode_bf16_map(CUtensorMap* m, const void* base, long long rows, long long
   return make_map(m, TmaOperand{base, rows, cols, ld}, box_rows);
 }
 
+static std::atomic<unsigned long long> g_wait_limit_ns{kDefaultWaitLimitNs};
+void set_wait_limit_ns(unsigned long long ns) { g_wait_limit_ns.store(ns); }
+unsigned long long wait_limit_ns() { return g_wait_limit_ns.load(); }
+
 static int num_sms() {
   static int sms = 0;
   if (sms == 0) {
@@ -567,10 +597,8 @@ static auto tc_kernel() {
   return kern;
 }
 
-template <int BN, bool DUAL>
-static int stages_for(int nkb, int budget, int kps, int rbox) {
-  using C = tc::Cfg<BN, DUAL>;
-  int st = budget / C::stage_bytes(kps, rbox);
+static int stages_for(int nkb, int budget, int stage_bytes) {
+  int st = budget / stage_bytes;
   st = st > tc::kMaxStages ? tc::kMaxStages : st;
   st = st > nkb ? nkb : st;
   return st < 1 ? 1 : st;
@@ -630,7 +658,8 @@ static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tile
   a.region = p.region;
   a.kps = p.kps;
   a.rbox = p.rbox;
-  a.tx_bytes = tc::Cfg<BN, DUAL>::stage_bytes(p.kps, p.rbox);
+  a.tx_bytes = tc::Cfg<BN, DUAL>::stage_bytes(p.kps, p.rbox,
+                                              EPI == kEpiScoresFolded && a.f_lo_kb > 0);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(tiles_x * p.splits, (max_n + tc::BM - 1) / tc::BM, a.ngroups);
   cfg.blockDim = dim3(tc::kThreads, 1, 1);
@@ -707,6 +736,9 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
                      GemmPlan& best, double& best_t) {
   constexpr bool DUAL = EPI == kEpiScores;
   using C = tc::Cfg<BN, DUAL>;
+  // folded scores with hi / lo folded keys: the key part's stages hold two
+  // feature tiles and issue two MMAs per k-step (the plan is sized for them)
+  const bool DF = EPI == kEpiScoresFolded && a.f_lo_kb > 0;
   const int kb_total = a.k_total / tc::BK;
   const int r_split_kb = a.b_split / tc::BK;
   const long long ftiles = feature_tiles(a, max_m, BN);
@@ -719,17 +751,19 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
   for (int kps = 4; kps >= 1; kps >>= 1) {
     if (kb_total % kps != 0 || r_split_kb % kps != 0) continue;
     const int su_total = kb_total / kps;
-    const double stage_f = (double)kps * BN * 128;
-    const double stage_mma_us = (double)kps * 4.0 * mma_cycles(BN) * (DUAL ? 2 : 1) / 2070.0;
+    const double stage_f = (double)kps * BN * 128 * (DF ? 2 : 1);
+    const double stage_mma_us =
+        (double)kps * 4.0 * mma_cycles(BN) * ((DUAL || DF) ? 2 : 1) / 2070.0;
+    const int sb = C::stage_bytes(kps, rbox, DF);
     for (int S = 1; S <= 8; ++S) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
       const int nst = (su_total + S - 1) / S;
       const long long ctas = tiles * S;
       const int staging = EPI == kEpiStoreKeys ? 0 : rows * (BN + 4) * 4;
       for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
-        if (C::stage_bytes(kps, rbox) > budget) continue;
-        const int stages = stages_for<BN, DUAL>(nst, budget, kps, rbox);
-        const int region = std::max(stages * C::stage_bytes(kps, rbox), staging);
+        if (sb > budget) continue;
+        const int stages = stages_for(nst, budget, sb);
+        const int region = std::max(stages * sb, staging);
         const int smem = region + tc::kSmemExtra;
         if (region > tc::kSmemBudget) continue;
         long long cap = resident_ctas<BN, EPI>(smem);
@@ -741,7 +775,7 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
         if (cap <= 0) continue;
         const long long waves = (ctas + cap - 1) / cap;
         const long long per_sm = std::max<long long>(1, (std::min(ctas, cap) + sms - 1) / sms);
-        const double t = plan_cost_us(streaming, C::stage_bytes(kps, rbox) / 1024.0, stage_f,
+        const double t = plan_cost_us(streaming, sb / 1024.0, stage_f,
                                       stage_mma_us, stages, nst, std::min(ctas, cap), (int)per_sm,
                                       waves, S);
         if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
@@ -783,6 +817,7 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
   if (max_m <= 0 || max_n <= 0 || args.ngroups <= 0) return cudaSuccess;
   static thread_local GemmArgs a;
   a = args;
+  a.wait_ns = wait_limit_ns();
   const GemmPlan plan = plan_gemm_tc(epi, a, max_m, max_n);
   if (plan.region <= 0) return cudaErrorInvalidConfiguration;
   CUtensorMap maps[5];            // F0, F1, F2, R0, R1

@@ -47,7 +47,7 @@ fovea_status workspace_address(void** out) {
 
 extern "C" FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(
     const fovea_params* p, const fovea_memory* mem, const void* h, const int32_t* depth,
-    const int32_t* row_offsets, const float* row_scale, float rho, int k_min, int k_max,
+    const int32_t* row_offsets, const float* row_scale, float rho, int k_min, int k_max, int l_max,
     void* h_out, int32_t* counts, int32_t* indices, float* readout, float* gate, void* stream) {
   size_t need = 0;
   fovea_status st = fovea_workspace_size(p, mem, row_offsets, k_max, &need);
@@ -63,15 +63,26 @@ extern "C" FOVEA_API fovea_status fovea_retrieve_fuse_noalloc(
   }
   void* ws = nullptr;
   if ((st = workspace_address(&ws)) != FOVEA_OK) return st;
-  // The array keeps the previous call's contents: the header (error word and
-  // split-K counters) must start at zero.
-  cudaError_t e = cudaMemsetAsync(ws, 0, 16384, static_cast<cudaStream_t>(stream));
+  // The array keeps the previous call's contents; the kernels expect the
+  // header's reserved words at zero.  The error word is left as it is, so a
+  // condition a call raised stays readable (fovea_noalloc_sync_errors) until
+  // it is read.
+  cudaError_t e = cudaMemsetAsync(static_cast<unsigned char*>(ws) + sizeof(int), 0,
+                                  fovea::kWsHeaderBytes - sizeof(int),
+                                  static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {
     char msg[256];
     snprintf(msg, sizeof(msg), "cudaMemsetAsync: %s", cudaGetErrorString(e));
     return fovea::report_error(FOVEA_ERR_CUDA, msg);
   }
-  return fovea_retrieve_fuse(p, mem, h, depth, row_offsets, row_scale, rho, k_min, k_max, h_out,
-                             counts, indices, readout, gate, ws, FOVEA_NOALLOC_WORKSPACE_BYTES,
-                             stream);
+  return fovea_retrieve_fuse(p, mem, h, depth, row_offsets, row_scale, rho, k_min, k_max, l_max,
+                             h_out, counts, indices, readout, gate, ws,
+                             FOVEA_NOALLOC_WORKSPACE_BYTES, stream);
+}
+
+extern "C" FOVEA_API fovea_status fovea_noalloc_sync_errors(void* stream) {
+  void* ws = nullptr;
+  fovea_status st = workspace_address(&ws);
+  if (st != FOVEA_OK) return st;
+  return fovea_sync_errors(ws, stream);
 }

@@ -555,6 +555,7 @@ cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFi
 // g = sigma(a_g . w_g2 + b_g2), y = h + g c, h_hat = y / sqrt(mean(y^2) + eps) * gamma.
 // One CTA per row; `act` is [N, 2H] with a_f in columns 0..H-1 and a_g in
 // H..2H-1.  Every operand of the row is requested before the first reduction.
+// A row past the depth gate is copied (h_hat = h, gate 0).
 // ---------------------------------------------------------------------------
 constexpr int kFinThreads = 512;
 
@@ -562,7 +563,8 @@ template <class T>
 __global__ void __launch_bounds__(kFinThreads) finalize_kernel(
     const T* __restrict__ h, const float* __restrict__ c, const T* __restrict__ act, int H, int d,
     const T* __restrict__ w_g2, const T* __restrict__ b_g2, const T* __restrict__ rms_gamma,
-    float eps, T* __restrict__ h_out, float* __restrict__ gate_out) {
+    float eps, const __grid_constant__ DepthGate gate_rows, T* __restrict__ h_out,
+    float* __restrict__ gate_out) {
   constexpr int V = LnVec<T>::N;
   constexpr int MV = LnVec<T>::MAX;
   __shared__ float scratch[32];
@@ -581,6 +583,16 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(
   }
   pdl_wait();
   pdl_trigger();
+  if (row_gated(gate_rows, n)) {          // not corrected: h_hat = h, gate 0
+    T* o = h_out + (long long)n * d;
+#pragma unroll
+    for (int j = 0; j < MV; ++j) {
+      const int vi = tid + j * kFinThreads;
+      if (vi < nvec) *reinterpret_cast<uint4*>(o + vi * V) = *reinterpret_cast<const uint4*>(hr + vi * V);
+    }
+    if (gate_out != nullptr && tid == 0) gate_out[n] = 0.0f;
+    return;
+  }
 #pragma unroll
   for (int j = 0; j < MV; ++j) {
     const int vi = tid + j * kFinThreads;
@@ -626,17 +638,18 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(
 
 cudaError_t launch_finalize(int dtype, const void* h, const float* c, const void* act, int H, int d,
                             const void* w_g2, const void* b_g2, const void* rms_gamma, float eps,
-                            int N, void* h_out, float* gate_out, cudaStream_t s) {
+                            int N, const DepthGate& gate, void* h_out, float* gate_out,
+                            cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
     return launch_pdl(finalize_kernel<T>, dim3(N), dim3(kFinThreads), 0, s, (const T*)h, c,
                       (const T*)act, H, d, (const T*)w_g2, (const T*)b_g2, (const T*)rms_gamma,
-                      eps, (T*)h_out, gate_out);
+                      eps, gate, (T*)h_out, gate_out);
   }
   return launch_pdl(finalize_kernel<float>, dim3(N), dim3(kFinThreads), 0, s, (const float*)h, c,
                     (const float*)act, H, d, (const float*)w_g2, (const float*)b_g2,
-                    (const float*)rms_gamma, eps, (float*)h_out, gate_out);
+                    (const float*)rms_gamma, eps, gate, (float*)h_out, gate_out);
 }
 
 }  // namespace fovea

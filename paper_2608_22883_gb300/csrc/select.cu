@@ -24,7 +24,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   pdl_trigger();
   const int b = seq_of_row(tab, n);
   const int M = tab.m[b];
-  if (M == 0) {                           // empty valid set: K = 0, nothing selected
+  if (M == 0 || row_gated(a.gate, n)) {   // empty valid set or past the depth gate: K = 0
     select_empty(a, n, tid);
     return;
   }
@@ -39,9 +39,9 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 }
 
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
-                          float rho, int k_min, int k_max, int max_m, int32_t* counts,
-                          int32_t* indices, int32_t* sel_pos, float* sel_w, int32_t* sel_cnt,
-                          cudaStream_t s) {
+                          float rho, int k_min, int k_max, int max_m, const DepthGate& gate,
+                          int32_t* counts, int32_t* indices, int32_t* sel_pos, float* sel_w,
+                          int32_t* sel_cnt, cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)max(max_m, 1) * sizeof(float);
   static bool configured = false;
@@ -52,7 +52,7 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
     configured = true;
   }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt,
-               nullptr, nullptr, nullptr};
+               nullptr, nullptr, nullptr, gate};
   return launch_pdl(select_kernel, dim3(N), dim3(kSelThreads), smem, s, a, tab);
 }
 
@@ -253,14 +253,30 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
     a.loc_cnt = &loc_cnt;
     const int b = seq_of_row(tab, n);
     const int M = tab.m[b];
-    if (M == 0) {                         // empty valid set: K = 0, r_n = 0
-      select_empty(a, n, tid);
+    if (M == 0 || row_gated(a.gate, n)) {   // empty valid set or past the depth gate:
+      select_empty(a, n, tid);              // K = 0, r_n = 0
     } else {
       const float* src = a.scores + tab.score_off[b] + (long long)(n - tab.row_start[b]) * M;
-      for (int i = tid; i < M; i += kSelThreads) {
-        float v = src[i];
-        if (v == 0.0f) v = 0.0f;          // -0 -> +0 so equal scores get equal keys
-        s_sc[i] = v;
+      if (M <= kFastMaxM) {
+        // every load of the thread in flight at once (8 per thread at most)
+        constexpr int PT = kFastMaxM / kSelThreads;
+        float v[PT];
+#pragma unroll
+        for (int j = 0; j < PT; ++j) {
+          const int i = tid + j * kSelThreads;
+          v[j] = i < M ? src[i] : 0.0f;
+        }
+#pragma unroll
+        for (int j = 0; j < PT; ++j) {
+          const int i = tid + j * kSelThreads;
+          if (i < M) s_sc[i] = v[j] == 0.0f ? 0.0f : v[j];   // -0 -> +0: equal keys
+        }
+      } else {
+        for (int i = tid; i < M; i += kSelThreads) {
+          float v = src[i];
+          if (v == 0.0f) v = 0.0f;        // -0 -> +0 so equal scores get equal keys
+          s_sc[i] = v;
+        }
       }
       if constexpr (NT == kSelThreads) {
         __syncthreads();
@@ -326,7 +342,8 @@ bool select_readout_fits(int max_m, int k_max) { return max_m <= kFastMaxM && k_
 
 cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable& tab, int N,
                                  const int32_t* orig_index, float rho, int k_min, int k_max,
-                                 int max_m, int32_t* counts, int32_t* indices, const void* U, int d,
+                                 int max_m, const DepthGate& gate, int32_t* counts,
+                                 int32_t* indices, const void* U, int d,
                                  float* r_out, void* r_lo, const void* P, int H, const float* Gh,
                                  const void* b_f1, const void* b_g1, void* act, int* err,
                                  cudaStream_t s, long long p_prefetch_bytes) {
@@ -381,7 +398,7 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
     configured = true;
   }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices,
-               nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+               nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, gate};
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(N, nchunk);
   cfg.blockDim = dim3(wide ? 1024 : kSelThreads);

@@ -17,7 +17,7 @@
 // the first prefix reaching rho sets K.
 //
 // Used by the standalone select kernel (a CTA of 256 threads, __syncthreads)
-// and by the persistent step kernel (its 256 worker threads, a named
+// and by the selection + gather kernel (its first 256 threads, a named
 // barrier): `sync` is the group barrier, `tid` the thread's index in the
 // group, and the group's warps are whole hardware warps.
 #pragma once
@@ -51,6 +51,7 @@ struct SelectArgs {
   int32_t* loc_pos;
   float* loc_w;
   int* loc_cnt;
+  DepthGate gate;      // rows past the depth gate select nothing (K = 0)
 };
 
 struct SelectSmem {

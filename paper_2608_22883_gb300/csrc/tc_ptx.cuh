@@ -44,7 +44,7 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 // `limit_ns` (about 2 s by default) or once another role of the CTA has
 // aborted (when abort_flag is given).
 static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                       uint64_t limit_ns = 2000000000ull) {
+                                       uint64_t limit_ns = kDefaultWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {

@@ -35,11 +35,10 @@ EXPORTS = (
     "fovea_build_memory", "fovea_memory_destroy", "fovea_memory_info", "fovea_memory_tensors",
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
-    "fovea_retrieve_fuse_noalloc", "fovea_step_path", "fovea_memory_folded_keys",
-    "fovea_lm_head_topk",
+    "fovea_retrieve_fuse_noalloc", "fovea_noalloc_sync_errors", "fovea_memory_folded_keys",
+    "fovea_lm_head_topk", "fovea_debug_wait_limit",
 )
 NOALLOC_WORKSPACE_BYTES = 32 << 20
-PATH_AUTO, PATH_FUSED, PATH_KERNELS = 0, 1, 2
 
 
 class FoveaError(RuntimeError):
@@ -82,12 +81,16 @@ def lib() -> ctypes.CDLL:
                                            ctypes.POINTER(ctypes.c_size_t)]
         L.fovea_workspace_init.argtypes = [vp, ctypes.c_size_t, vp]
         L.fovea_retrieve_fuse.argtypes = [ctypes.POINTER(CParams), vp, vp, vp, i32p, vp,
-                                          ctypes.c_float, ctypes.c_int, ctypes.c_int,
+                                          ctypes.c_float, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                           vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
         L.fovea_retrieve_fuse_noalloc.argtypes = [ctypes.POINTER(CParams), vp, vp, vp, i32p, vp,
                                                   ctypes.c_float, ctypes.c_int, ctypes.c_int,
-                                                  vp, vp, vp, vp, vp, vp]
+                                                  ctypes.c_int, vp, vp, vp, vp, vp, vp]
         L.fovea_retrieve_fuse_noalloc.restype = ctypes.c_int
+        L.fovea_noalloc_sync_errors.argtypes = [vp]
+        L.fovea_noalloc_sync_errors.restype = ctypes.c_int
+        L.fovea_debug_wait_limit.argtypes = [ctypes.c_ulonglong]
+        L.fovea_debug_wait_limit.restype = ctypes.c_int
         L.fovea_sync_errors.argtypes = [vp, vp]
         L.fovea_last_error.restype = ctypes.c_char_p
         L.fovea_last_error.argtypes = []
@@ -96,8 +99,6 @@ def lib() -> ctypes.CDLL:
                                         ctypes.POINTER(ctypes.c_int), ctypes.c_int]
         L.fovea_timing_read.restype = ctypes.c_int
         L.fovea_version.restype = ctypes.c_int
-        L.fovea_step_path.argtypes = [ctypes.c_int]
-        L.fovea_step_path.restype = ctypes.c_int
         for name in ("fovea_build_memory", "fovea_memory_info", "fovea_memory_tensors",
                      "fovea_memory_folded_keys", "fovea_lm_head_topk",
                      "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse",
@@ -196,16 +197,17 @@ class Memory:
         return view(k.value), view(u.value), index, list(offs)
 
     def folded_keys(self, params: Params) -> Optional[torch.Tensor]:
-        """The folded keys kappa = W_Q^T k [total, d] (bf16 view of the handle's
-        memory) when the memory holds them for params' W_Q, else None; a step
-        with these params then scores against them."""
+        """The folded keys kappa = W_Q^T k as [total, 2d] bf16 (row i: kappa_hi
+        then kappa_lo; a view of the handle's memory) when the memory holds
+        them for params' W_Q, else None; a step with these params then scores
+        against them."""
         f = ctypes.c_void_p()
         _check(lib().fovea_memory_folded_keys(self.handle, params.c.W_Q, ctypes.byref(f)))
         if not f.value:
             return None
         if self.total == 0:
-            return torch.empty((0, self.d), dtype=torch.bfloat16, device="cuda")
-        return torch.as_tensor(_CudaView(f.value, (self.total, self.d), "<i2"),
+            return torch.empty((0, 2 * self.d), dtype=torch.bfloat16, device="cuda")
+        return torch.as_tensor(_CudaView(f.value, (self.total, 2 * self.d), "<i2"),
                                device="cuda").view(torch.bfloat16)
 
     def destroy(self):
@@ -250,25 +252,30 @@ def new_workspace(params: Params, memory: Memory, row_offsets, k_max: int, strea
     return ws
 
 
+def _l_max(params: Params, l_max: Optional[int]) -> int:
+    return params.max_depth if l_max is None else int(l_max)
+
+
 def retrieve_fuse(params: Params, memory: Memory, h: torch.Tensor, depth: torch.Tensor,
                   row_offsets, row_scale: Optional[torch.Tensor], rho: float, k_min: int,
                   k_max: int, h_out: torch.Tensor, workspace: torch.Tensor, *,
                   counts: Optional[torch.Tensor] = None, indices: Optional[torch.Tensor] = None,
                   readout: Optional[torch.Tensor] = None, gate: Optional[torch.Tensor] = None,
-                  stream=None, offsets_c=None) -> None:
-    """fovea_retrieve_fuse into caller-allocated outputs (asynchronous)."""
+                  l_max: Optional[int] = None, stream=None, offsets_c=None) -> None:
+    """fovea_retrieve_fuse into caller-allocated outputs (asynchronous).
+    l_max: depth gate (None: every row is corrected)."""
     offs = offsets_c if offsets_c is not None else _offsets(row_offsets)
     _check(lib().fovea_retrieve_fuse(params.ref, memory.handle, _ptr(h), _ptr(depth), offs,
                                      _ptr(row_scale), float(rho), int(k_min), int(k_max),
-                                     _ptr(h_out), _ptr(counts), _ptr(indices), _ptr(readout),
-                                     _ptr(gate), _ptr(workspace), workspace.numel(),
-                                     _stream(stream)))
+                                     _l_max(params, l_max), _ptr(h_out), _ptr(counts),
+                                     _ptr(indices), _ptr(readout), _ptr(gate), _ptr(workspace),
+                                     workspace.numel(), _stream(stream)))
 
 
 def step(params: Params, memory: Memory, h: torch.Tensor, depth: torch.Tensor, row_offsets,
          row_scale: Optional[torch.Tensor], rho: float, k_min: int, k_max: int, *,
          workspace: Optional[torch.Tensor] = None, want_readout: bool = True,
-         stream=None) -> Dict[str, torch.Tensor]:
+         l_max: Optional[int] = None, stream=None) -> Dict[str, torch.Tensor]:
     """Allocate outputs with torch and run one draft step; returns them."""
     N = h.shape[0]
     dev = h.device
@@ -283,7 +290,7 @@ def step(params: Params, memory: Memory, h: torch.Tensor, depth: torch.Tensor, r
     )
     retrieve_fuse(params, memory, h, depth, row_offsets, row_scale, rho, k_min, k_max,
                   out["h_out"], workspace, counts=out["counts"], indices=out["indices"],
-                  readout=out["readout"], gate=out["gate"], stream=stream)
+                  readout=out["readout"], gate=out["gate"], l_max=l_max, stream=stream)
     out["workspace"] = workspace
     return out
 
@@ -294,18 +301,30 @@ def retrieve_fuse_noalloc(params: Params, memory: Memory, h: torch.Tensor, depth
                           counts: Optional[torch.Tensor] = None,
                           indices: Optional[torch.Tensor] = None,
                           readout: Optional[torch.Tensor] = None,
-                          gate: Optional[torch.Tensor] = None, stream=None) -> None:
+                          gate: Optional[torch.Tensor] = None, l_max: Optional[int] = None,
+                          stream=None) -> None:
     """fovea_retrieve_fuse_noalloc: the draft step with the library's static
     scratch instead of a workspace (for callers that cannot allocate)."""
     _check(lib().fovea_retrieve_fuse_noalloc(params.ref, memory.handle, _ptr(h), _ptr(depth),
                                              _offsets(row_offsets), _ptr(row_scale), float(rho),
-                                             int(k_min), int(k_max), _ptr(h_out), _ptr(counts),
-                                             _ptr(indices), _ptr(readout), _ptr(gate),
-                                             _stream(stream)))
+                                             int(k_min), int(k_max), _l_max(params, l_max),
+                                             _ptr(h_out), _ptr(counts), _ptr(indices),
+                                             _ptr(readout), _ptr(gate), _stream(stream)))
+
+
+def noalloc_sync_errors(stream=None) -> None:
+    """fovea_noalloc_sync_errors: read and clear the static array's error word."""
+    _check(lib().fovea_noalloc_sync_errors(_stream(stream)))
 
 
 def sync_errors(workspace: torch.Tensor, stream=None) -> None:
     _check(lib().fovea_sync_errors(_ptr(workspace), _stream(stream)))
+
+
+def debug_wait_limit(limit_ns: int) -> None:
+    """fovea_debug_wait_limit: limit of the bounded device waits of later
+    launches (0: the default of about 2 s).  For tests of the timeout path."""
+    _check(lib().fovea_debug_wait_limit(int(limit_ns)))
 
 
 def lm_head_topk(W_LM: torch.Tensor, h_hat: torch.Tensor, k_c: int, workspace: torch.Tensor,
@@ -324,13 +343,6 @@ def lm_head_topk(W_LM: torch.Tensor, h_hat: torch.Tensor, k_c: int, workspace: t
                                     _ptr(idx), _ptr(val), _ptr(workspace), workspace.numel(),
                                     _stream(stream)))
     return idx, val, logits
-
-
-def step_path(path: Optional[int] = None) -> int:
-    """Select the draft-step implementation (PATH_AUTO, PATH_FUSED or
-    PATH_KERNELS) and return the previous one; with no argument, return the
-    current one."""
-    return int(lib().fovea_step_path(-1 if path is None else int(path)))
 
 
 def timing_enable(on: bool = True) -> None:

@@ -16,6 +16,15 @@ the boundary exemption spelled out):
   <= 1e-4 for fp32.
 The order inside a selected list is compared up to swaps of entries whose
 scores lie within the same tie band.
+
+The oracle is always the paper-order form (q = W_Q x against the keys), also
+for GPU steps that score against the memory's folded keys: the folded keys
+carry kappa = W_Q^T k as a hi / lo pair, so both forms agree with q . k to
+within fp32 accumulation, far inside the boundary band.
+
+Boundary rows are reported by kind ("mass": the mass reading; "tie": the tie
+reading of the cut), and a caller bounds their share (``max_exempt``), so a
+band that swallows many rows fails instead of passing silently.
 """
 
 from __future__ import annotations
@@ -31,6 +40,10 @@ import workloads
 
 BAND = 1e-4
 TOL = {"bf16": 2e-2, "fp32": 1e-4}
+# The gate g = sigma(a_g . w_g2 + b_g2) lies in (0, 1); its absolute error
+# comes from the bf16 activations a_g (one ulp flips of single elements move
+# the sum by ~1e-4) and from the projected readout's fp32 sum.
+GATE_TOL = {"bf16": 5e-3, "fp32": 1e-5}
 # The library receives its epsilons as fp32; the oracle uses the same values.
 LN_EPS = float(np.float32(1e-5))
 RMS_EPS = float(np.float32(1e-6))
@@ -93,7 +106,10 @@ class RowReport:
 def classify_rows(orc: dict, w: workloads.Workload, rows) -> Dict[int, str]:
     """Rows whose decision sits on a boundary: the cumulative mass lies within
     BAND of rho at K_raw (or K_raw - 1) and moving K_raw by one would change the
-    clamped count K, or the cut falls inside a score tie band."""
+    clamped count K ("mass"), or the cut falls inside a score tie band
+    ("cut-tie": the order of equal scores is a reading, so a cut between
+    near-equal scores decides nothing the paper fixes).  Rows past the depth
+    gate have no selection and are never boundary rows."""
     rho = float(np.float32(w.rho))
     out = {}
     for n in rows:
@@ -129,19 +145,35 @@ def rel_err_rows(x: np.ndarray, ref: np.ndarray) -> np.ndarray:
 
 
 def compare(gpu: Dict[str, np.ndarray], orc: dict, s: Stored, rows=None,
-            mem: Optional[oracle.Memory] = None, mirror: bool = True) -> dict:
+            mem: Optional[oracle.Memory] = None, mirror: bool = True,
+            max_exempt: float = 0.05) -> dict:
     """Assert parity of GPU outputs with the oracle on `rows` (default: all).
-    Returns a summary dict (exempt rows, max errors)."""
+    At most a `max_exempt` share of the rows may be boundary rows.  Returns a
+    summary dict (exempt rows by kind, max errors)."""
     w = s.w
     N = w.N
     rows = list(range(N)) if rows is None else list(rows)
     tol = TOL[w.dtype]
     exempt = classify_rows(orc, w, rows)
+    n_mass = sum(1 for r in exempt.values() if "mass" in r)
+    n_tie = sum(1 for r in exempt.values() if "cut-tie" in r)
+    assert len(exempt) <= max(3, max_exempt * len(rows)), \
+        f"{len(exempt)} boundary rows of {len(rows)} ({n_mass} mass, {n_tie} tie) exceed {max_exempt:.0%}"
     p = oracle_params(s)
     ref_r = orc["readout"].copy()
     ref_h = orc["h_out"].copy()
     ref_g = orc["gate"].copy()
+    gated = orc.get("gated")
+    differ = []                  # boundary rows whose GPU selection is not the oracle's
     for n in rows:
+        if gated is not None and gated[n]:
+            # past the depth gate: not corrected, bit for bit
+            assert int(gpu["counts"][n]) == 0, f"gated row {n}: count {gpu['counts'][n]}"
+            assert np.all(gpu["indices"][n] == -1), f"gated row {n}: indices set"
+            assert np.array_equal(gpu["h_out"][n].astype(np.float64), s.f64["h"][n]), \
+                f"gated row {n}: h_out differs from h"
+            assert gpu["gate"][n] == 0.0
+            continue
         K_o = int(orc["counts"][n])
         K_g = int(gpu["counts"][n])
         idx_g = [int(x) for x in gpu["indices"][n, :K_g]]
@@ -155,6 +187,8 @@ def compare(gpu: Dict[str, np.ndarray], orc: dict, s: Stored, rows=None,
                 _check_order(orc, w, mem, n, idx_g)
             continue
         # boundary row: checked separately
+        if K_g != K_o or sorted(idx_g) != sorted(int(x) for x in orc["indices"][n, :K_o]):
+            differ.append(n)
         assert abs(K_g - K_o) <= 1, f"boundary row {n}: count {K_g} vs oracle {K_o}"
         b = int(orc["seq_of"][n])
         pos_of = {int(i): j for j, i in enumerate(mem.index[b])}
@@ -173,8 +207,9 @@ def compare(gpu: Dict[str, np.ndarray], orc: dict, s: Stored, rows=None,
     eg = np.abs(gpu["gate"][rows] - ref_g[rows]).max() if len(rows) else 0.0
     assert er.max() <= tol, f"readout max rel err {er.max():.3e} > {tol} (row {rows[int(er.argmax())]})"
     assert eh.max() <= tol, f"h_out max rel err {eh.max():.3e} > {tol} (row {rows[int(eh.argmax())]})"
-    assert eg <= (2e-2 if w.dtype == "bf16" else 1e-5), f"gate max abs err {eg:.3e}"
-    return dict(exempt=exempt, readout_err=float(er.max()), h_out_err=float(eh.max()),
+    assert eg <= GATE_TOL[w.dtype], f"gate max abs err {eg:.3e}"
+    return dict(exempt=exempt, exempt_mass=n_mass, exempt_tie=n_tie, exempt_differ=differ,
+                readout_err=float(er.max()), h_out_err=float(eh.max()),
                 gate_err=float(eg), rows=len(rows))
 
 
@@ -188,33 +223,29 @@ def _check_order(orc, w, mem, n, idx_g):
         assert a >= c - BAND * max(1.0, abs(a)) * 4, f"row {n}: selected list not in descending order"
 
 
-def run_gpu(s: Stored, fovea, params=None, memory=None):
+def run_gpu(s: Stored, fovea, params=None, memory=None, l_max=None):
     """Build the memory and run one step through the C ABI; returns numpy outputs."""
     w = s.w
     params = params or params_for(s, fovea)
     mem = memory or fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
     out = fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets,
-                     s.dev.get("row_scale"), w.rho, w.k_min, w.k_max)
+                     s.dev.get("row_scale"), w.rho, w.k_min, w.k_max, l_max=l_max)
     fovea.sync_errors(out["workspace"])
     res = {k: (v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy())
            for k, v in out.items() if v is not None and k != "workspace"}
     res["_memory"] = mem
     res["_params"] = params
-    res["_folded"] = step_is_folded(fovea, params, mem)
+    res["_folded"] = mem.folded_keys(params) is not None
     return res
 
 
-def step_is_folded(fovea, params, mem) -> bool:
-    """True when a per-stage step with these params scores against the
-    memory's folded keys (the persistent step kernel never does)."""
-    return fovea.step_path() != fovea.PATH_FUSED and mem.folded_keys(params) is not None
-
-
-def run_oracle(s: Stored, mirror: bool, rows=None, fold: bool = False):
+def run_oracle(s: Stored, mirror: bool, rows=None, l_max=None):
+    """The oracle in the paper's order of operations (q = W_Q x against the
+    keys), in mirror mode for bf16 workloads."""
     w = s.w
     p = oracle_params(s)
     mem = oracle.build_memory(p, s.f64["v"], s.f64.get("mask"), mirror=mirror, ln_eps=LN_EPS)
     out = oracle.retrieve_fuse(p, mem, s.f64["h"], s.f64["depth"], w.row_offsets,
                                s.f64.get("row_scale"), w.rho, w.k_min, w.k_max, mirror=mirror,
-                               rows=rows, ln_eps=LN_EPS, rms_eps=RMS_EPS, fold=fold)
+                               rows=rows, ln_eps=LN_EPS, rms_eps=RMS_EPS, l_max=l_max)
     return out, mem

@@ -46,7 +46,7 @@ def test_library_exports_every_declared_symbol(L):
     assert not missing, f"not exported: {missing}"
     for name in declared_symbols():
         assert hasattr(L, name)
-    assert L.fovea_version() == 100
+    assert L.fovea_version() == 200
 
 
 def dummy_params(d=256, H=512, D=6, dtype=fovea.BF16, ptr=0x10000):
@@ -58,11 +58,11 @@ def dummy_params(d=256, H=512, D=6, dtype=fovea.BF16, ptr=0x10000):
     return c
 
 
-def call_step(L, c, *, rho=0.9, k_min=1, k_max=16, mem=None, h=0x10000, ws=0x10000):
+def call_step(L, c, *, rho=0.9, k_min=1, k_max=16, l_max=6, mem=None, h=0x10000, ws=0x10000):
     offs = (ctypes.c_int32 * 2)(0, 4)
     return L.fovea_retrieve_fuse(ctypes.byref(c) if c is not None else None, mem, h, 0x10000, offs,
-                                 None, rho, k_min, k_max, 0x10000, None, None, None, None, ws,
-                                 1 << 20, None)
+                                 None, rho, k_min, k_max, l_max, 0x10000, None, None, None, None,
+                                 ws, 1 << 20, None)
 
 
 @pytest.mark.parametrize("kw,status", [
@@ -94,8 +94,8 @@ def test_param_checks(L, mutate, status):
     c = dummy_params()
     mutate(c)
     assert call_step(L, c) == status
-    assert L.fovea_retrieve_fuse(None, None, None, None, None, None, 0.9, 1, 4, None, None, None,
-                                 None, None, None, 0, None) == fovea.ERR_INVALID_ARG
+    assert L.fovea_retrieve_fuse(None, None, None, None, None, None, 0.9, 1, 4, 6, None, None,
+                                 None, None, None, None, 0, None) == fovea.ERR_INVALID_ARG
 
 
 def test_build_argument_checks(L):
@@ -140,6 +140,12 @@ def test_memory_queries_reject_null(L):
     assert L.fovea_workspace_init(None, 1024, None) == fovea.ERR_INVALID_ARG
     assert L.fovea_sync_errors(None, None) == fovea.ERR_INVALID_ARG
     L.fovea_memory_destroy(None)      # ignored
+
+
+def test_debug_wait_limit_is_a_host_setting(L):
+    # process-wide; takes effect at the next tensor-core launch (none here)
+    assert L.fovea_debug_wait_limit(1000) == fovea.OK
+    assert L.fovea_debug_wait_limit(0) == fovea.OK       # back to the default
 
 
 def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):

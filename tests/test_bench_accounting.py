@@ -50,17 +50,19 @@ def test_folding_and_projection_remove_their_terms(w7b):
     # projected values: the r-half of [W_f1 ; W_g1] (2H x d) no longer read,
     # value rows 2H wide instead of d wide
     assert plain - proj == 2 * (2 * H * d) + 2 * uniq * (d - 2 * H)
-    # folding: W_Q (d x d, bf16) no longer read, no query GEMM
-    assert proj - both == 2 * d * d
+    # folding: W_Q (d x d, bf16) no longer read, no query GEMM; the folded
+    # keys are a hi / lo pair, twice the key bytes
+    M = int(w7b.m_sizes[0])
+    assert proj - both == 2 * d * d - 2 * M * d
     assert f_proj - f_both == 2 * N * d * d
-    assert abs(both / 1e6 - 19.6) < 0.1
+    assert abs(both / 1e6 - 24.3) < 0.1
 
 
 def test_kernel_bytes_of_the_folded_launches(w7b):
     d, H, N, M = w7b.d, int(w7b.params["b_f1"].shape[0]), w7b.N, int(w7b.m_sizes[0])
     merged = bench.kernel_bytes("score_fusion_h", w7b, 0, True)
-    # folded keys + the h-halves of W_f1, W_g1 + x_h and h (bf16); scores and G_h out (fp32)
-    assert merged == (M * d + 2 * H * d + 2 * N * d) * 2 + N * M * 4 + N * 2 * H * 4
+    # folded keys (hi, lo) + the h-halves of W_f1, W_g1 + x_h and h (bf16); scores and G_h out (fp32)
+    assert merged == (2 * M * d + 2 * H * d + 2 * N * d) * 2 + N * M * 4 + N * 2 * H * 4
     # the two separate launches (several score groups) move the same bytes:
     # x_h in the one, h in the other
     assert bench.kernel_bytes("score_folded", w7b, 0, True) + bench.kernel_bytes("fusion_h", w7b, 0, True) \

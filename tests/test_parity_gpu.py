@@ -3,13 +3,14 @@
 Small cases span several 128-row tiles, ragged tails, masks, empty and single
 entry memories, the selection clamps (k_max = 1, k_max > |V|, the paper's
 rho = 0.8 / K_min = 32 / K_max = 256, fixed top-16, dense), per-row
-temperatures, clustered keys and the fp32 path.  The five named workloads run
-at full size (the long-memory one on sampled rows and steps).
+temperatures, clustered keys, the depth gate and the fp32 path.  The five
+named workloads run at full size (the long-memory one on every row of four of
+its hundred steps).
 
-Every parity test runs on both implementations of the draft step: "fused"
-(the persistent step kernel, which covers every bf16 case here except the
-long-memory one; fp32 cases skip it) and "kernels" (one kernel per stage,
-the default).
+The oracle is always the paper's order of operations: q = W_Q (LN(h) + E_dep)
+scored against the keys.  The default bf16 step scores x = LN(h) + E_dep
+against the memory's folded keys W_Q^T k (a hi / lo pair), and is held to the
+same oracle.
 """
 
 import dataclasses
@@ -20,7 +21,7 @@ import torch
 
 import oracle
 import workloads
-from parity import (compare, params_for, rel_err_rows, run_gpu, run_oracle, step_is_folded,
+from parity import (LN_EPS, RMS_EPS, compare, params_for, rel_err_rows, run_gpu, run_oracle,
                     store)
 
 pytestmark = pytest.mark.gpu
@@ -32,21 +33,6 @@ def fovea():
     from paper_2608_22883_gb300 import fovea as f
     f.lib()          # raises if the library was not built: no fallback
     return f
-
-
-PATHS = {"fused": 1, "kernels": 2}
-
-
-@pytest.fixture(params=sorted(PATHS))
-def path(request, fovea):
-    prev = fovea.step_path(PATHS[request.param])
-    yield request.param
-    fovea.step_path(prev)
-
-
-def skip_fp32_on_fused(path, dtype):
-    if path == "fused" and dtype != "bf16":
-        pytest.skip("the persistent step kernel covers bf16 calls only")
 
 
 SMALL = {
@@ -83,16 +69,24 @@ def small_workload(name):
     return workloads.generate_custom(name, kw.pop("d"), kw.pop("m_sizes"), kw.pop("rows"), **kw)
 
 
+# Boundary-row share allowed per small case (at least three rows; the
+# boundary rows follow from the oracle alone, so the counts are fixed per
+# seeded case): clustered keys cut between near-equal scores, temperatures
+# up to 10 widen the score scale, and the paper's defaults with K_min = 32
+# sit near the mass threshold on a few rows.
+SMALL_MAX_EXEMPT = {"bf16-clustered": 0.1, "bf16-temperature": 0.1, "bf16-paper-defaults": 0.1}
+
+
 @pytest.mark.parametrize("name", sorted(SMALL))
-def test_small_parity(fovea, path, name):
+def test_small_parity(fovea, name):
     w = small_workload(name)
-    skip_fp32_on_fused(path, w.dtype)
     s = store(w)
     gpu = run_gpu(s, fovea)
-    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"), fold=gpu["_folded"])
-    rep = compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"))
+    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
+    rep = compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"),
+                  max_exempt=SMALL_MAX_EXEMPT.get(name, 0.05))
     print(f"{name} (folded: {gpu['_folded']}): boundary rows {rep['exempt']}, readout err {rep['readout_err']:.2e}, "
-          f"h_out err {rep['h_out_err']:.2e}")
+          f"h_out err {rep['h_out_err']:.2e}, gate err {rep['gate_err']:.2e}")
 
 
 @pytest.mark.parametrize("name", ["bf16-ragged", "bf16-scattered-mask-d320", "fp32-ragged",
@@ -111,20 +105,23 @@ def test_memory_build_matches_oracle(fovea, name):
     kappa = mem.folded_keys(params)
     assert (kappa is not None) == (w.dtype == "bf16" and mem.total > 0)
     if kappa is not None:
-        orc = oracle.fold_keys({n: s.f64[n] for n in workloads.PARAM_NAMES}, orc, mirror=True)
+        # the exact fold of the (bf16) keys: the GPU keeps it as hi + lo
+        orc = oracle.fold_keys({n: s.f64[n] for n in workloads.PARAM_NAMES}, orc, mirror=False)
+        kappa = kappa.double().cpu().numpy()
+        kappa = kappa[:, :w.d] + kappa[:, w.d:]
     for b in range(w.B):
         lo, hi = offs[b], offs[b + 1]
         np.testing.assert_array_equal(idx[lo:hi], orc.index[b])
         if hi == lo:
             continue
-        pairs = [(K, orc.keys[b]), (U, orc.values[b])]
-        if kappa is not None:
-            pairs.append((kappa, orc.folded[b]))
-        for got, ref in pairs:
+        for got, ref in [(K, orc.keys[b]), (U, orc.values[b])]:
             g = got[lo:hi].double().cpu().numpy()
             assert rel_err_rows(g, ref).max() <= tol
             if w.dtype == "bf16":
                 assert np.mean(g == ref) > 0.99     # same bf16 value almost everywhere
+        if kappa is not None:
+            # about 16 significant bits plus the fp32 accumulation of W_Q^T k
+            assert rel_err_rows(kappa[lo:hi], orc.folded[b]).max() <= 2e-4
     mem.destroy()
 
 
@@ -141,7 +138,7 @@ def test_plain_fusion_when_weights_differ(fovea):
     fovea.timing_enable(True)
     proj = run_gpu(s, fovea, params=params)
     names_proj = set(fovea.timing_read())
-    orc, mem = run_oracle(s, mirror=True, fold=proj["_folded"])
+    orc, mem = run_oracle(s, mirror=True)
     weights = {n: s.dev[n] for n in workloads.PARAM_NAMES}
     weights["W_f1"] = weights["W_f1"].clone()
     weights["W_g1"] = weights["W_g1"].clone()
@@ -161,13 +158,15 @@ def test_plain_fusion_when_weights_differ(fovea):
     assert rel_err_rows(proj["h_out"].astype(np.float64), plain["h_out"].astype(np.float64)).max() <= 2e-2
 
 
-def test_unfolded_scores_when_memory_has_no_folded_keys(fovea):
+@pytest.mark.parametrize("name", ["bf16-temperature", "bf16-clustered", "bf16-paper-defaults"])
+def test_folded_and_unfolded_steps_select_the_same_entries(fovea, name):
     """A memory built without W_Q holds no folded keys: the step then forms
     q = W_Q x_h (hi / lo pair) and scores it against the keys, the paper's
-    own order, and matches the unfolded oracle.  A memory built with W_Q
-    scores x_h against kappa = W_Q^T k and matches the folded oracle; the
-    two agree on every non-boundary row's selection."""
-    w = small_workload("bf16-temperature")
+    own order.  A memory built with W_Q scores x_h against the folded keys
+    (hi / lo pair).  Both match the paper-order oracle, and both give the
+    same counts and the same ordered index lists on every row outside the
+    boundary band."""
+    w = small_workload(name)
     s = store(w)
     params = params_for(s, fovea)
     no_wq = {n: s.dev[n] for n in workloads.PARAM_NAMES if n != "W_Q"}
@@ -183,56 +182,70 @@ def test_unfolded_scores_when_memory_has_no_folded_keys(fovea):
     names_folded = set(fovea.timing_read())
     fovea.timing_enable(False)
     assert not plain["_folded"] and folded["_folded"]
-    assert {"query_proj", "score"} <= names_plain and "score_folded" not in names_plain
-    assert {"fusion_h", "score_folded"} <= names_folded and "query_proj" not in names_folded
-    orc_p, mem_p = run_oracle(s, mirror=True, fold=False)
-    orc_f, mem_f = run_oracle(s, mirror=True, fold=True)
-    rp = compare(plain, orc_p, s, mem=mem_p, mirror=True)
-    rf = compare(folded, orc_f, s, mem=mem_f, mirror=True)
-    same = [n for n in range(w.N) if n not in rp["exempt"] and n not in rf["exempt"]]
+    assert "query_proj" in names_plain and not any(n.startswith("score_f") for n in names_plain)
+    assert "query_proj" not in names_folded
+    assert any(n in names_folded for n in ("score_folded", "score_fusion_h"))
+    orc, mem = run_oracle(s, mirror=True)
+    cap = SMALL_MAX_EXEMPT.get(name, 0.05)
+    rp = compare(plain, orc, s, mem=mem, mirror=True, max_exempt=cap)
+    rf = compare(folded, orc, s, mem=mem, mirror=True, max_exempt=cap)
+    same = [n for n in range(w.N) if n not in rp["exempt"]]
     np.testing.assert_array_equal(plain["counts"][same], folded["counts"][same])
+    for n in same:
+        assert sorted(plain["indices"][n]) == sorted(folded["indices"][n]), f"row {n}: sets differ"
+    # the order inside a list may differ only between near-equal scores (both
+    # lists passed the oracle's order check above)
+    differ = [n for n in range(w.N) if set(plain["indices"][n]) != set(folded["indices"][n])]
+    reordered = [n for n in range(w.N) if n not in differ
+                 and not np.array_equal(plain["indices"][n], folded["indices"][n])]
+    print(f"{name}: rows whose selected sets differ between the folded and unfolded steps: "
+          f"{differ} (boundary rows {sorted(rp['exempt'])}); same set, near-tie order swapped: "
+          f"{len(reordered)}")
 
 
 def test_paths_are_taken(fovea):
-    """AUTO runs the per-stage kernels: for bf16 rows of up to 2048 entries
-    the selection, the projected readout and the first fusion layer's
-    activation in one kernel; beyond that, selection and readout as two
-    kernels and the first fusion layer as a GEMM.  FUSED runs the persistent
-    step kernel for a bf16 call and refuses an fp32 one (outside its
-    coverage)."""
-    prev = fovea.step_path(fovea.PATH_AUTO)
+    """bf16 rows of up to 2048 entries run the selection, the projected
+    readout and the first fusion layer's activation in one kernel; beyond
+    that, selection and readout run as two kernels and the first fusion layer
+    as a GEMM; fp32 takes the unfolded SIMT path."""
     try:
-        for path, name, want, absent in (
-                (fovea.PATH_AUTO, "bf16-ragged",
+        for name, want, absent in (
+                ("bf16-ragged",
                  {"ln_query", "fusion_h", "score_folded", "select_fuse", "fuse_out", "finalize"},
                  "fuse_hidden"),
-                (fovea.PATH_AUTO, "bf16-paper-defaults",
-                 {"ln_query", "score_fusion_h", "select_fuse", "fuse_out", "finalize"},
-                 "fusion_h"),
-                (fovea.PATH_AUTO, "bf16-one-group-offset", {"score_fusion_h", "select_fuse"},
-                 "score_folded"),
-                (fovea.PATH_AUTO, "bf16-long-rows",
-                 {"score_folded", "select", "readout", "fuse_hidden"}, "query_proj"),
-                (fovea.PATH_AUTO, "fp32-ragged",
-                 {"query_proj", "score", "select_readout", "fuse_hidden"}, "select_fuse"),
-                (fovea.PATH_FUSED, "bf16-ragged", {"fused_step"}, "query_proj")):
-            fovea.step_path(path)
+                ("bf16-paper-defaults",
+                 {"ln_query", "score_fusion_h", "select_fuse", "fuse_out", "finalize"}, "fusion_h"),
+                ("bf16-one-group-offset", {"score_fusion_h", "select_fuse"}, "score_folded"),
+                ("bf16-long-rows", {"score_folded", "select", "readout", "fuse_hidden"},
+                 "query_proj"),
+                ("fp32-ragged", {"query_proj", "score", "select_readout", "fuse_hidden"},
+                 "select_fuse")):
             s = store(small_workload(name))
             fovea.timing_enable(True)
             run_gpu(s, fovea)
             names = set(fovea.timing_read())
             fovea.timing_enable(False)
-            assert want <= names and absent not in names, (path, names)
-        fovea.step_path(fovea.PATH_FUSED)
-        s = store(small_workload("fp32-ragged"))
-        with pytest.raises(fovea.FoveaError, match="UNSUPPORTED"):
-            run_gpu(s, fovea)
+            assert want <= names and absent not in names, (name, names)
     finally:
         fovea.timing_enable(False)
-        fovea.step_path(prev)
 
 
-def test_zero_gate_returns_rmsnorm_of_h(fovea, path):
+@pytest.mark.parametrize("name", ["bf16-ragged", "bf16-long-rows", "fp32-ragged"])
+def test_depth_gate(fovea, name):
+    """l_max = 1 (the experimental setup corrects nodes of depth <= 1): a
+    deeper row keeps h (bit for bit), count 0, indices -1, gate 0, readout 0;
+    the other rows match the oracle.  Runs the projected path, the path of
+    rows beyond 2048 entries, and fp32."""
+    w = small_workload(name)
+    s = store(w)
+    gpu = run_gpu(s, fovea, l_max=1)
+    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"), l_max=1)
+    assert orc["gated"].sum() > 0 and (~orc["gated"]).sum() > 0
+    compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"))
+    assert np.all(gpu["readout"][orc["gated"]] == 0.0)
+
+
+def test_zero_gate_returns_rmsnorm_of_h(fovea):
     w = small_workload("bf16-ragged")
     w.params["w_g2"] = np.zeros_like(w.params["w_g2"])
     w.params["b_g2"] = np.array([-1000.0], dtype=np.float32)
@@ -244,7 +257,7 @@ def test_zero_gate_returns_rmsnorm_of_h(fovea, path):
     assert rel_err_rows(gpu["h_out"].astype(np.float64), want).max() <= 2e-2
 
 
-def test_planted_rows_select_one_entry(fovea, path):
+def test_planted_rows_select_one_entry(fovea):
     spec = workloads.Spec(0, "planted-d512", d=512, B=1, rows_per_seq=24, rho=0.9, k_max=32,
                           k_min=1, dtype="bf16", seed=31, m_fixed=300, peaked_rows=6)
     w = workloads.generate(spec)
@@ -252,11 +265,11 @@ def test_planted_rows_select_one_entry(fovea, path):
     gpu = run_gpu(s, fovea)
     for row, entry in w.planted.items():
         assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
-    orc, mem = run_oracle(s, mirror=True, fold=gpu["_folded"])
+    orc, mem = run_oracle(s, mirror=True)
     compare(gpu, orc, s, mem=mem)
 
 
-def test_repeat_calls_are_deterministic(fovea, path):
+def test_repeat_calls_are_deterministic(fovea):
     w = small_workload("bf16-temperature")
     s = store(w)
     params = params_for(s, fovea)
@@ -274,7 +287,7 @@ def test_repeat_calls_are_deterministic(fovea, path):
     fovea.sync_errors(ws)
 
 
-def test_invalid_depth_sets_error_word(fovea, path):
+def test_invalid_depth_sets_error_word(fovea):
     w = small_workload("bf16-ragged")
     w.depth = w.depth.copy()
     w.depth[3] = 9
@@ -287,7 +300,38 @@ def test_invalid_depth_sets_error_word(fovea, path):
     fovea.sync_errors(o["workspace"])      # the word was cleared
 
 
-def test_bad_row_offsets_and_workspace(fovea, path):
+def test_bounded_wait_that_gives_up_reports_timeout(fovea):
+    """Every mbarrier wait of the tensor-core kernels is bounded.  With the
+    limit cut to 1 ns (fovea_debug_wait_limit) the waits give up while the
+    copies and MMAs they wait for are still in flight: each kernel records
+    FOVEA_ERR_TIMEOUT, waits for the work it issued with its fixed limits,
+    and exits.  The call's status reads TIMEOUT through fovea_sync_errors,
+    which clears the workspace header; after fovea_workspace_init the same
+    workspace serves a normal call that matches the oracle."""
+    w = small_workload("bf16-temperature")
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], s.dev.get("mask"))
+    ws = fovea.new_workspace(params, mem, w.row_offsets, w.k_max)
+    fovea.debug_wait_limit(1)
+    try:
+        fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets,
+                   s.dev.get("row_scale"), w.rho, w.k_min, w.k_max, workspace=ws)
+        with pytest.raises(fovea.FoveaError, match="TIMEOUT"):
+            fovea.sync_errors(ws)
+    finally:
+        fovea.debug_wait_limit(0)
+    fovea.lib().fovea_workspace_init(ws.data_ptr(), ws.numel(), None)
+    out = fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets,
+                     s.dev.get("row_scale"), w.rho, w.k_min, w.k_max, workspace=ws)
+    fovea.sync_errors(ws)
+    gpu = {k: (v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy())
+           for k, v in out.items() if v is not None and k != "workspace"}
+    orc, omem = run_oracle(s, mirror=True)
+    compare(gpu, orc, s, mem=omem, max_exempt=SMALL_MAX_EXEMPT["bf16-temperature"])
+
+
+def test_bad_row_offsets_and_workspace(fovea):
     w = small_workload("bf16-ragged")
     s = store(w)
     params = params_for(s, fovea)
@@ -314,35 +358,24 @@ def test_bad_row_offsets_and_workspace(fovea, path):
 # The five named workloads at full size
 # ---------------------------------------------------------------------------
 
-_NAMED = {}
-
-
-def _named(idx, fold):
-    """Inputs and oracle result of a named workload, computed once per score
-    form (folded keys or the query) for both paths."""
-    if idx not in _NAMED:
-        w = workloads.generate(workloads.WORKLOADS[idx])
-        _NAMED[idx] = (w, store(w), {})
-    w, s, orcs = _NAMED[idx]
-    if fold not in orcs:
-        orcs[fold] = run_oracle(s, mirror=(w.dtype == "bf16"), fold=fold)
-    orc, mem = orcs[fold]
-    return w, s, orc, mem
+# Boundary-row share allowed per named workload.  In the long-memory one every
+# row reaches the 256 cap, and its clustered keys put 11-13 % of those cuts
+# between scores within the tie band.
+NAMED_MAX_EXEMPT = {1: 0.05, 2: 0.05, 3: 0.05, 4: 0.05, 5: 0.15}
 
 
 @pytest.mark.parametrize("idx", [1, 2, 3, 4])
-def test_named_workload_parity(fovea, path, idx):
-    if path == "fused" and workloads.WORKLOADS[idx].dtype != "bf16":
-        pytest.skip("the persistent step kernel covers bf16 calls only")
-    w = workloads.generate(workloads.WORKLOADS[idx]) if idx not in _NAMED else _NAMED[idx][0]
-    if idx not in _NAMED:
-        _NAMED[idx] = (w, store(w), {})
-    s = _NAMED[idx][1]
+def test_named_workload_parity(fovea, idx):
+    w = workloads.generate(workloads.WORKLOADS[idx])
+    s = store(w)
     gpu = run_gpu(s, fovea)
-    w, s, orc, mem = _named(idx, gpu["_folded"])
-    mirror = w.dtype == "bf16"
-    rep = compare(gpu, orc, s, mem=mem, mirror=mirror)
-    print(f"workload {idx} ({path}): {rep}")
+    orc, mem = run_oracle(s, mirror=(w.dtype == "bf16"))
+    rep = compare(gpu, orc, s, mem=mem, mirror=(w.dtype == "bf16"),
+                  max_exempt=NAMED_MAX_EXEMPT[idx])
+    print(f"workload {idx} (folded keys: {gpu['_folded']}): {rep['rows']} rows, boundary rows "
+          f"{len(rep['exempt'])} ({rep['exempt_mass']} mass, {rep['exempt_tie']} tie; GPU selection "
+          f"differs from the oracle's on {rep['exempt_differ']}) {rep['exempt']}, readout err "
+          f"{rep['readout_err']:.2e}, h_out err {rep['h_out_err']:.2e}, gate err {rep['gate_err']:.2e}")
     if idx == 2:
         for row, entry in w.planted.items():
             assert gpu["counts"][row] == 1 and gpu["indices"][row, 0] == entry
@@ -351,24 +384,18 @@ def test_named_workload_parity(fovea, path, idx):
         assert gpu["counts"].min() == 1 and gpu["counts"].max() == w.k_max
 
 
-def test_long_memory_sampled_steps(fovea):
+def test_long_memory_steps(fovea):
     """Long-memory workload: one memory of 4 x 8192 clustered entries queried
-    over 100 draft steps.  The GPU runs every step; the oracle checks sampled
-    rows of two sequences at steps 0, 1, 49 and 99."""
+    over 100 draft steps.  The GPU runs every step; the oracle checks every
+    row of every sequence at steps 0, 1, 49 and 99."""
     spec = workloads.WORKLOADS[5]
     w0 = workloads.generate(spec, step=0)
     s0 = store(w0)
     params = params_for(s0, fovea)
     mem = fovea.build_memory(params, s0.dev["v"], s0.dev.get("mask"))
     ws = fovea.new_workspace(params, mem, w0.row_offsets, w0.k_max)
-    seqs = [0, 3]
     p64 = {n: s0.f64[n] for n in workloads.PARAM_NAMES}
-    omem = oracle.build_memory(p64, s0.f64["v"][seqs], None, mirror=True)
-    fold = step_is_folded(fovea, params, mem)
-    if fold:
-        omem = oracle.fold_keys(p64, omem, mirror=True)
-    R = spec.rows_per_seq
-    rng = np.random.default_rng(5)
+    omem = oracle.build_memory(p64, s0.f64["v"], None, mirror=True, ln_eps=LN_EPS)
     checked = {}
     for t in range(spec.steps):
         h = workloads.hidden_states(spec.seed, w0.N, spec.d, step=t)
@@ -380,17 +407,14 @@ def test_long_memory_sampled_steps(fovea):
         torch.cuda.synchronize()
         gpu = {k: (v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy())
                for k, v in out.items() if v is not None and k != "workspace"}
-        rows = sorted(int(b * R + j) for b in seqs for j in rng.choice(R, size=12, replace=False))
-        # oracle over the two sequences only: a 2-sequence batch of the sampled rows
-        sub_offsets = np.array([0, 12, 24])
-        hw = dataclasses.replace(w0, h=h[rows], depth=w0.depth[rows], row_offsets=sub_offsets,
-                                 v=w0.v[seqs], mask=None)
-        sub = store(hw, device=None)
-        orc = oracle.retrieve_fuse(p64, omem, sub.f64["h"], sub.f64["depth"], sub_offsets, None,
-                                   w0.rho, w0.k_min, w0.k_max, mirror=True, fold=fold)
-        g_sub = {k: v[rows] for k, v in gpu.items()}
-        rep = compare(g_sub, orc, sub, mem=omem, mirror=True)
-        checked[t] = rep
+        ws_t = store(dataclasses.replace(w0, h=h), device=None)
+        orc = oracle.retrieve_fuse(p64, omem, ws_t.f64["h"], ws_t.f64["depth"], w0.row_offsets,
+                                   None, w0.rho, w0.k_min, w0.k_max, mirror=True,
+                                   ln_eps=LN_EPS, rms_eps=RMS_EPS)
+        rep = compare(gpu, orc, ws_t, mem=omem, mirror=True, max_exempt=NAMED_MAX_EXEMPT[5])
+        checked[t] = (len(rep["exempt"]), rep["exempt_mass"], rep["exempt_tie"],
+                      len(rep["exempt_differ"]), rep["readout_err"], rep["h_out_err"])
     fovea.sync_errors(ws)
     assert sorted(checked) == [0, 1, 49, 99]
-    print(checked)
+    print("long memory, step: (boundary rows, mass, tie, boundary rows whose GPU selection "
+          f"differs, readout err, h_out err) of {w0.N} rows: {checked}")

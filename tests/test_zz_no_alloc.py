@@ -5,9 +5,11 @@ step recorded into a CUDA graph, a runtime with a fixed memory plan, a loop
 that must not pay cudaMalloc's implicit synchronisation).  For them the
 library keeps its scratch in a static device array.  This test calls that
 entry point through the C ABI, twice in a row on the same array, and checks
-each call against fovea_retrieve_fuse with a caller workspace: counts and
-indices equal, readout, gate and corrected hidden state within the bf16
-tolerance the parity tests use.  It also checks that a call too large for the
+each call against fovea_retrieve_fuse with a caller workspace (counts and
+indices equal; readout, gate and corrected hidden state within the bf16
+tolerance the parity tests use) and against the CPU oracle under the parity
+rules.  It checks that the array's error word keeps a device-side condition
+until fovea_noalloc_sync_errors reads it, and that a call too large for the
 array is refused.  It runs last so a failure here cannot hide other results.
 """
 
@@ -16,12 +18,12 @@ import pytest
 import torch
 
 import workloads
-from parity import TOL, params_for, rel_err_rows, store
+from parity import TOL, compare, params_for, rel_err_rows, run_oracle, store
 
 pytestmark = pytest.mark.gpu
 
 
-def test_noalloc_entry_point_matches_workspace_entry_point():
+def test_noalloc_entry_point_matches_workspace_entry_point_and_oracle():
     from paper_2608_22883_gb300 import fovea
     w = workloads.generate_custom("noalloc", 512, [300, 77], [40, 9], rho=0.85, k_max=32,
                                   seed=19, temperature=(0.5, 2.0))
@@ -31,6 +33,8 @@ def test_noalloc_entry_point_matches_workspace_entry_point():
     ref = fovea.step(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets,
                      s.dev.get("row_scale"), w.rho, w.k_min, w.k_max)
     fovea.sync_errors(ref["workspace"])
+    orc, omem = run_oracle(s, mirror=True)
+    fovea.noalloc_sync_errors()            # whatever an earlier caller left
     for _ in range(2):
         out = dict(h_out=torch.empty_like(s.dev["h"]),
                    counts=torch.full((w.N,), -7, dtype=torch.int32, device="cuda"),
@@ -41,7 +45,7 @@ def test_noalloc_entry_point_matches_workspace_entry_point():
                                     s.dev.get("row_scale"), w.rho, w.k_min, w.k_max, out["h_out"],
                                     counts=out["counts"], indices=out["indices"],
                                     readout=out["readout"], gate=out["gate"])
-        torch.cuda.synchronize()
+        fovea.noalloc_sync_errors()
         assert torch.equal(out["counts"], ref["counts"])
         assert torch.equal(out["indices"], ref["indices"])
         tol = TOL[w.dtype]
@@ -49,6 +53,30 @@ def test_noalloc_entry_point_matches_workspace_entry_point():
             err = rel_err_rows(out[key].double().cpu().numpy(), ref[key].double().cpu().numpy())
             assert err.max() <= tol, (key, err.max())
         assert (out["gate"] - ref["gate"]).abs().max().item() <= tol
+        gpu = {k: (v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy())
+               for k, v in out.items()}
+        compare(gpu, orc, s, mem=omem, mirror=True)
+    mem.destroy()
+
+
+def test_noalloc_error_word_is_kept_until_read():
+    from paper_2608_22883_gb300 import fovea
+    w = workloads.generate_custom("noalloc-depth", 256, [64], [6], k_max=8, seed=23)
+    w.depth = w.depth.copy()
+    w.depth[2] = 99                      # outside [0, D]: flagged on the device
+    s = store(w)
+    params = params_for(s, fovea)
+    mem = fovea.build_memory(params, s.dev["v"], None)
+    h_out = torch.empty_like(s.dev["h"])
+    fovea.noalloc_sync_errors()
+    fovea.retrieve_fuse_noalloc(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets, None,
+                                w.rho, w.k_min, w.k_max, h_out)
+    s.dev["depth"][2] = 0
+    fovea.retrieve_fuse_noalloc(params, mem, s.dev["h"], s.dev["depth"], w.row_offsets, None,
+                                w.rho, w.k_min, w.k_max, h_out)   # a clean call after it
+    with pytest.raises(fovea.FoveaError, match="INVALID_ARG"):
+        fovea.noalloc_sync_errors()
+    fovea.noalloc_sync_errors()          # read and cleared
     mem.destroy()
 
 
