@@ -169,21 +169,25 @@ __global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
   }
   pdl_wait();
   pdl_trigger();
+  // the row and the depth are requested together; the depth embedding row
+  // (from the staged table) is read once the depth is known
+  const T* xr = x + (long long)row * d;
+#pragma unroll
+  for (int j = 0; j < kLnMaxVec; ++j) {
+    const int vi = tid + j * kLnThreads;
+    if (vi < nvec) ln_load<T>(xr + vi * V, xv[j]);
+  }
   int dep = depth[row];
   if (dep < 0 || dep > max_depth) {
     if (tid == 0) atomicOr(err, kErrDepth);
     dep = 0;
   }
-  const T* xr = x + (long long)row * d;
   const T* er = (e_smem ? e_s : E) + (long long)dep * d;
   if (e_smem) cp_async_wait_all();          // this thread's own copies
 #pragma unroll
   for (int j = 0; j < kLnMaxVec; ++j) {
     const int vi = tid + j * kLnThreads;
-    if (vi < nvec) {
-      ln_load<T>(xr + vi * V, xv[j]);
-      ln_load<T>(er + vi * V, ev[j]);
-    }
+    if (vi < nvec) ln_load<T>(er + vi * V, ev[j]);
   }
   // pass 1: mean
   float s = 0.0f;

@@ -74,6 +74,8 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
 // their partial sums are combined in group order (fixed order, fp32).  CTA
 // rank 0 writes counts and indices.
 constexpr int kRoUnroll = 8;
+constexpr int kStageRows = 64;                 // staged gather: rows per round
+constexpr int kGatherSmemMax = 200 * 1024;     // dynamic shared memory of the gather kernel
 static inline size_t align_up_sz(size_t x, size_t a) { return (x + a - 1) / a * a; }
 using tc::cluster_sync;
 using tc::ld_dsmem_f4;
@@ -112,6 +114,11 @@ struct GatherArgs {
   void* act;                        // [N, HP]
   long long p_prefetch;             // bytes of P prefetched into L2 before the wait
   int red_floats;                   // dynamic shared memory: the row's scores
+  // > 0: the selected rows of P are staged in shared memory by bulk copies,
+  // this many per round, at dyn + stage_off, with the group sums at dyn + red_off
+  int stage_rows, stage_off, red_off;
+  int self_select;                  // the CTAs of a row each select (no cluster)
+  int* err;
 };
 
 // Weighted gather-sum over the selected rows of X [*, ld], columns
@@ -176,6 +183,62 @@ __device__ __forceinline__ void gather_chunk(const T* X, long long ld, int c0, i
   }
 }
 
+// Weighted sum over the selected rows of X [*, ld], columns [c0, c0 + w),
+// staged in shared memory: each selected row's w elements arrive by one bulk
+// copy (cp.async.bulk into buf, completing on the mbarrier `bar`), up to
+// buf_rows rows per round.  Thread tid owns column vector tid % nvec of entry
+// group tid / nvec (a warp reads 512 contiguous bytes of one staged row, free
+// of bank conflicts); the groups' sums meet in `red` [G][w] fp32 and are
+// added in group order (deterministic).  out(column, sum) once per column.
+// A wait that gives up sets kErrTimeout; the copies already issued are waited
+// for before the function returns.
+template <class T, int NT, class Out>
+__device__ __forceinline__ void gather_rows_smem(const T* X, long long ld, int c0, int w, int K,
+                                                 const int32_t* pos, const float* wt, int tid,
+                                                 T* buf, int buf_rows, float* red, uint64_t* bar,
+                                                 int* err, Out out) {
+  constexpr int V = 16 / (int)sizeof(T);
+  const int nvec = w / V;
+  const int G = NT / nvec;                       // entry groups (NT % nvec == 0)
+  const int vec = tid % nvec, grp = tid / nvec;
+  const uint32_t row_bytes = (uint32_t)(w * sizeof(T));
+  float acc[V];
+#pragma unroll
+  for (int i = 0; i < V; ++i) acc[i] = 0.0f;
+  uint32_t parity = 0;
+  for (int t0 = 0; t0 < K; t0 += buf_rows) {
+    const int cnt = min(buf_rows, K - t0);
+    if (tid == 0) tc::mbar_expect_tx(bar, (uint32_t)cnt * row_bytes);
+    __syncthreads();                             // bytes posted; buf free for this round
+    if (tid < cnt)
+      tc::bulk_load(buf + (size_t)tid * w, X + (long long)pos[t0 + tid] * ld + c0, row_bytes, bar);
+    bool landed = tc::mbar_wait(bar, parity, nullptr);
+    if (!landed) {
+      if (tid == 0) atomicOr(err, kErrTimeout);
+      tc::mbar_wait(bar, parity, nullptr);      // the copies in flight land first
+    }
+    parity ^= 1u;
+    if (!__syncthreads_and(landed)) break;
+    for (int t = grp; t < cnt; t += G) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(buf + (size_t)t * w + vec * V);
+      const float wj = wt[t0 + t];
+      const T* e = reinterpret_cast<const T*>(&raw);
+#pragma unroll
+      for (int i = 0; i < V; ++i) acc[i] = fmaf(wj, to_f32(e[i]), acc[i]);
+    }
+  }
+  float* mine = red + (size_t)grp * w + vec * V;
+#pragma unroll
+  for (int i = 0; i < V; i += 4)
+    *reinterpret_cast<float4*>(mine + i) = make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+  __syncthreads();
+  for (int c = tid; c < w; c += NT) {
+    float sum = 0.0f;
+    for (int g = 0; g < G; ++g) sum += red[(size_t)g * w + c];
+    out(c, sum);
+  }
+}
+
 // The selection group: the first kSelThreads threads of the CTA, synchronised
 // with a named barrier when the CTA is larger.
 struct SelGroupSync {
@@ -198,9 +261,14 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
   __shared__ __align__(16) int32_t loc_pos[kRankMax];
   __shared__ __align__(16) float loc_w[kRankMax];
   __shared__ int loc_cnt;
+  __shared__ __align__(8) uint64_t stage_bar;      // staged gather rounds
   const int n = blockIdx.x;
   const int tid = threadIdx.x;
   const uint32_t rank = cluster_rank();
+  if (tid == 0 && ga.stage_rows > 0) {
+    tc::mbar_init(&stage_bar, 1);
+    tc::fence_mbar_init();
+  }
   float* s_sc = dyn;
   float* gh_s = dyn + ga.red_floats;
   T* bias_s = reinterpret_cast<T*>(gh_s + ga.chunk_p);
@@ -223,7 +291,13 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
   // original positions of the sequence's entries: requested now, used last
   int32_t* orig_s = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(bias_s) +
                                                ((ga.chunk_p * (int)sizeof(T) + 15) & ~15));
-  if (rank == 0 && args.indices != nullptr) {
+  // self_select: every CTA of the row selects for itself (the selection is
+  // deterministic, so all reach the same result) and CTA y = 0 writes the
+  // row's counts and indices; otherwise CTA rank 0 of the row's cluster
+  // selects and the others copy its result through distributed shared memory
+  const bool selector = ga.self_select || rank == 0;
+  const bool writer = ga.self_select ? blockIdx.y == 0 : rank == 0;
+  if (writer && args.indices != nullptr) {
     const int b = seq_of_row(tab, n);
     const int M = tab.m[b];
     const int32_t* src = args.orig_index + tab.key_off[b];
@@ -244,7 +318,7 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
                             : static_cast<const T*>(ga.b_g1) + (c - ga.H);
     cp_async16(bias_s + q * V, src);
   }
-  if (rank == 0 && tid < kSelThreads) {
+  if (selector && tid < kSelThreads) {
     SelectArgs a = args;
     a.counts = nullptr;                   // written after the cluster barrier (below), so
     a.indices = nullptr;                  // the barrier's release has no global writes to wait for
@@ -289,9 +363,9 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
   }
   // rank 0's selection visible to the cluster (one CTA: a CTA barrier, which
   // does not wait for the selection's global writes to complete)
-  const bool clustered = gridDim.y > 1;
+  const bool clustered = !ga.self_select && gridDim.y > 1;
   if (clustered) cluster_sync(); else __syncthreads();
-  if (rank != 0) {
+  if (!selector) {
     const int K = ld_dsmem_s32(map_dsmem(smem_u32(&loc_cnt), 0));
     for (int q = tid; q < (K + 3) / 4; q += NT) {
       const float4 p4 = ld_dsmem_f4(map_dsmem(smem_u32(&loc_pos[4 * q]), 0));
@@ -305,7 +379,7 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
   cp_async_wait_all();
   __syncthreads();
   const int K = loc_cnt;
-  if (rank == 0) {                        // counts and indices of row n
+  if (writer) {                           // counts and indices of row n
     const long long out_row = (long long)n * args.k_max;
     if (args.indices != nullptr) {
       const int key_off = tab.key_off[seq_of_row(tab, n)];
@@ -322,7 +396,15 @@ __global__ void __launch_bounds__(NT) select_gather_kernel(
       const float z = sum + gh_s[c] + to_f32(bias_s[c]);
       act[c] = from_f32<T>(z * sigmoidf_(z));
     };
-    gather_chunk<T, NT>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid, fin);
+    if (ga.stage_rows > 0) {
+      T* buf = reinterpret_cast<T*>(reinterpret_cast<uint8_t*>(dyn) + ga.stage_off);
+      float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(dyn) + ga.red_off);
+      auto fin_c = [&](int c, float sum) { fin(c / V, c % V, sum); };
+      gather_rows_smem<T, NT>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid,
+                              buf, ga.stage_rows, red, &stage_bar, ga.err, fin_c);
+    } else {
+      gather_chunk<T, NT>(static_cast<const T*>(ga.P), ga.HP, cp0, wp, K, loc_pos, loc_w, tid, fin);
+    }
   }
   // readout r_n
   const int cu0 = blockIdx.y * ga.chunk_u;
@@ -356,16 +438,21 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
   if (e != cudaSuccess) return e;
   const int HP = 2 * H;
-  // projected readout: one CTA of 1024 threads per row (the selection on
-  // 256 of them; a cluster barrier costs about a microsecond, more than the
-  // gathers gain from spreading over more SMs); the readout alone: a cluster
-  // of CTAs of 256 threads per row, about two CTAs per SM in one wave, each
-  // chunk a multiple of 64 columns
+  // projected readout: CTAs of 1024 threads (the selection on 256 of them),
+  // one per row, or two per row that each select for themselves when the
+  // batch leaves most SMs idle; the readout alone: a cluster of CTAs of 256
+  // threads per row, about two CTAs per SM in one wave, each chunk a multiple
+  // of 64 columns
   const bool wide = P != nullptr;
   int nchunk = 1;
   while (!wide && nchunk < 8 && (long long)N * nchunk * 2 <= 2LL * sms &&
          d % (nchunk * 2 * 64) == 0)
     nchunk *= 2;
+  // projected readout: a batch that leaves most SMs idle gives each row two
+  // CTAs, each selecting for itself and gathering half of the 2H columns (the
+  // gather of a row's selected projected rows is bound by what one SM takes
+  // in from L2)
+  if (wide && (long long)N * 2 <= sms && HP % 128 == 0) nchunk = 2;
   GatherArgs ga{};
   ga.U = U;
   ga.d = d;
@@ -383,16 +470,31 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   ga.p_prefetch = P != nullptr ? p_prefetch_bytes : 0;
   ga.red_floats = (int)align_up_sz((size_t)std::max(max_m, 1), 4);
   const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
-  const size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
-                      align_up_sz((size_t)ga.chunk_p * es, 16) + (size_t)ga.red_floats * 4;
+  // dynamic: scores | G_h | biases | original positions
+  size_t smem = (size_t)ga.red_floats * 4 + (size_t)ga.chunk_p * 4 +
+                align_up_sz((size_t)ga.chunk_p * es, 16) + (size_t)ga.red_floats * 4;
   if (smem > 64 * 1024) return cudaErrorInvalidValue;
+  ga.err = err;
+  if (wide && dtype == FOVEA_BF16 && ga.chunk_p % 8 == 0 && 1024 % (ga.chunk_p / 8) == 0) {
+    // stage the selected projected rows in shared memory: up to 64 rows per
+    // round (128 KB at 2H = 1024), the group sums after them
+    const int rows = std::min(k_max, kStageRows);
+    ga.stage_off = (int)align_up_sz(smem, 128);
+    const size_t stage_bytes = (size_t)rows * ga.chunk_p * es;
+    ga.red_off = (int)align_up_sz(ga.stage_off + stage_bytes, 128);
+    const size_t red_bytes = (size_t)(1024 / (ga.chunk_p / 8)) * ga.chunk_p * 4;
+    if (ga.red_off + red_bytes <= (size_t)kGatherSmemMax) {
+      ga.stage_rows = rows;
+      smem = ga.red_off + red_bytes;
+    }
+  }
   static bool configured = false;
   if (!configured) {
     for (auto k : {(const void*)select_gather_kernel<__nv_bfloat16, 1024>,
                    (const void*)select_gather_kernel<__nv_bfloat16, kSelThreads>,
                    (const void*)select_gather_kernel<float, 1024>,
                    (const void*)select_gather_kernel<float, kSelThreads>}) {
-      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kGatherSmemMax);
       if (e != cudaSuccess) return e;
     }
     configured = true;
@@ -412,7 +514,8 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
   attr[1].val.clusterDim.y = nchunk;
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = wide ? 1 : 2;              // projected rows: self-selecting CTAs, no cluster
+  ga.self_select = wide ? 1 : 0;
   if (dtype == FOVEA_BF16)
     return wide ? cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16, 1024>, a, tab, ga)
                 : cudaLaunchKernelEx(&cfg, select_gather_kernel<__nv_bfloat16, kSelThreads>, a, tab, ga);

@@ -58,6 +58,9 @@ SMALL = {
     # rows beyond 2048 entries: selection and readout run as two kernels
     "bf16-long-rows": dict(d=256, m_sizes=[2500, 300], rows=[12, 5], k_max=64),
     "bf16-hidden-128": dict(d=256, m_sizes=[100], rows=[9], k_max=16, H=128),
+    # fewer entries than d: the memory holds folded keys; clustered near-ties
+    "bf16-clustered-folded": dict(d=1024, m_sizes=[768], rows=[96], clusters=16,
+                                  cluster_sigma=0.2, k_max=128),
     "fp32-ragged": dict(d=256, m_sizes=[64, 130], rows=[4, 11], dtype="fp32", k_max=16),
     "fp32-temperature": dict(d=192, m_sizes=[300, 20], rows=[17, 3], dtype="fp32", k_max=64,
                              temperature=(0.1, 10.0), rho=0.8),
@@ -150,7 +153,7 @@ def test_plain_fusion_when_weights_differ(fovea):
     fovea.timing_enable(False)
     assert "select_fuse" in names_proj and "fuse_hidden" not in names_proj
     assert "fuse_hidden" in names_plain and "select_fuse" not in names_plain
-    assert proj["_folded"] and plain["_folded"]          # same W_Q: both fold
+    assert proj["_folded"] == plain["_folded"]           # same W_Q: the same score form
     for gpu in (proj, plain):
         compare(gpu, orc, s, mem=mem, mirror=True)
     np.testing.assert_array_equal(proj["counts"], plain["counts"])
@@ -158,7 +161,8 @@ def test_plain_fusion_when_weights_differ(fovea):
     assert rel_err_rows(proj["h_out"].astype(np.float64), plain["h_out"].astype(np.float64)).max() <= 2e-2
 
 
-@pytest.mark.parametrize("name", ["bf16-temperature", "bf16-clustered", "bf16-paper-defaults"])
+@pytest.mark.parametrize("name", ["bf16-clustered-folded", "bf16-scattered-mask-d320",
+                                  "bf16-one-group-offset"])
 def test_folded_and_unfolded_steps_select_the_same_entries(fovea, name):
     """A memory built without W_Q holds no folded keys: the step then forms
     q = W_Q x_h (hi / lo pair) and scores it against the keys, the paper's
@@ -210,11 +214,10 @@ def test_paths_are_taken(fovea):
     as a GEMM; fp32 takes the unfolded SIMT path."""
     try:
         for name, want, absent in (
+                # several score groups: G_h in a launch of its own
                 ("bf16-ragged",
                  {"ln_query", "fusion_h", "score_folded", "select_fuse", "fuse_out", "finalize"},
-                 "fuse_hidden"),
-                ("bf16-paper-defaults",
-                 {"ln_query", "score_fusion_h", "select_fuse", "fuse_out", "finalize"}, "fusion_h"),
+                 "query_proj"),
                 ("bf16-one-group-offset", {"score_fusion_h", "select_fuse"}, "score_folded"),
                 ("bf16-long-rows", {"score_folded", "select", "readout", "fuse_hidden"},
                  "query_proj"),
