@@ -125,6 +125,11 @@ struct fovea_memory {
   // were built with (a call with other W_f1 / W_g1 pointers or H does not
   // use them)
   void* proj = nullptr;
+  // the projected values transposed per image, [B, 2H, proj_ld] with
+  // proj_ld = max valid count rounded up to 64 (zero-padded): the feature
+  // operand of the weighted-sum GEMM over dense selection weights
+  void* projT = nullptr;
+  int proj_ld = 0;
   const void* proj_wf1 = nullptr;
   const void* proj_wg1 = nullptr;
   int proj_h = 0;
@@ -207,6 +212,7 @@ static void free_memory(fovea_memory* m) {
   cudaFree(m->keys);
   cudaFree(m->values);
   cudaFree(m->proj);
+  cudaFree(m->projT);
   cudaFree(m->folded);
   cudaFree(m->orig_index);
   cudaFree(m->err);
@@ -441,6 +447,22 @@ FOVEA_API fovea_status fovea_build_memory(const fovea_params* p, const void* v,
                                TmaOperand{nullptr, 0, 0, 0}, 2 * H, total, s); }
         if (err == cudaSuccess) err = cudaStreamSynchronize(s);
         if (err != cudaSuccess) return cuda_fail(err, "fusion projection of the values");
+        int m_max = 0;
+        for (int b = 0; b < B; ++b) m_max = std::max(m_max, m->counts[b]);
+        const int ld = (m_max + 63) / 64 * 64;
+        if ((ps = alloc_dev(&m->projT, (size_t)B * 2 * H * ld * 2, "transposed projected values")) != FOVEA_OK)
+          return ps;
+        static thread_local ImageTable itab;
+        itab.B = B;
+        for (int b = 0; b < B; ++b) {
+          itab.off[b] = (int)m->offsets[b];
+          itab.m[b] = m->counts[b];
+        }
+        { KernelTimer t("memory_proj_transpose", s);
+          err = launch_transpose_images(m->proj, 2 * H, ld, itab, m->projT, s); }
+        if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+        if (err != cudaSuccess) return cuda_fail(err, "transposing the projected values");
+        m->proj_ld = ld;
         m->proj_wf1 = p->W_f1;
         m->proj_wg1 = p->W_g1;
         m->proj_h = H;
@@ -500,10 +522,23 @@ FOVEA_API fovea_status fovea_memory_tensors(const fovea_memory* mem, const void*
 // ---------------------------------------------------------------------------
 namespace {
 struct WsLayout {
-  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, total;
+  size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, alpha_hi, alpha_lo, total;
 };
 
-WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems) {
+int device_sms() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+  }
+  return sms;
+}
+
+// alpha_ld: entries of a dense weight row (the memory's padded per-image
+// count when it keeps the transposed projected values, else 0).
+WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_elems, int alpha_ld) {
   WsLayout L;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -523,6 +558,8 @@ WsLayout ws_layout(int dtype, int d, int H, int N, int k_max, long long score_el
   L.act = take((size_t)N * 2 * H * es);
   L.c = take((size_t)N * d * 4);
   L.gh = take(dtype == FOVEA_BF16 ? (size_t)N * 2 * H * 4 : 0);   // [W_f1 ; W_g1]_h h, fp32
+  L.alpha_hi = take((size_t)N * alpha_ld * 2);                     // dense weights, bf16 hi
+  L.alpha_lo = take((size_t)N * alpha_ld * 2);                     // and lo
   L.total = off;
   return L;
 }
@@ -569,7 +606,8 @@ FOVEA_API fovea_status fovea_workspace_size(const fovea_params* p, const fovea_m
   int N, mm, mr, ng;
   long long se;
   if ((st = check_rows(mem, row_offsets, &N, &se, &mm, &mr, &ng)) != FOVEA_OK) return st;
-  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se).total;
+  *bytes = ws_layout(p->dtype, p->d_model, p->mlp_hidden, N, k_max, se,
+                     mem->projT != nullptr ? mem->proj_ld : 0).total;
   return FOVEA_OK;
 }
 
@@ -642,7 +680,8 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   const int d = p->d_model, H = p->mlp_hidden, dt = p->dtype;
-  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems);
+  const WsLayout L = ws_layout(dt, d, H, N, k_max, score_elems,
+                              mem->projT != nullptr ? mem->proj_ld : 0);
   if (workspace_bytes < L.total)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", workspace_bytes, L.total);
 
@@ -697,9 +736,16 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   // the scores take x_h against the folded keys, and the launch computes
   // G_h alone (or is skipped without the projected values).
   const bool bf = dt == FOVEA_BF16;
-  const bool use_proj = bf && mem->proj != nullptr && mem->proj_wf1 == p->W_f1 &&
-                        mem->proj_wg1 == p->W_g1 && mem->proj_h == H &&
-                        select_readout_fits(max_m, k_max);
+  // The r-half of the first fusion layer from the projected values: either
+  // gathered row by row in the selection kernel (rows of <= 2048 entries,
+  // k_max <= 256, a batch that fills the GPU in about a wave), or, with the
+  // selection weights written as dense rows, one GEMM against the memory's
+  // transposed projected values (long rows, large caps, large batches).
+  const bool have_proj = bf && mem->proj != nullptr && mem->proj_wf1 == p->W_f1 &&
+                         mem->proj_wg1 == p->W_g1 && mem->proj_h == H;
+  const bool alpha_path = have_proj && mem->projT != nullptr &&
+                          (!select_readout_fits(max_m, k_max) || N > 2 * device_sms());
+  const bool use_proj = have_proj && (alpha_path || select_readout_fits(max_m, k_max));
   const bool use_fold = bf && mem->folded != nullptr && mem->fold_wq == p->W_Q;
   // the folded keys are [total, 2d] (hi | lo per entry)
   const long long score_key_bytes = (long long)mem->total * d * 2 * (use_fold ? 2 : 1);
@@ -849,7 +895,47 @@ FOVEA_API fovea_status fovea_retrieve_fuse(const fovea_params* p, const fovea_me
   // (4) softmax, cumulative-mass cardinality, selected set, renormalised weights;
   // (5) r = sum alpha u; with the projected values, also
   // (6) [a_f | a_g] = SiLU(G_h + sum alpha p + [b_f1 | b_g1])
-  if (use_proj) {
+  if (alpha_path) {
+    // the selection writes the weights as dense bf16 hi / lo rows; the
+    // readout, when asked for, gathers the values row by row
+    void* alpha_hi = ws + L.alpha_hi;
+    void* alpha_lo = ws + L.alpha_lo;
+    { KernelTimer t("select", s);
+      e = launch_select(scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m, gate_rows,
+                        counts, indices, readout ? sel_pos : nullptr, readout ? sel_w : nullptr,
+                        readout ? sel_cnt : nullptr, s, alpha_hi, alpha_lo, mem->proj_ld); }
+    if (e != cudaSuccess) return cuda_fail(e, "select");
+    if (readout != nullptr) {
+      { KernelTimer t("readout", s);
+        e = launch_readout(dt, mem->values, sel_cnt, sel_pos, sel_w, N, k_max, d, readout, r_lo, s); }
+      if (e != cudaSuccess) return cuda_fail(e, "readout");
+    }
+    // [a_f | a_g] = SiLU(G_h + alpha P + [b_f1 | b_g1]): per image, the
+    // weights' hi / lo rows against the image's transposed projected values
+    init_args(a);
+    a.k_total = mem->proj_ld; a.b_split = mem->proj_ld;
+    a.A0 = mem->projT; a.lda0 = mem->proj_ld;
+    a.B0 = alpha_hi; a.B1 = alpha_lo; a.ldb0 = mem->proj_ld; a.ldb1 = mem->proj_ld;
+    a.epi_split = H;
+    a.out0 = act; a.ldc = 2 * H;
+    a.bias0 = p->b_f1; a.bias1 = p->b_g1;
+    a.add_in = gh; a.ldc2 = 2 * H;
+    a.err = err;
+    int g = 0, max_rows = 0;
+    for (int b = 0; b < mem->B; ++b) {
+      const int r = row_offsets[b + 1] - row_offsets[b];
+      if (r == 0) continue;
+      a.groups[g++] = GemmGroup{b * 2 * H, 2 * H, row_offsets[b], r, 0};
+      max_rows = std::max(max_rows, r);
+    }
+    a.ngroups = g;
+    { KernelTimer t("act_gemm", s);
+      e = launch_gemm_tc(kEpiAct, a, TmaOperand{mem->projT, (long long)mem->B * 2 * H, mem->proj_ld,
+                                                mem->proj_ld},
+                         TmaOperand{nullptr, 0, 0, 0}, TmaOperand{alpha_hi, N, mem->proj_ld, mem->proj_ld},
+                         TmaOperand{alpha_lo, N, mem->proj_ld, mem->proj_ld}, 2 * H, max_rows, s); }
+    if (e != cudaSuccess) return cuda_fail(e, "act_gemm");
+  } else if (use_proj) {
     { KernelTimer t("select_fuse", s);
       e = launch_select_gather(dt, scores, tab, N, mem->orig_index, rho, k_min, k_max, max_m,
                                gate_rows, counts, indices, mem->values, d, readout, nullptr,

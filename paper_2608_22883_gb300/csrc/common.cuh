@@ -52,7 +52,13 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
   return __float2bfloat16_rn(x);
 }
 
-__device__ __forceinline__ float sigmoidf_(float z) { return 1.0f / (1.0f + expf(-z)); }
+// Logistic sigmoid with the hardware exponential and a correctly rounded
+// reciprocal (a few fp32 ulps from the exact value, far below the bf16
+// rounding of the activations and the gate's tolerance; exp(-z) = inf for
+// z < -88 gives exactly 0, as the zero-gate reading needs).  The activation
+// epilogues evaluate it per element, where the full-precision expf and
+// division dominated their time.
+__device__ __forceinline__ float sigmoidf_(float z) { return __frcp_rn(1.0f + __expf(-z)); }
 
 // Programmatic dependent launch: kernels of the step are launched so that a
 // kernel may start while its predecessor finishes.  pdl_wait() blocks until
@@ -137,6 +143,10 @@ enum EpiKind : int {
                          // keys, a hi / lo pair of feature tiles (f_lo_kb), for columns
                          // < epi_split (row stride min(m, epi_split)); columns >=
                          // epi_split: out2 (fp32)[row * ldc2 + col - epi_split] = acc
+  kEpiAct = 8,           // the first fusion layer from dense selection weights: the row
+                         // operand is the weights' hi / lo pair (B0, B1, both multiplied by
+                         // the same feature tile); out0[row * ldc + col] =
+                         // T(silu(acc + add_in[row * ldc2 + col] + bias{0,1}[col]))
 };
 
 struct KeyFix {       // one listed key element: memory row, feature
@@ -170,6 +180,7 @@ struct GemmArgs {
   int kps;            // tensor-core path: k-blocks of 64 per ring stage
   int rbox;           // tensor-core path: rows of a row-operand tile (64 or 128)
   int region;         // tensor-core path: bytes of the ring / partial-tile staging region
+  const float* add_in;          // kEpiAct: fp32 term added before the activation
   unsigned long long wait_ns;   // tensor-core path: limit of a bounded mbarrier wait
   int* err;
   // tensor-core path: byte ranges whose share each CTA prefetches into L2 once
@@ -235,10 +246,15 @@ cudaError_t launch_count_valid(const uint8_t* mask, int B, int M_max, int32_t* c
                                cudaStream_t s);
 cudaError_t launch_compact(const uint8_t* mask, int B, int M_max, const int32_t* key_off,
                            int32_t* orig_index, int32_t* src_row, cudaStream_t s);
+// Selection alone (select.cu): counts, indices, and per row the selected
+// compacted memory rows and weights (sel_pos, sel_w, sel_cnt; any may be
+// null), and / or the weights as dense bf16 hi / lo rows over the row's
+// sequence [N, alpha_ld], zero where not selected (alpha_hi null: none).
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
                           float rho, int k_min, int k_max, int max_m, const DepthGate& gate,
                           int32_t* counts, int32_t* indices, int32_t* sel_pos, float* sel_w,
-                          int32_t* sel_cnt, cudaStream_t s);
+                          int32_t* sel_cnt, cudaStream_t s, void* alpha_hi = nullptr,
+                          void* alpha_lo = nullptr, int alpha_ld = 0);
 cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, const int32_t* sel_pos,
                            const float* sel_w, int N, int k_max, int d, float* r_out, void* r_lo,
                            cudaStream_t s);
@@ -262,6 +278,17 @@ cudaError_t launch_select_gather(int dtype, const float* scores, const SeqTable&
 // out[c * rows + r] = in[r * cols + c] for a bf16 [rows, cols] matrix, rows
 // and cols multiples of 32 (the query folding's W_Q^T, once per memory build).
 cudaError_t launch_transpose_bf16(const void* in, int rows, int cols, void* out, cudaStream_t s);
+
+// Images of a memory: first entry and valid count of each (kernel parameter).
+struct ImageTable {
+  int B;
+  int off[FOVEA_MAX_SEQ];
+  int m[FOVEA_MAX_SEQ];
+};
+// out [B, C, ld]: image b's [m_b, C] rows of `in` (from row off_b) transposed,
+// zero-padded to ld entries (C and ld multiples of 32).
+cudaError_t launch_transpose_images(const void* in, int C, int ld, const ImageTable& tab,
+                                    void* out, cudaStream_t s);
 
 // Per row of logits [N, V] fp32: the k <= FOVEA_MAX_KC largest in
 // descending order (ties: smaller index first), indices and values.

@@ -22,11 +22,12 @@ __device__ __forceinline__ void gemm_epilogue(const GemmArgs& a, const GemmGroup
     const int stride = EPI == kEpiScoresFolded ? min(g.m, a.epi_split) : g.m;
     const float rs = a.row_scale ? a.row_scale[g.b_row0 + n] : 1.0f;
     static_cast<float*>(a.out0)[g.c_off + (long long)n * stride + m] = acc * a.scale * rs;
-  } else if constexpr (EPI == kEpiBiasSilu) {
+  } else if constexpr (EPI == kEpiBiasSilu || EPI == kEpiAct) {
     const long long row = (long long)g.b_row0 + n;
     const float bias = m < a.epi_split ? to_f32(static_cast<const T*>(a.bias0)[m])
                                        : to_f32(static_cast<const T*>(a.bias1)[m - a.epi_split]);
-    const float z = acc + bias;
+    float z = acc + bias;
+    if constexpr (EPI == kEpiAct) z += a.add_in[row * a.ldc2 + m];
     static_cast<T*>(a.out0)[row * a.ldc + m] = from_f32<T>(z * sigmoidf_(z));
   } else if constexpr (EPI == kEpiStoreHiLo || EPI == kEpiQueryH) {
     const long long row = (long long)g.b_row0 + n;
@@ -53,7 +54,7 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
   typedef __nv_bfloat16 T;
   const long long row = (long long)g.b_row0 + n;
   bool vec = nv == 4;
-  if constexpr (EPI == kEpiStore || EPI == kEpiBiasSilu)
+  if constexpr (EPI == kEpiStore || EPI == kEpiBiasSilu || EPI == kEpiAct)
     vec = vec && (m + 3 < a.epi_split || m >= a.epi_split);
   if constexpr (EPI == kEpiScores || EPI == kEpiScoresFolded) {
     if (EPI == kEpiScoresFolded && m >= a.epi_split) {
@@ -99,13 +100,18 @@ __device__ __forceinline__ void gemm_epilogue4(const GemmArgs& a, const GemmGrou
       *reinterpret_cast<uint2*>(static_cast<T*>(a.out1) + o) = *reinterpret_cast<const uint2*>(lo);
       return;
     }
-  } else if constexpr (EPI == kEpiBiasSilu) {
+  } else if constexpr (EPI == kEpiBiasSilu || EPI == kEpiAct) {
     const long long o = row * a.ldc + m;
     if (vec && (o & 3) == 0) {
+      float add[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      if constexpr (EPI == kEpiAct) {
+        const float4 a4 = *reinterpret_cast<const float4*>(a.add_in + row * a.ldc2 + m);
+        add[0] = a4.x; add[1] = a4.y; add[2] = a4.z; add[3] = a4.w;
+      }
       T r[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const float z = v[j] + bias4[j];
+        const float z = v[j] + bias4[j] + add[j];
         r[j] = from_f32<T>(z * sigmoidf_(z));
       }
       *reinterpret_cast<uint2*>(static_cast<T*>(a.out0) + o) = *reinterpret_cast<const uint2*>(r);

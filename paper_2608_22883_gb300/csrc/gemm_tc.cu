@@ -118,12 +118,67 @@ __device__ __forceinline__ void store_key(const GemmArgs& a, const GemmGroup& g,
   }
 }
 
+// kEpiAct: the fp32 term added before the activation (G_h), for the column
+// quads [qlo, qlo + qn) of the tile's rows, staged in shared memory as
+// addt[rows_real][qn * 4] with every thread's loads in flight together
+// (read row by row inside the epilogue they would serialise its rounds).
+__device__ __forceinline__ void stage_add_tile(const GemmArgs& a, const GemmGroup& g, int m0,
+                                               int n0, int rows_real, int n_cols, int qlo, int qn,
+                                               float* addt) {
+  constexpr int kBatch = 8;
+  const int total = rows_real * qn;
+  for (int it0 = threadIdx.x; it0 < total; it0 += kThreads * kBatch) {
+    float4 v[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int it = it0 + j * kThreads;
+      v[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      if (it < total) {
+        const int rr = it / qn, col = (qlo + it - rr * qn) * 4;
+        if (col < n_cols)
+          v[j] = __ldg(reinterpret_cast<const float4*>(
+              a.add_in + ((long long)g.b_row0 + n0 + rr) * a.ldc2 + m0 + col));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int it = it0 + j * kThreads;
+      if (it < total) *reinterpret_cast<float4*>(addt + 4 * (long long)it) = v[j];
+    }
+  }
+}
+
+// kEpiAct: four consecutive activations of output row n (group-local),
+// columns m .. m + nv - 1: SiLU(acc + added term + bias), stored as bf16 (one
+// 8-byte store for a full, aligned quad).
+__device__ __forceinline__ void act_store4(const GemmArgs& a, const GemmGroup& g, int m, int n,
+                                           const float (&v)[4], const float* add4,
+                                           const float* bias4, int nv) {
+  __nv_bfloat16* out = static_cast<__nv_bfloat16*>(a.out0) + ((long long)g.b_row0 + n) * a.ldc + m;
+  float y[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float z = v[j] + add4[j] + bias4[j];
+    y[j] = z * sigmoidf_(z);
+  }
+  if (nv == 4 && (reinterpret_cast<uintptr_t>(out) & 7) == 0) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(y[0], y[1]);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(y[2], y[3]);
+    uint2 u;
+    u.x = *reinterpret_cast<const uint32_t*>(&lo);
+    u.y = *reinterpret_cast<const uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(out) = u;
+  } else {
+    for (int j = 0; j < nv; ++j) out[j] = __float2bfloat16_rn(y[j]);
+  }
+}
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmF0, const __grid_constant__ CUtensorMap tmF1,
                    const __grid_constant__ CUtensorMap tmF2, const __grid_constant__ CUtensorMap tmR0,
                    const __grid_constant__ CUtensorMap tmR1, const __grid_constant__ GemmArgs args) {
-  constexpr bool DUAL = EPI == kEpiScores;
+  constexpr bool DUAL = EPI == kEpiScores || EPI == kEpiAct;
   using C = Cfg<BN, DUAL>;
   const int S = args.splits;
   const uint32_t rank = (uint32_t)((int)blockIdx.x % S);
@@ -308,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- epilogue: all eight warps.  Warp w reads accumulator lanes (rows)
   // 32 (w % 4) .. +31; warps w and w + 4 take the two halves of the columns.
-  if constexpr (EPI == kEpiBiasSilu || EPI == kEpiBiasF32) {
+  if constexpr (EPI == kEpiBiasSilu || EPI == kEpiBiasF32 || EPI == kEpiAct) {
     // the tile's biases (weights: independent of the predecessor), fetched by
     // warps 2-7 while the accumulator is produced
     typedef __nv_bfloat16 Tb;
@@ -317,7 +372,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m = m0 + c;
       float b = 0.0f;
       if (m < m_end) {
-        if (EPI == kEpiBiasSilu && m >= args.epi_split)
+        if ((EPI == kEpiBiasSilu || EPI == kEpiAct) && m >= args.epi_split)
           b = to_f32(static_cast<const Tb*>(args.bias1)[m - args.epi_split]);
         else
           b = to_f32(static_cast<const Tb*>(args.bias0)[m]);
@@ -406,12 +461,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncthreads();
       const int q4 = BN / 4;
       const int items = rows_real * q4;
+      float* addt = part + rows_real * ldp;        // kEpiAct: the added term, [rows][BN]
+      if constexpr (EPI == kEpiAct) {
+        stage_add_tile(args, g, m0, n0, rows_real, n_cols, 0, q4, addt);
+        __syncthreads();
+      }
       for (int it = threadIdx.x; it < items; it += kThreads) {
         const int rr = it / q4, cc = (it - rr * q4) * 4;
         const float4 a4 = *reinterpret_cast<const float4*>(part + rr * ldp + cc);
         if (ok && cc < n_cols) {
-          const float vals[4] = {a4.x, a4.y, a4.z, a4.w};
-          gemm_epilogue4<EPI>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc), bias_s + cc);
+          float vals[4] = {a4.x, a4.y, a4.z, a4.w};
+          if constexpr (EPI == kEpiAct) {
+            act_store4(args, g, m0 + cc, n0 + rr, vals, addt + 4 * it, bias_s + cc,
+                       min(4, n_cols - cc));
+          } else {
+            gemm_epilogue4<EPI>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc), bias_s + cc);
+          }
         }
       }
     } else {
@@ -446,6 +511,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qlo = (int)rank * (BN / 4) / S, qhi = ((int)rank + 1) * (BN / 4) / S;
       const int q4 = qhi - qlo;
       const int items = rows_real * q4;
+      float* addt = part + rows_real * ldp;        // kEpiAct: the added term, [rows][q4 * 4]
+      if constexpr (EPI == kEpiAct) {
+        stage_add_tile(args, g, m0, n0, rows_real, n_cols, qlo, q4, addt);
+        __syncthreads();
+      }
       // two items per thread and round, all their remote loads in flight
       // together.  The closing cluster barrier is split: each thread arrives
       // once its last round's remote loads have been summed, before that
@@ -491,9 +561,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int k = 0; k < 2; ++k) {
           if (rr[k] < 0) continue;
           if (ok && cc[k] < n_cols) {
-            const float vals[4] = {acc[k].x, acc[k].y, acc[k].z, acc[k].w};
-            gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
-                                bias_s + cc[k]);
+            float vals[4] = {acc[k].x, acc[k].y, acc[k].z, acc[k].w};
+            if constexpr (EPI == kEpiAct) {
+              const int it = it0 + k * kThreads;
+              act_store4(args, g, m0 + cc[k], n0 + rr[k], vals, addt + 4 * it, bias_s + cc[k],
+                         min(4, n_cols - cc[k]));
+            } else {
+              gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
+                                  bias_s + cc[k]);
+            }
           }
         }
       }
@@ -651,7 +727,7 @@ static int resident_clusters(int smem, int S) {
 template <int BN, int EPI>
 static cudaError_t launch_tc_inst(GemmArgs& a, const CUtensorMap* maps, int tiles_x, int max_n,
                                   const GemmPlan& p, cudaStream_t s) {
-  constexpr bool DUAL = EPI == kEpiScores;
+  constexpr bool DUAL = EPI == kEpiScores || EPI == kEpiAct;
   auto kern = tc_kernel<BN, EPI>();
   a.splits = p.splits;
   a.stages = p.stages;
@@ -734,7 +810,7 @@ static double plan_cost_us(bool streaming, double stage_kb, double stage_f_bytes
 template <int BN, int EPI>
 static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tiles,
                      GemmPlan& best, double& best_t) {
-  constexpr bool DUAL = EPI == kEpiScores;
+  constexpr bool DUAL = EPI == kEpiScores || EPI == kEpiAct;
   using C = tc::Cfg<BN, DUAL>;
   // folded scores with hi / lo folded keys: the key part's stages hold two
   // feature tiles and issue two MMAs per k-step (the plan is sized for them)
@@ -757,9 +833,16 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
     const int sb = C::stage_bytes(kps, rbox, DF);
     for (int S = 1; S <= 8; ++S) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
+      // the weighted-sum GEMM over <= 1024 entries: its split-K reduction and
+      // activation epilogue (measured ~4 us per round) outweigh the shorter
+      // main loop, so it runs unsplit
+      if (S > 1 && EPI == kEpiAct && kb_total <= 16) break;
       const int nst = (su_total + S - 1) / S;
       const long long ctas = tiles * S;
-      const int staging = EPI == kEpiStoreKeys ? 0 : rows * (BN + 4) * 4;
+      // the accumulator tile [rows][BN + 4] fp32 (and for kEpiAct the added
+      // term [rows][BN] after it)
+      const int staging = EPI == kEpiStoreKeys ? 0
+                          : rows * (BN + 4 + (EPI == kEpiAct ? BN : 0)) * 4;
       for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
         if (sb > budget) continue;
         const int stages = stages_for(nst, budget, sb);
@@ -807,6 +890,7 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
     case kEpiStoreKeys: return plan_epi<kEpiStoreKeys>(a, max_m, max_n);
     case kEpiQueryH: return plan_epi<kEpiQueryH>(a, max_m, max_n);
     case kEpiScoresFolded: return plan_epi<kEpiScoresFolded>(a, max_m, max_n);
+    case kEpiAct: return plan_epi<kEpiAct>(a, max_m, max_n);
     default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
   }
 }
@@ -837,6 +921,7 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
     case kEpiStoreKeys: return launch_tc_epi<kEpiStoreKeys>(a, maps, plan, tiles_x, max_n, s);
     case kEpiQueryH: return launch_tc_epi<kEpiQueryH>(a, maps, plan, tiles_x, max_n, s);
     case kEpiScoresFolded: return launch_tc_epi<kEpiScoresFolded>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiAct: return launch_tc_epi<kEpiAct>(a, maps, plan, tiles_x, max_n, s);
     default: return launch_tc_epi<kEpiBiasF32>(a, maps, plan, tiles_x, max_n, s);
   }
 }

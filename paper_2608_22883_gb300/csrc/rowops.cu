@@ -533,6 +533,37 @@ __global__ void __launch_bounds__(256) transpose_bf16_kernel(const __nv_bfloat16
   for (int j = ty; j < 32; j += 8) out[(long long)(c0 + j) * rows + r0 + tx] = t[tx][j];
 }
 
+// Per image b: out[(b C + c) * ld + j] = in[(off_b + j) * C + c] for entries
+// j < m_b and columns c < C, zero for m_b <= j < ld (the transposed projected
+// values the weighted-sum GEMM reads, K-major over the image's entries).
+// 32 x 32 tiles through shared memory, reads and writes coalesced.
+__global__ void __launch_bounds__(256) transpose_images_kernel(const __nv_bfloat16* __restrict__ in,
+                                                               int C, int ld,
+                                                               const __grid_constant__ ImageTable tab,
+                                                               __nv_bfloat16* __restrict__ out) {
+  __shared__ __nv_bfloat16 t[32][34];
+  const int b = blockIdx.z;
+  const int j0 = blockIdx.x * 32, c0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int m = tab.m[b];
+  for (int jj = ty; jj < 32; jj += 8) {
+    const int j = j0 + jj;
+    t[jj][tx] = j < m ? in[((long long)tab.off[b] + j) * C + c0 + tx] : __float2bfloat16_rn(0.0f);
+  }
+  __syncthreads();
+  for (int cc = ty; cc < 32; cc += 8)
+    out[((long long)b * C + c0 + cc) * ld + j0 + tx] = t[tx][cc];
+}
+
+cudaError_t launch_transpose_images(const void* in, int C, int ld, const ImageTable& tab,
+                                    void* out, cudaStream_t s) {
+  if (tab.B <= 0 || C <= 0 || ld <= 0) return cudaSuccess;
+  if (C % 32 != 0 || ld % 32 != 0) return cudaErrorInvalidValue;
+  transpose_images_kernel<<<dim3(ld / 32, C / 32, tab.B), 256, 0, s>>>(
+      (const __nv_bfloat16*)in, C, ld, tab, (__nv_bfloat16*)out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_transpose_bf16(const void* in, int rows, int cols, void* out, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return cudaSuccess;
   if (rows % 32 != 0 || cols % 32 != 0) return cudaErrorInvalidValue;

@@ -22,6 +22,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   const int tid = threadIdx.x;
   pdl_wait();
   pdl_trigger();
+  clear_alpha(a, n, tid, kSelThreads);    // ordered before the weights by the group barriers
   const int b = seq_of_row(tab, n);
   const int M = tab.m[b];
   if (M == 0 || row_gated(a.gate, n)) {   // empty valid set or past the depth gate: K = 0
@@ -41,7 +42,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
                           float rho, int k_min, int k_max, int max_m, const DepthGate& gate,
                           int32_t* counts, int32_t* indices, int32_t* sel_pos, float* sel_w,
-                          int32_t* sel_cnt, cudaStream_t s) {
+                          int32_t* sel_cnt, cudaStream_t s, void* alpha_hi, void* alpha_lo,
+                          int alpha_ld) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)max(max_m, 1) * sizeof(float);
   static bool configured = false;
@@ -52,7 +54,9 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
     configured = true;
   }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt,
-               nullptr, nullptr, nullptr, gate};
+               nullptr, nullptr, nullptr, gate,
+               static_cast<__nv_bfloat16*>(alpha_hi), static_cast<__nv_bfloat16*>(alpha_lo),
+               alpha_ld};
   return launch_pdl(select_kernel, dim3(N), dim3(kSelThreads), smem, s, a, tab);
 }
 

@@ -52,7 +52,33 @@ struct SelectArgs {
   float* loc_w;
   int* loc_cnt;
   DepthGate gate;      // rows past the depth gate select nothing (K = 0)
+  // the renormalised weights as dense rows over the sequence's entries, a
+  // bf16 hi / lo pair [N, alpha_ld] (zero where not selected), or null
+  __nv_bfloat16* alpha_hi;
+  __nv_bfloat16* alpha_lo;
+  int alpha_ld;
 };
+
+// Weight alpha of the entry at position pos (within its sequence) of row n
+// into the dense rows (the caller zero-filled them first).
+__device__ __forceinline__ void put_alpha(const SelectArgs& a, int n, int pos, float w) {
+  if (a.alpha_hi == nullptr) return;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(w);
+  const long long o = (long long)n * a.alpha_ld + pos;
+  a.alpha_hi[o] = hi;
+  a.alpha_lo[o] = __float2bfloat16_rn(w - __bfloat162float(hi));
+}
+
+// Zero-fills row n of the dense weights (group of `nthreads`, index tid).
+__device__ __forceinline__ void clear_alpha(const SelectArgs& a, int n, int tid, int nthreads) {
+  if (a.alpha_hi == nullptr) return;
+  const long long o = (long long)n * a.alpha_ld;
+  const __nv_bfloat16 z = __float2bfloat16_rn(0.0f);
+  for (int j = tid; j < a.alpha_ld; j += nthreads) {
+    a.alpha_hi[o + j] = z;
+    a.alpha_lo[o + j] = z;
+  }
+}
 
 struct SelectSmem {
   unsigned long long cand[FOVEA_MAX_K];      // (key << 32) | ~position
@@ -118,9 +144,12 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
   const int K_eff = min(k_max, M);
 
   // ---- radix select of the K_eff-th largest key ----------------------------
+  // (every entry selected, the dense setting: no threshold to find; every
+  // key is above 0, so T = 0 takes them all)
   uint32_t prefix = 0, pmask = 0;
   int krem = K_eff;                       // entries still to take at the current prefix
-  for (int shift = 24; shift >= 0; shift -= 8) {
+  if (K_eff == M) krem = 0;
+  for (int shift = 24; shift >= 0 && K_eff < M; shift -= 8) {
     for (int i = tid; i < 256; i += kSelThreads) sm.hist[i] = 0;
     sync();
     // warp-aggregated histogram: lanes with the same digit add once
@@ -297,6 +326,7 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
       const int row = key_off + pos;
       if (a.sel_pos) a.sel_pos[out_row + t] = row;
       if (a.sel_w) a.sel_w[out_row + t] = e / denom;
+      put_alpha(a, n, pos, e / denom);
       if (a.loc_pos) {
         a.loc_pos[t] = row;
         a.loc_w[t] = e / denom;
@@ -497,6 +527,7 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
       const int row = key_off + pu;
       if (a.sel_pos) a.sel_pos[out_row + u] = row;
       if (a.sel_w) a.sel_w[out_row + u] = eu / denom;
+      put_alpha(a, n, pu, eu / denom);
       if (a.loc_pos) {
         a.loc_pos[u] = row;
         a.loc_w[u] = eu / denom;

@@ -55,6 +55,10 @@ SMALL = {
     "bf16-clustered": dict(d=256, m_sizes=[2048], rows=[128], clusters=16, cluster_sigma=0.2,
                            k_max=256),
     "bf16-many-rows": dict(d=256, m_sizes=[130, 500], rows=[300, 4], k_max=64),
+    # more rows than twice the SMs: the selection writes dense weights and one
+    # GEMM against the transposed projected values forms the first fusion layer
+    "bf16-many-rows-dense-weights": dict(d=256, m_sizes=[130, 500, 77], rows=[300, 10, 40],
+                                         k_max=64, temperature=(0.3, 3.0)),
     # rows beyond 2048 entries: selection and readout run as two kernels
     "bf16-long-rows": dict(d=256, m_sizes=[2500, 300], rows=[12, 5], k_max=64),
     "bf16-hidden-128": dict(d=256, m_sizes=[100], rows=[9], k_max=16, H=128),
@@ -208,10 +212,12 @@ def test_folded_and_unfolded_steps_select_the_same_entries(fovea, name):
 
 
 def test_paths_are_taken(fovea):
-    """bf16 rows of up to 2048 entries run the selection, the projected
-    readout and the first fusion layer's activation in one kernel; beyond
-    that, selection and readout run as two kernels and the first fusion layer
-    as a GEMM; fp32 takes the unfolded SIMT path."""
+    """bf16 rows of up to 2048 entries, caps of up to 256 and batches of up
+    to twice the SMs run the selection, the projected readout and the first
+    fusion layer's activation in one kernel; otherwise the selection writes
+    dense weights and one GEMM against the transposed projected values forms
+    the activation (the readout, when asked for, has its own kernel); fp32
+    takes the unfolded SIMT path with the first fusion layer as a GEMM."""
     try:
         for name, want, absent in (
                 # several score groups: G_h in a launch of its own
@@ -219,8 +225,11 @@ def test_paths_are_taken(fovea):
                  {"ln_query", "fusion_h", "score_folded", "select_fuse", "fuse_out", "finalize"},
                  "query_proj"),
                 ("bf16-one-group-offset", {"score_fusion_h", "select_fuse"}, "score_folded"),
-                ("bf16-long-rows", {"score_folded", "select", "readout", "fuse_hidden"},
-                 "query_proj"),
+                # long rows: selection with dense weights, the weighted sum as a GEMM
+                ("bf16-long-rows", {"score_folded", "select", "readout", "act_gemm", "fuse_out"},
+                 "fuse_hidden"),
+                ("bf16-many-rows-dense-weights", {"select", "act_gemm"}, "select_fuse"),
+                ("bf16-dense-wide", {"select", "act_gemm"}, "fuse_hidden"),
                 ("fp32-ragged", {"query_proj", "score", "select_readout", "fuse_hidden"},
                  "select_fuse")):
             s = store(small_workload(name))
