@@ -677,7 +677,7 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
     gen = torch.Generator(device=h_hat.device)
     gen.manual_seed(seed)
     W = (torch.randn((vocab, d), generator=gen, device=h_hat.device) / math.sqrt(d)).to(torch.bfloat16)
-    ws = torch.zeros(1 << 14, dtype=torch.uint8, device=h_hat.device)
+    ws = fovea.lm_head_workspace(vocab, d, N, k_c)
     logits = torch.empty((N, vocab), dtype=torch.float32, device=h_hat.device)
     ms = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits), flush, n_steps)
     fovea.sync_errors(ws)

@@ -288,15 +288,26 @@ FOVEA_API fovea_status fovea_noalloc_sync_errors(void* stream);
  *   logits    [N, vocab] device fp32, caller-owned: z (written)
  *   top_idx   [N, k_c] device int32: token indices (written)
  *   top_val   [N, k_c] device fp32: their logits (or NULL)
- *   workspace an initialised step workspace (its error word; >= 16 KB)
+ *   workspace device memory of fovea_lm_head_workspace_size bytes (256-byte
+ *             aligned), its header initialised with fovea_workspace_init:
+ *             the error word, then the candidates (the GEMM's epilogue keeps
+ *             each row's k_c largest logits of every tile; a second kernel
+ *             merges them)
  * bf16 only (fp32 returns UNSUPPORTED); 1 <= k_c <= FOVEA_MAX_KC <= vocab;
  * accumulation in fp32.  Enqueued on `stream`, no host synchronisation.
+ * Enqueued on the stream of a draft step right after fovea_retrieve_fuse, the
+ * LM-head GEMM starts streaming W_LM while the step's last kernel runs
+ * (programmatic dependent launch): the logits follow the corrected states
+ * without a host round trip.
  * Errors: INVALID_ARG, UNSUPPORTED (nothing enqueued), CUDA.
  */
 FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_model, int dtype,
                                           const void* h_hat, int N, int k_c, float* logits,
                                           int32_t* top_idx, float* top_val, void* workspace,
                                           size_t workspace_bytes, void* stream);
+/* Workspace bytes of fovea_lm_head_topk for this shape.  Errors: INVALID_ARG. */
+FOVEA_API fovea_status fovea_lm_head_workspace_size(int vocab, int d_model, int N, int k_c,
+                                                    size_t* bytes);
 
 /* Synchronise `stream`, read and clear the workspace's sticky error word.
  * Returns FOVEA_OK, FOVEA_ERR_INVALID_ARG (a depth outside [0, D] was seen)

@@ -525,6 +525,11 @@ struct WsLayout {
   size_t err, xh, q, scores, sel_pos, sel_w, sel_cnt, r_lo, act, c, gh, alpha_hi, alpha_lo, total;
 };
 
+// LM head workspace: the header, then the candidate keys [N, slots, k_c].
+size_t lm_head_ws_bytes(int N, int slots, int k_c) {
+  return kWsHeaderBytes + (size_t)N * slots * k_c * sizeof(unsigned long long);
+}
+
 int device_sms() {
   static int sms = 0;
   if (sms == 0) {
@@ -1023,32 +1028,53 @@ FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_mod
   if (top_idx == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "top_idx is NULL");
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");
-  if (workspace_bytes < kWsHeaderBytes)
-    return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs at least %zu",
-                workspace_bytes, kWsHeaderBytes);
   if (dtype != FOVEA_BF16)
     return fail(FOVEA_ERR_UNSUPPORTED, "the LM head runs on bf16 weights and states only");
   if (N == 0) return FOVEA_OK;
+  const int slots = lm_head_slots(vocab, d_model, N);
+  const size_t need = lm_head_ws_bytes(N, slots, k_c);
+  if (workspace_bytes < need)
+    return fail(FOVEA_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu "
+                "(fovea_lm_head_workspace_size)", workspace_bytes, need);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // z = h_hat W_LM^T: W_LM [vocab, d] is the feature operand, streamed once;
-  // every column goes to the fp32 output (the G_h epilogue with its split at 0)
+  // every column goes to the fp32 logits, and the epilogue keeps each row's
+  // k_c largest of every tile as candidates after the header
+  unsigned long long* cand = reinterpret_cast<unsigned long long*>(
+      static_cast<uint8_t*>(workspace) + kWsHeaderBytes);
   static thread_local GemmArgs a;
   init_args(a);
   a.k_total = d_model; a.b_split = d_model;
   a.epi_split = 0;
   a.out2 = logits; a.ldc2 = vocab;
+  a.cand = cand; a.cand_k = k_c; a.cand_ld = (long long)slots * k_c;
   a.err = static_cast<int*>(workspace);
   a.ngroups = 1;
   a.groups[0] = GemmGroup{0, vocab, 0, N, 0};
   cudaError_t e;
   { KernelTimer t("lm_head", s);
-    e = launch_gemm_tc(kEpiQueryH, a, TmaOperand{W_LM, vocab, d_model, d_model},
+    e = launch_gemm_tc(kEpiLogits, a, TmaOperand{W_LM, vocab, d_model, d_model},
                        TmaOperand{nullptr, 0, 0, 0}, TmaOperand{h_hat, N, d_model, d_model},
                        TmaOperand{nullptr, 0, 0, 0}, vocab, N, s); }
   if (e != cudaSuccess) return cuda_fail(e, "lm_head");
-  { KernelTimer t("topk", s);
-    e = launch_topk_rows(logits, N, vocab, k_c, top_idx, top_val, s); }
-  if (e != cudaSuccess) return cuda_fail(e, "topk");
+  { KernelTimer t("merge_candidates", s);
+    e = launch_merge_candidates(cand, N, slots, k_c, top_idx, top_val, s); }
+  if (e != cudaSuccess) return cuda_fail(e, "merge_candidates");
+  return FOVEA_OK;
+}
+
+FOVEA_API fovea_status fovea_lm_head_workspace_size(int vocab, int d_model, int N, int k_c,
+                                                    size_t* bytes) {
+  g_last_error.clear();
+  if (bytes == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "bytes is NULL");
+  if (d_model <= 0 || d_model % 64 != 0 || d_model > FOVEA_MAX_D)
+    return fail(FOVEA_ERR_INVALID_ARG, "d_model %d must be a positive multiple of 64 (<= %d)",
+                d_model, FOVEA_MAX_D);
+  if (N < 0) return fail(FOVEA_ERR_INVALID_ARG, "N = %d < 0", N);
+  if (k_c < 1 || k_c > FOVEA_MAX_KC)
+    return fail(FOVEA_ERR_INVALID_ARG, "k_c = %d must lie in [1, %d]", k_c, FOVEA_MAX_KC);
+  if (vocab < k_c) return fail(FOVEA_ERR_INVALID_ARG, "vocab %d < k_c %d", vocab, k_c);
+  *bytes = N == 0 ? kWsHeaderBytes : lm_head_ws_bytes(N, lm_head_slots(vocab, d_model, N), k_c);
   return FOVEA_OK;
 }
 

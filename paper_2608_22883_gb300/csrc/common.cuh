@@ -147,6 +147,10 @@ enum EpiKind : int {
                          // operand is the weights' hi / lo pair (B0, B1, both multiplied by
                          // the same feature tile); out0[row * ldc + col] =
                          // T(silu(acc + add_in[row * ldc2 + col] + bias{0,1}[col]))
+  kEpiLogits = 9,        // the draft logits: out2 (fp32)[row * ldc2 + col] = acc, and per row
+                         // the cand_k largest of the CTA's columns as 64-bit keys (logit order
+                         // key << 32 | ~column) into cand[row * cand_ld + slot * cand_k + r],
+                         // slot = feature tile * splits + rank
 };
 
 struct KeyFix {       // one listed key element: memory row, feature
@@ -181,6 +185,9 @@ struct GemmArgs {
   int rbox;           // tensor-core path: rows of a row-operand tile (64 or 128)
   int region;         // tensor-core path: bytes of the ring / partial-tile staging region
   const float* add_in;          // kEpiAct: fp32 term added before the activation
+  unsigned long long* cand;     // kEpiLogits: per-row candidate keys
+  long long cand_ld;
+  int cand_k;
   unsigned long long wait_ns;   // tensor-core path: limit of a bounded mbarrier wait
   int* err;
   // tensor-core path: byte ranges whose share each CTA prefetches into L2 once
@@ -290,10 +297,14 @@ struct ImageTable {
 cudaError_t launch_transpose_images(const void* in, int C, int ld, const ImageTable& tab,
                                     void* out, cudaStream_t s);
 
-// Per row of logits [N, V] fp32: the k <= FOVEA_MAX_KC largest in
-// descending order (ties: smaller index first), indices and values.
-cudaError_t launch_topk_rows(const float* logits, int N, long long V, int k, int32_t* top_idx,
-                             float* top_val, cudaStream_t s);
+// Per row n: the k <= FOVEA_MAX_KC largest of the candidate keys
+// cand[n * slots * k .. + slots * k) (logit order key << 32 | ~index) in
+// descending order, as token indices and logits.
+cudaError_t launch_merge_candidates(const unsigned long long* cand, int N, int slots, int k,
+                                    int32_t* top_idx, float* top_val, cudaStream_t s);
+// Candidate slots per row the LM-head GEMM writes for this shape (its feature
+// tiles times its split-K factor).
+int lm_head_slots(int vocab, int d_model, int N);
 
 cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFix* list,
                                const int* count, int cap, int rows, void* K, cudaStream_t s);

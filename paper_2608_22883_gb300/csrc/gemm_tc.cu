@@ -47,6 +47,7 @@
 // stages before griddepcontrol.wait; those operands never depend on the
 // previous kernel, so the weight stream starts while the predecessor drains.
 #include <atomic>
+#include <cstring>
 
 #include "gemm_epilogue.cuh"
 #include "tc_ptx.cuh"
@@ -144,6 +145,79 @@ __device__ __forceinline__ void stage_add_tile(const GemmArgs& a, const GemmGrou
     for (int j = 0; j < kBatch; ++j) {
       const int it = it0 + j * kThreads;
       if (it < total) *reinterpret_cast<float4*>(addt + 4 * (long long)it) = v[j];
+    }
+  }
+}
+
+// Order-preserving map of a float to an unsigned key (larger float, larger key).
+__device__ __forceinline__ uint32_t logit_order_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// kEpiLogits: per row of the tile, the cand_k largest of `ncols` logits
+// (vals [rows_real][ld] in shared memory, column c is token col0 + c) into
+// the row's candidate slot as 64-bit keys, logit order key << 32 | ~token
+// (on equal logits the smaller token is larger).  One warp per row, each lane
+// holding the order keys of columns lane, lane + 32, ...; each of the k rounds
+// takes the lane maxima (the smallest column on equal keys), a warp maximum,
+// the smallest column holding it (warp minimum), and clears that key: short,
+// independent steps.  A zero key (fewer columns than cand_k) sorts below every
+// real one.
+template <int BN>
+__device__ __forceinline__ void tile_topk(const GemmArgs& a, long long row0, int rows_real,
+                                          const float* vals, int ld, int col0, int ncols,
+                                          int slot) {
+  constexpr int J = (BN + 31) / 32;
+  constexpr int R = 4;                       // rows a warp works on together (independent chains)
+  constexpr int kWarps = kThreads / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = a.cand_k;
+  for (int base = warp; base < rows_real; base += kWarps * R) {
+    uint32_t key[R][J];
+#pragma unroll
+    for (int u = 0; u < R; ++u) {
+      const int rr = base + u * kWarps;
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const int c = lane + 32 * j;
+        key[u][j] = (rr < rows_real && c < ncols) ? logit_order_key(vals[rr * ld + c]) : 0u;
+      }
+    }
+    for (int r = 0; r < k; ++r) {
+      uint32_t w[R], cmin[R];
+#pragma unroll
+      for (int u = 0; u < R; ++u) {
+        uint32_t m = key[u][0];
+        int jm = 0;
+#pragma unroll
+        for (int j = 1; j < J; ++j)
+          if (key[u][j] > m) {
+            m = key[u][j];
+            jm = j;
+          }
+        w[u] = __reduce_max_sync(0xffffffffu, m);
+        const uint32_t col = m == w[u] ? (uint32_t)(lane + 32 * jm) : 0xFFFFFFFFu;
+        cmin[u] = __reduce_min_sync(0xffffffffu, col);
+        if (col == cmin[u]) {
+#pragma unroll
+          for (int j = 0; j < J; ++j)
+            if (j == jm) key[u][j] = 0u;
+        }
+      }
+      if (lane < R) {
+        const int rr = base + lane * kWarps;
+        uint32_t wl = 0u, cl = 0u;
+#pragma unroll
+        for (int u = 0; u < R; ++u)
+          if (u == lane) {
+            wl = w[u];
+            cl = cmin[u];
+          }
+        if (rr < rows_real)
+          a.cand[(row0 + rr) * a.cand_ld + (long long)slot * k + r] =
+              wl == 0u ? 0ull : ((unsigned long long)wl << 32) | (0xFFFFFFFFu - (uint32_t)col0 - cl);
+      }
     }
   }
 }
@@ -474,11 +548,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           if constexpr (EPI == kEpiAct) {
             act_store4(args, g, m0 + cc, n0 + rr, vals, addt + 4 * it, bias_s + cc,
                        min(4, n_cols - cc));
+          } else if constexpr (EPI == kEpiLogits) {
+            gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc),
+                                       bias_s + cc);
           } else {
             gemm_epilogue4<EPI>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc), bias_s + cc);
           }
         }
       }
+      if constexpr (EPI == kEpiLogits)
+        tile_topk<BN>(args, (long long)g.b_row0 + n0, rows_real, part, ldp, m0, n_cols, tx);
     } else {
       // Split K: each CTA stages its fp32 partial tile row-major [rows][BN + 4]
       // over its idle ring (the pitch spreads a warp's 16-byte stores over all
@@ -512,6 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int q4 = qhi - qlo;
       const int items = rows_real * q4;
       float* addt = part + rows_real * ldp;        // kEpiAct: the added term, [rows][q4 * 4]
+      float* sums = part + rows_real * ldp;        // kEpiLogits: the reduced logits, [rows][q4 * 4]
       if constexpr (EPI == kEpiAct) {
         stage_add_tile(args, g, m0, n0, rows_real, n_cols, qlo, q4, addt);
         __syncthreads();
@@ -566,6 +646,11 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int it = it0 + k * kThreads;
               act_store4(args, g, m0 + cc[k], n0 + rr[k], vals, addt + 4 * it, bias_s + cc[k],
                          min(4, n_cols - cc[k]));
+            } else if constexpr (EPI == kEpiLogits) {
+              const int it = it0 + k * kThreads;
+              *reinterpret_cast<float4*>(sums + 4 * it) = acc[k];
+              gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc[k], n0 + rr[k], vals,
+                                         min(4, n_cols - cc[k]), bias_s + cc[k]);
             } else {
               gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
                                   bias_s + cc[k]);
@@ -576,6 +661,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (rounds == 0) {
         __syncwarp();
         cluster_arrive();
+      }
+      if constexpr (EPI == kEpiLogits) {
+        __syncthreads();
+        tile_topk<BN>(args, (long long)g.b_row0 + n0, rows_real, sums, q4 * 4, m0 + qlo * 4,
+                      max(0, min(q4 * 4, n_cols - qlo * 4)), tx * S + (int)rank);
       }
       cluster_wait();   // no CTA leaves while another still reads its partial tile
     }
@@ -839,10 +929,10 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
       if (S > 1 && EPI == kEpiAct && kb_total <= 16) break;
       const int nst = (su_total + S - 1) / S;
       const long long ctas = tiles * S;
-      // the accumulator tile [rows][BN + 4] fp32 (and for kEpiAct the added
-      // term [rows][BN] after it)
+      // the accumulator tile [rows][BN + 4] fp32 (and after it, for kEpiAct
+      // the added term, for split kEpiLogits the reduced logits, [rows][BN])
       const int staging = EPI == kEpiStoreKeys ? 0
-                          : rows * (BN + 4 + (EPI == kEpiAct ? BN : 0)) * 4;
+                          : rows * (BN + 4 + ((EPI == kEpiAct || (EPI == kEpiLogits && S > 1)) ? BN : 0)) * 4;
       for (int budget : {tc::kSmemBudget, tc::kSmemBudgetPair}) {
         if (sb > budget) continue;
         const int stages = stages_for(nst, budget, sb);
@@ -891,8 +981,23 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
     case kEpiQueryH: return plan_epi<kEpiQueryH>(a, max_m, max_n);
     case kEpiScoresFolded: return plan_epi<kEpiScoresFolded>(a, max_m, max_n);
     case kEpiAct: return plan_epi<kEpiAct>(a, max_m, max_n);
+    case kEpiLogits: return plan_epi<kEpiLogits>(a, max_m, max_n);
     default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
   }
+}
+
+int lm_head_slots(int vocab, int d_model, int N) {
+  static thread_local GemmArgs a;
+  memset(&a, 0, sizeof(a));
+  a.k_total = d_model;
+  a.b_split = d_model;
+  a.a_split = 0x7fffffff;
+  a.a_split2 = 0x7fffffff;
+  a.epi_split = 0;
+  a.ngroups = 1;
+  a.groups[0] = GemmGroup{0, vocab, 0, N, 0};
+  const GemmPlan p = plan_gemm_tc(kEpiLogits, a, vocab, N);
+  return feature_tiles(a, vocab, p.bn) * p.splits;
 }
 
 cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, const TmaOperand& A1,
@@ -922,6 +1027,7 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
     case kEpiQueryH: return launch_tc_epi<kEpiQueryH>(a, maps, plan, tiles_x, max_n, s);
     case kEpiScoresFolded: return launch_tc_epi<kEpiScoresFolded>(a, maps, plan, tiles_x, max_n, s);
     case kEpiAct: return launch_tc_epi<kEpiAct>(a, maps, plan, tiles_x, max_n, s);
+    case kEpiLogits: return launch_tc_epi<kEpiLogits>(a, maps, plan, tiles_x, max_n, s);
     default: return launch_tc_epi<kEpiBiasF32>(a, maps, plan, tiles_x, max_n, s);
   }
 }

@@ -2,41 +2,33 @@
 // hidden_correction) and, per row, the K_c largest logits in descending
 // order, ties broken by the smaller token index (the candidate width K_c of
 // the experimental setup).  The logits come from the tensor-core GEMM
-// (gemm_tc.cu) streaming W_LM; this file holds the per-row candidate
-// selection.
+// (gemm_tc.cu) streaming W_LM, whose epilogue also keeps, per row and tile,
+// the K_c largest of the tile's logits; this file merges those candidates.
 #include "common.cuh"
 
 namespace fovea {
 
 namespace {
 
-constexpr int kTopKThreads = 256;    // registers: up to FOVEA_MAX_KC 64-bit keys per thread
-constexpr int kBatch = 16;           // logits loaded together per thread
+constexpr int kMergeThreads = 256;   // registers: up to FOVEA_MAX_KC 64-bit keys per thread
 
-// Order-preserving map of a float to an unsigned key (larger float, larger key).
-__device__ __forceinline__ uint32_t logit_key(float f) {
-  const uint32_t u = __float_as_uint(f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-
-// One CTA per row.  Each thread keeps the k largest of its strided logits as
-// 64-bit keys (logit key << 32 | ~index: distinct, and on equal logits the
-// smaller index is larger) in KC register slots (KC >= k, a compile-time
+// One CTA per row over the row's candidate keys (each the cand_k largest of
+// one GEMM tile's columns, as logit order key << 32 | ~token: distinct, and
+// on equal logits the smaller token is larger).  Each thread keeps the k
+// largest of its strided keys in KC register slots (KC >= k, a compile-time
 // size so the slots stay in registers), unsorted, with the position of the
-// smallest: a larger key replaces the smallest.  Then k rounds of a
-// block-wide maximum over the threads' largest keys, the owner clearing the
-// winner.  A zero key is below every real one (the key of -inf is
-// 0x007FFFFF in the upper half); slots k .. KC-1 stay zero.
+// smallest; then k rounds of a block-wide maximum, the owner clearing the
+// winner.  A zero key (a tile with fewer columns than k) is below every real
+// one.  The logit is recovered from the key (the order map is a bijection).
 template <int KC>
-__global__ void __launch_bounds__(kTopKThreads) topk_rows_kernel(const float* __restrict__ logits,
-                                                                long long V, int k,
-                                                                int32_t* __restrict__ top_idx,
-                                                                float* __restrict__ top_val) {
-  __shared__ unsigned long long red[kTopKThreads / 32];
+__global__ void __launch_bounds__(kMergeThreads) merge_candidates_kernel(
+    const unsigned long long* __restrict__ cand, int total, int k, int32_t* __restrict__ top_idx,
+    float* __restrict__ top_val) {
+  __shared__ unsigned long long red[kMergeThreads / 32];
   __shared__ unsigned long long best;
   const int n = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const float* z = logits + (long long)n * V;
+  const unsigned long long* c = cand + (long long)n * total;
   pdl_wait();
   pdl_trigger();
   unsigned long long loc[KC];
@@ -44,21 +36,17 @@ __global__ void __launch_bounds__(kTopKThreads) topk_rows_kernel(const float* __
   for (int i = 0; i < KC; ++i) loc[i] = 0ull;
   unsigned long long lowest = 0ull;           // the smallest of slots 0 .. k-1
   int low_pos = 0;
-  // the thread's logits in batches of kBatch, every load of a batch in
-  // flight before the first comparison
-  for (long long j0 = tid; j0 < V; j0 += (long long)kBatch * kTopKThreads) {
-    float v[kBatch];
+  constexpr int kBatch = 4;
+  for (int j0 = tid; j0 < total; j0 += kBatch * kMergeThreads) {
+    unsigned long long v[kBatch];
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {
-      const long long j = j0 + (long long)u * kTopKThreads;
-      v[u] = j < V ? z[j] : 0.0f;
+      const int j = j0 + u * kMergeThreads;
+      v[u] = j < total ? c[j] : 0ull;
     }
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {
-      const long long j = j0 + (long long)u * kTopKThreads;
-      if (j >= V) continue;
-      const unsigned long long key =
-          ((unsigned long long)logit_key(v[u]) << 32) | (0xFFFFFFFFu - (uint32_t)j);
+      const unsigned long long key = v[u];
       if (key <= lowest) continue;
 #pragma unroll
       for (int i = 0; i < KC; ++i)
@@ -91,7 +79,7 @@ __global__ void __launch_bounds__(kTopKThreads) topk_rows_kernel(const float* __
     if (lane == 0) red[warp] = m;
     __syncthreads();
     if (warp == 0) {
-      m = lane < kTopKThreads / 32 ? red[lane] : 0ull;
+      m = lane < kMergeThreads / 32 ? red[lane] : 0ull;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const unsigned long long t = __shfl_xor_sync(0xffffffffu, m, o);
@@ -107,24 +95,26 @@ __global__ void __launch_bounds__(kTopKThreads) topk_rows_kernel(const float* __
         if (i == mine_pos) loc[i] = 0ull;
     }
     if (tid == 0) {
-      const uint32_t j = 0xFFFFFFFFu - (uint32_t)(b & 0xFFFFFFFFull);
-      top_idx[(long long)n * k + r] = (int32_t)j;
-      if (top_val != nullptr) top_val[(long long)n * k + r] = z[j];
+      const uint32_t key = (uint32_t)(b >> 32);
+      const uint32_t bits = (key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key;
+      top_idx[(long long)n * k + r] = (int32_t)(0xFFFFFFFFu - (uint32_t)(b & 0xFFFFFFFFull));
+      if (top_val != nullptr) top_val[(long long)n * k + r] = __uint_as_float(bits);
     }
   }
 }
 
 }  // namespace
 
-cudaError_t launch_topk_rows(const float* logits, int N, long long V, int k, int32_t* top_idx,
-                             float* top_val, cudaStream_t s) {
+cudaError_t launch_merge_candidates(const unsigned long long* cand, int N, int slots, int k,
+                                    int32_t* top_idx, float* top_val, cudaStream_t s) {
   if (N == 0) return cudaSuccess;
-  if (k < 1 || k > FOVEA_MAX_KC || V < k) return cudaErrorInvalidValue;
+  if (k < 1 || k > FOVEA_MAX_KC || slots < 1) return cudaErrorInvalidValue;
+  const int total = slots * k;
   if (k <= 8)
-    return launch_pdl(topk_rows_kernel<8>, dim3(N), dim3(kTopKThreads), 0, s, logits, V, k,
-                      top_idx, top_val);
-  return launch_pdl(topk_rows_kernel<FOVEA_MAX_KC>, dim3(N), dim3(kTopKThreads), 0, s, logits, V,
-                    k, top_idx, top_val);
+    return launch_pdl(merge_candidates_kernel<8>, dim3(N), dim3(kMergeThreads), 0, s, cand, total,
+                      k, top_idx, top_val);
+  return launch_pdl(merge_candidates_kernel<FOVEA_MAX_KC>, dim3(N), dim3(kMergeThreads), 0, s, cand,
+                    total, k, top_idx, top_val);
 }
 
 }  // namespace fovea

@@ -36,7 +36,7 @@ EXPORTS = (
     "fovea_workspace_size", "fovea_workspace_init", "fovea_retrieve_fuse", "fovea_sync_errors",
     "fovea_last_error", "fovea_timing_enable", "fovea_timing_read", "fovea_version",
     "fovea_retrieve_fuse_noalloc", "fovea_noalloc_sync_errors", "fovea_memory_folded_keys",
-    "fovea_lm_head_topk", "fovea_debug_wait_limit",
+    "fovea_lm_head_topk", "fovea_debug_wait_limit", "fovea_lm_head_workspace_size",
 )
 NOALLOC_WORKSPACE_BYTES = 32 << 20
 
@@ -87,6 +87,9 @@ def lib() -> ctypes.CDLL:
                                                   ctypes.c_float, ctypes.c_int, ctypes.c_int,
                                                   ctypes.c_int, vp, vp, vp, vp, vp, vp]
         L.fovea_retrieve_fuse_noalloc.restype = ctypes.c_int
+        L.fovea_lm_head_workspace_size.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                    ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]
+        L.fovea_lm_head_workspace_size.restype = ctypes.c_int
         L.fovea_noalloc_sync_errors.argtypes = [vp]
         L.fovea_noalloc_sync_errors.restype = ctypes.c_int
         L.fovea_debug_wait_limit.argtypes = [ctypes.c_ulonglong]
@@ -325,6 +328,15 @@ def debug_wait_limit(limit_ns: int) -> None:
     """fovea_debug_wait_limit: limit of the bounded device waits of later
     launches (0: the default of about 2 s).  For tests of the timeout path."""
     _check(lib().fovea_debug_wait_limit(int(limit_ns)))
+
+
+def lm_head_workspace(vocab: int, d_model: int, N: int, k_c: int, stream=None) -> torch.Tensor:
+    """An initialised workspace for fovea_lm_head_topk of this shape."""
+    n = ctypes.c_size_t()
+    _check(lib().fovea_lm_head_workspace_size(vocab, d_model, N, k_c, ctypes.byref(n)))
+    ws = torch.empty(n.value, dtype=torch.uint8, device="cuda")
+    _check(lib().fovea_workspace_init(_ptr(ws), ws.numel(), _stream(stream)))
+    return ws
 
 
 def lm_head_topk(W_LM: torch.Tensor, h_hat: torch.Tensor, k_c: int, workspace: torch.Tensor,

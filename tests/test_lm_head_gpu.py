@@ -38,7 +38,7 @@ def check(fovea, V, d, N, k_c, seed, ties=False):
     Wt, ht = bf16(W).cuda(), bf16(h).cuda()
     W64 = Wt.double().cpu().numpy()
     h64 = ht.double().cpu().numpy()
-    ws = torch.zeros(1 << 14, dtype=torch.uint8, device="cuda")
+    ws = fovea.lm_head_workspace(V, d, N, k_c)
     idx, val, logits = fovea.lm_head_topk(Wt, ht, k_c, ws)
     torch.cuda.synchronize()
     fovea.sync_errors(ws)
