@@ -481,10 +481,32 @@ cudaError_t launch_readout(int dtype, const void* U, const int32_t* sel_cnt, con
 
 // ---------------------------------------------------------------------------
 // Exact rounding of listed key elements (memory equation k_i = W_K LN(v_i)):
-// one warp per element; products of two bf16 values are exact in fp32 and are
-// summed in double-float, then rounded once.
+// one warp per element, 16-byte loads of both rows.  Products of two bf16
+// values are exact in fp32; each lane sums its products with the cascaded
+// (compensated) summation of Ogita, Rump and Oishi ("Accurate sum and dot
+// product", 2005, Algorithm Sum2: TwoSum of the running sum and the product,
+// the rounding errors added separately), whose error is below
+// eps |S| + (n eps)^2 sum |p| -- about 2^-27 of the key for d <= 8192, far
+// inside the distance of any listed element from a bf16 midpoint that matters
+// -- and the lanes' (sum, error) pairs are combined in double-float before
+// the single rounding to bf16.
 // ---------------------------------------------------------------------------
 constexpr int kRefineThreads = 256;
+
+__device__ __forceinline__ void sum2_bf16x8(const uint4& xa, const uint4& wa, float& s, float& c) {
+  const uint32_t xs[4] = {xa.x, xa.y, xa.z, xa.w}, ws[4] = {wa.x, wa.y, wa.z, wa.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float xf = __uint_as_float(h ? (xs[q] & 0xFFFF0000u) : (xs[q] << 16));
+      const float wf = __uint_as_float(h ? (ws[q] & 0xFFFF0000u) : (ws[q] << 16));
+      const dfloat t = df_two_sum(s, __fmul_rn(xf, wf));       // the product is exact
+      s = t.hi;
+      c = __fadd_rn(c, t.lo);
+    }
+  }
+}
 
 __global__ void __launch_bounds__(kRefineThreads) refine_keys_kernel(
     const __nv_bfloat16* __restrict__ xv, const __nv_bfloat16* __restrict__ W, int d,
@@ -493,6 +515,7 @@ __global__ void __launch_bounds__(kRefineThreads) refine_keys_kernel(
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (kRefineThreads / 32);
   const long long n_items = list ? (long long)min(*count, cap) : total;
+  const int nv = d / 8;                                          // d % 64 == 0
   for (long long it = blockIdx.x * (kRefineThreads / 32) + (threadIdx.x >> 5); it < n_items;
        it += warps) {
     long long row;
@@ -504,13 +527,20 @@ __global__ void __launch_bounds__(kRefineThreads) refine_keys_kernel(
       row = it / d;
       col = (int)(it % d);
     }
-    const __nv_bfloat16* x = xv + row * d;
-    const __nv_bfloat16* w = W + (long long)col * d;
-    dfloat acc = {0.0f, 0.0f};
-    for (int l = lane; l < d; l += 32) {
-      const float p = __bfloat162float(x[l]) * __bfloat162float(w[l]);   // exact
-      acc = df_add_f(acc, p);
+    const uint4* x = reinterpret_cast<const uint4*>(xv + row * d);
+    const uint4* w = reinterpret_cast<const uint4*>(W + (long long)col * d);
+    float s0 = 0.0f, c0 = 0.0f, s1 = 0.0f, c1 = 0.0f;
+    for (int l = lane; l < nv; l += 64) {
+      const uint4 xa = x[l], wa = w[l];
+      uint4 xb = make_uint4(0u, 0u, 0u, 0u), wb = xb;
+      if (l + 32 < nv) {
+        xb = x[l + 32];
+        wb = w[l + 32];
+      }
+      sum2_bf16x8(xa, wa, s0, c0);
+      sum2_bf16x8(xb, wb, s1, c1);
     }
+    dfloat acc = df_add(df_two_sum(s0, c0), df_two_sum(s1, c1));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const dfloat t = {__shfl_xor_sync(0xffffffffu, acc.hi, o), __shfl_xor_sync(0xffffffffu, acc.lo, o)};
