@@ -1061,6 +1061,15 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
   static thread_local GemmArgs a;
   a = args;
   a.wait_ns = wait_limit_ns();
+  // L2 prefetch for later kernels: at most half of the 129 MB L2 in all (a
+  // larger range evicts its own first lines before they are read, and its
+  // HBM reads compete with this GEMM's), taken from the front of each range
+  // in order
+  long long pf_left = 64ll << 20;
+  for (int r = 0; r < a.n_prefetch; ++r) {
+    a.pf_bytes[r] = std::min(a.pf_bytes[r], pf_left);
+    pf_left -= a.pf_bytes[r];
+  }
   const GemmPlan plan = plan_gemm_tc(epi, a, max_m, max_n);
   if (plan.region <= 0) return cudaErrorInvalidConfiguration;
   CUtensorMap maps[5];            // F0, F1, F2, R0, R1

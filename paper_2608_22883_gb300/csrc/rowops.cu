@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kLnThreads) ln_rows_kernel(
 // 10^4; the query it feeds moves by ~1e-6 of its scale).  Same loads, depth
 // check and shared-memory depth table as ln_rows_kernel; one CTA per row.
 template <class T>
-__global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
+__global__ void __launch_bounds__(kLnThreads, 2) ln_query_kernel(
     const T* __restrict__ x, int d, const T* __restrict__ gamma, const T* __restrict__ beta,
     float eps, const T* __restrict__ E, const int32_t* __restrict__ depth, int max_depth,
     int e_smem, int* err, T* __restrict__ out) {
@@ -155,13 +155,16 @@ __global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
   const int row = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nvec = d / V;
-  float xv[kLnMaxVec][V], gv[kLnMaxVec][V], bv[kLnMaxVec][V], ev[kLnMaxVec][V];
+  // the row in fp32; gamma, beta and the depth row kept as loaded (16-byte
+  // vectors) and widened in the last pass: two CTAs fit on an SM
+  float xv[kLnMaxVec][V];
+  uint4 gv[kLnMaxVec], bv[kLnMaxVec], ev[kLnMaxVec];
 #pragma unroll
   for (int j = 0; j < kLnMaxVec; ++j) {      // weights: independent of the predecessor
     const int vi = tid + j * kLnThreads;
     if (vi < nvec) {
-      ln_load<T>(gamma + vi * V, gv[j]);
-      ln_load<T>(beta + vi * V, bv[j]);
+      gv[j] = *reinterpret_cast<const uint4*>(gamma + vi * V);
+      bv[j] = *reinterpret_cast<const uint4*>(beta + vi * V);
       if (e_smem)
         for (int r = 0; r <= max_depth; ++r)
           cp_async16(e_s + (long long)r * d + vi * V, E + (long long)r * d + vi * V);
@@ -187,7 +190,7 @@ __global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
 #pragma unroll
   for (int j = 0; j < kLnMaxVec; ++j) {
     const int vi = tid + j * kLnThreads;
-    if (vi < nvec) ln_load<T>(er + vi * V, ev[j]);
+    if (vi < nvec) ev[j] = *reinterpret_cast<const uint4*>(er + vi * V);
   }
   // pass 1: mean
   float s = 0.0f;
@@ -226,9 +229,13 @@ __global__ void __launch_bounds__(kLnThreads) ln_query_kernel(
     const int vi = tid + j * kLnThreads;
     if (vi < nvec) {
       T res[V];
+      float gf[V], bf[V], ef[V];
+      ln_unpack<T>(gv[j], gf);
+      ln_unpack<T>(bv[j], bf);
+      ln_unpack<T>(ev[j], ef);
 #pragma unroll
       for (int i = 0; i < V; ++i) {
-        const float y = fmaf((xv[j][i] - mean) * rstd, gv[j][i], bv[j][i]) + ev[j][i];
+        const float y = fmaf((xv[j][i] - mean) * rstd, gf[i], bf[i]) + ef[i];
         res[i] = from_f32<T>(y);
       }
       *reinterpret_cast<uint4*>(o + vi * V) = *reinterpret_cast<const uint4*>(res);
@@ -243,7 +250,16 @@ cudaError_t launch_ln_query(int dtype, const void* h, int rows, int d, const voi
   constexpr int kESmemMax = 64 * 1024;
   const size_t es = dtype == FOVEA_BF16 ? 2 : 4;
   const size_t e_bytes = (size_t)(max_depth + 1) * d * es;
-  const int e_smem = e_bytes <= (size_t)kESmemMax ? 1 : 0;
+  // the depth table staged in shared memory by every CTA when the rows are
+  // few (it hides the dependent load of the row's depth embedding); for many
+  // rows the CTAs read the one row they need instead
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  const int e_smem = e_bytes <= (size_t)kESmemMax && rows <= 2 * sms ? 1 : 0;
   const size_t smem = e_smem ? e_bytes : 0;
   if (dtype == FOVEA_BF16) {
     using T = __nv_bfloat16;
@@ -625,7 +641,7 @@ cudaError_t launch_refine_keys(const void* xv, const void* W, int d, const KeyFi
 constexpr int kFinThreads = 512;
 
 template <class T>
-__global__ void __launch_bounds__(kFinThreads) finalize_kernel(
+__global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(
     const T* __restrict__ h, const float* __restrict__ c, const T* __restrict__ act, int H, int d,
     const T* __restrict__ w_g2, const T* __restrict__ b_g2, const T* __restrict__ rms_gamma,
     float eps, const __grid_constant__ DepthGate gate_rows, T* __restrict__ h_out,
