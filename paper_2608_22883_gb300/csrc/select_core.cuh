@@ -343,6 +343,86 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
   }
 }
 
+// Ranking of the C (>= K_eff) candidates in sm.cand by (score desc,
+// position asc), which puts the top K_eff in order in sm.sorted; then the
+// cumulative mass, one ordered entry per thread (K_eff <= kRankMax), the
+// count K and the outputs of draft state n.
+template <class Sync>
+__device__ __forceinline__ void select_tail(const SelectArgs& a, int n, int key_off,
+                                            const float* s_sc, int K_eff, int C, float smax,
+                                            float sumexp, SelectSmem& sm, int tid, Sync sync) {
+  const int lane = tid & 31, warp = tid >> 5;
+  const int k_max = a.k_max;
+  // ---- rank the candidates: rank = #larger (keys are distinct) -------------
+  for (int c = tid; c < C; c += kSelThreads) {
+    const unsigned long long me = sm.cand[c];
+    int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+    int j = 0;
+    for (; j + 3 < C; j += 4) {
+      r0 += sm.cand[j] > me;
+      r1 += sm.cand[j + 1] > me;
+      r2 += sm.cand[j + 2] > me;
+      r3 += sm.cand[j + 3] > me;
+    }
+    for (; j < C; ++j) r0 += sm.cand[j] > me;
+    const int r = (r0 + r1) + (r2 + r3);
+    if (r < K_eff) sm.sorted[r] = me;
+  }
+  sync();                                                     // (4)
+  // ---- cumulative mass, one ordered entry per thread -----------------------
+  const int t = tid;
+  float e = 0.0f;
+  int pos = 0;
+  if (t < K_eff) {
+    pos = (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[t] & 0xFFFFFFFFull));
+    e = expf(s_sc[pos] - smax);
+  }
+  float incl = e;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float u = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += u;
+  }
+  if (lane == 31) sm.warp_tot_f[warp] = incl;
+  sync();                                                     // (5)
+  float before = 0.0f;
+  for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
+  const float cum = before + incl;
+  if (t < K_eff) sm.cum[t] = cum;
+  {
+    const unsigned int bal = __ballot_sync(0xffffffffu, t < K_eff && cum / sumexp >= a.rho);
+    if (lane == 0) sm.warp_first[warp] = bal ? warp * 32 + __ffs(bal) - 1 : K_eff;
+  }
+  sync();                                                     // (6)
+  int first = K_eff;
+  for (int w = 0; w < kSelWarps; ++w) first = min(first, sm.warp_first[w]);
+  const int K = first < K_eff ? min(K_eff, max(a.k_min, first + 1)) : K_eff;
+  const float denom = sm.cum[K - 1];                          // sum over I_n of exp(s - s_max)
+  const long long out_row = (long long)n * k_max;
+  for (int u = tid; u < k_max; u += kSelThreads) {
+    if (u < K) {
+      const int pu = u == t ? pos : (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[u] & 0xFFFFFFFFull));
+      const float eu = u == t ? e : expf(s_sc[pu] - smax);
+      const int row = key_off + pu;
+      if (a.sel_pos) a.sel_pos[out_row + u] = row;
+      if (a.sel_w) a.sel_w[out_row + u] = eu / denom;
+      put_alpha(a, n, pu, eu / denom);
+      if (a.loc_pos) {
+        a.loc_pos[u] = row;
+        a.loc_w[u] = eu / denom;
+      }
+      if (a.indices) a.indices[out_row + u] = a.orig_index[row];
+    } else if (a.indices) {
+      a.indices[out_row + u] = -1;
+    }
+  }
+  if (tid == 0) {
+    if (a.sel_cnt) a.sel_cnt[n] = K;
+    if (a.loc_cnt) *a.loc_cnt = K;
+    if (a.counts) a.counts[n] = K;
+  }
+}
+
 // Fast path for rows of at most kFastMaxM entries and K_eff <= kRankMax,
 // with six group barriers and short dependency chains between them: the
 // threads keep their scores in registers; (1) the maximum and the minimum
@@ -474,86 +554,127 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
   sync();                                                     // (3)
   const int C = sm.sh_cnt_gt;
   if (C > kFastMaxCand) return false;                         // uniform
-  // ---- rank the candidates: rank = #larger (keys are distinct) -------------
-  for (int c = tid; c < C; c += kSelThreads) {
-    const unsigned long long me = sm.cand[c];
-    int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
-    int j = 0;
-    for (; j + 3 < C; j += 4) {
-      r0 += sm.cand[j] > me;
-      r1 += sm.cand[j + 1] > me;
-      r2 += sm.cand[j + 2] > me;
-      r3 += sm.cand[j + 3] > me;
-    }
-    for (; j < C; ++j) r0 += sm.cand[j] > me;
-    const int r = (r0 + r1) + (r2 + r3);
-    if (r < K_eff) sm.sorted[r] = me;
+  select_tail(a, n, key_off, s_sc, K_eff, C, smax, sumexp, sm, tid, sync);
+  return true;
+}
+
+// Wide path: the fast path's steps for rows of more than kFastMaxM entries
+// (K_eff <= kRankMax), the scores read from shared memory in strided passes
+// instead of registers and the distance to the maximum binned into kWideBins
+// bins (the histogram occupies sm.cum, which the mass scan only writes after
+// it is dead): (1) maximum and minimum; (2) softmax denominator (each
+// thread's terms in index order, then a fixed tree) and histogram; (3, 4) the
+// bin b* holding the K_eff-th largest score by a block scan of the bins;
+// (5) the entries of bins <= b* gathered as candidates.  Returns false,
+// having written nothing, when they exceed kFastMaxCand.
+constexpr int kWideBins = 1024;
+static_assert(kWideBins <= FOVEA_MAX_K, "the histogram lives in SelectSmem::cum");
+static_assert(kWideBins == 4 * kSelThreads, "four bins per thread in the scan");
+
+template <class Sync>
+__device__ bool select_wide(const SelectArgs& a, int n, int M, int key_off, const float* s_sc,
+                            SelectSmem& sm, int tid, Sync sync) {
+  const int lane = tid & 31, warp = tid >> 5;
+  const int K_eff = min(a.k_max, M);
+  unsigned int* hist = reinterpret_cast<unsigned int*>(sm.cum);
+  float lmax = -INFINITY, lmin = INFINITY;
+  for (int i = tid; i < M; i += kSelThreads) {
+    const float v = s_sc[i];
+    lmax = fmaxf(lmax, v);
+    lmin = fminf(lmin, v);
   }
-  sync();                                                     // (4)
-  // ---- cumulative mass, one ordered entry per thread -----------------------
-  const int t = tid;
-  float e = 0.0f;
-  int pos = 0;
-  if (t < K_eff) {
-    pos = (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[t] & 0xFFFFFFFFull));
-    e = expf(s_sc[pos] - smax);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, o));
+    lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, o));
   }
-  float incl = e;
+  for (int i = tid; i < kWideBins; i += kSelThreads) hist[i] = 0u;
+  if (lane == 0) {
+    sm.red_m[warp] = lmax;
+    sm.red_lo[warp] = lmin;
+  }
+  if (tid == 0) sm.sh_cnt_gt = 0;
+  sync();                                                     // (1)
+  float smax = sm.red_m[0], smin = sm.red_lo[0];
+#pragma unroll
+  for (int w = 1; w < kSelWarps; ++w) {
+    smax = fmaxf(smax, sm.red_m[w]);
+    smin = fminf(smin, sm.red_lo[w]);
+  }
+  const float range = smax - smin;
+  const float inv_w = range > 0.0f ? (float)(kWideBins - 1) / range : 0.0f;
+  auto bin_of = [&](float v) {
+    const int b = (int)((smax - v) * inv_w);
+    return b < 0 ? 0 : (b > kWideBins - 1 ? kWideBins - 1 : b);
+  };
+  float lsum = 0.0f;
+  for (int i = tid; i < M; i += kSelThreads) {
+    const float v = s_sc[i];
+    lsum += expf(v - smax);
+    atomicAdd(&hist[bin_of(v)], 1u);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+  if (lane == 0) sm.red_s[warp] = lsum;
+  sync();                                                     // (2)
+  float sumexp = sm.red_s[0];
+#pragma unroll
+  for (int w = 1; w < kSelWarps; ++w) sumexp += sm.red_s[w];
+  // thread tid owns bins 4 tid .. 4 tid + 3 (ascending distance)
+  unsigned int cnt[4], tot = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    cnt[j] = hist[4 * tid + j];
+    tot += cnt[j];
+  }
+  unsigned int incl = tot;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const float u = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += u;
+    const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
   }
-  if (lane == 31) sm.warp_tot_f[warp] = incl;
-  sync();                                                     // (5)
-  float before = 0.0f;
-  for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
-  const float cum = before + incl;
-  if (t < K_eff) sm.cum[t] = cum;
-  {
-    const unsigned int bal = __ballot_sync(0xffffffffu, t < K_eff && cum / sumexp >= a.rho);
-    if (lane == 0) sm.warp_first[warp] = bal ? warp * 32 + __ffs(bal) - 1 : K_eff;
-  }
-  sync();                                                     // (6)
-  int first = K_eff;
-  for (int w = 0; w < kSelWarps; ++w) first = min(first, sm.warp_first[w]);
-  const int K = first < K_eff ? min(K_eff, max(a.k_min, first + 1)) : K_eff;
-  const float denom = sm.cum[K - 1];                          // sum over I_n of exp(s - s_max)
-  const long long out_row = (long long)n * k_max;
-  for (int u = tid; u < k_max; u += kSelThreads) {
-    if (u < K) {
-      const int pu = u == t ? pos : (int)(0xFFFFFFFFu - (uint32_t)(sm.sorted[u] & 0xFFFFFFFFull));
-      const float eu = u == t ? e : expf(s_sc[pu] - smax);
-      const int row = key_off + pu;
-      if (a.sel_pos) a.sel_pos[out_row + u] = row;
-      if (a.sel_w) a.sel_w[out_row + u] = eu / denom;
-      put_alpha(a, n, pu, eu / denom);
-      if (a.loc_pos) {
-        a.loc_pos[u] = row;
-        a.loc_w[u] = eu / denom;
-      }
-      if (a.indices) a.indices[out_row + u] = a.orig_index[row];
-    } else if (a.indices) {
-      a.indices[out_row + u] = -1;
+  if (lane == 31) sm.warp_tot[warp] = (int)incl;
+  sync();                                                     // (3)
+  unsigned int run = incl - tot;
+  for (int w = 0; w < warp; ++w) run += (unsigned int)sm.warp_tot[w];
+  if (run < (unsigned)K_eff && run + tot >= (unsigned)K_eff) {   // exactly one thread
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (run < (unsigned)K_eff && run + cnt[j] >= (unsigned)K_eff) sm.sh_digit = 4 * tid + j;
+      run += cnt[j];
     }
   }
-  if (tid == 0) {
-    if (a.sel_cnt) a.sel_cnt[n] = K;
-    if (a.loc_cnt) *a.loc_cnt = K;
-    if (a.counts) a.counts[n] = K;
+  sync();                                                     // (4)
+  const int bstar = (int)sm.sh_digit;
+  for (int base = 0; base < M; base += kSelThreads) {
+    const int i = base + tid;
+    float v = 0.0f;
+    const bool take = i < M && bin_of(v = s_sc[i]) <= bstar;
+    const unsigned int bal = __ballot_sync(0xffffffffu, take);
+    int slot = 0;
+    if (lane == 0 && bal) slot = atomicAdd(&sm.sh_cnt_gt, __popc(bal));
+    slot = __shfl_sync(0xffffffffu, slot, 0) + __popc(bal & ((1u << lane) - 1u));
+    if (take && slot < kFastMaxCand)
+      sm.cand[slot] = ((unsigned long long)ord_key(v) << 32) | (0xFFFFFFFFu - (uint32_t)i);
   }
+  sync();                                                     // (5)
+  const int C = sm.sh_cnt_gt;
+  if (C > kFastMaxCand) return false;                         // uniform
+  select_tail(a, n, key_off, s_sc, K_eff, C, smax, sumexp, sm, tid, sync);
   return true;
 }
 
 // Selection of draft state n from its staged scores (s_sc, M >= 1 entries,
-// staged and visible to the group): the fast path where it applies, else the
-// radix path.
+// staged and visible to the group): the fast or wide path where it applies,
+// else the radix path.
 template <class Sync>
 __device__ __forceinline__ void select_row(const SelectArgs& a, int n, int M, int key_off,
                                            const float* s_sc, SelectSmem& sm, int tid, Sync sync) {
-  if (M <= kFastMaxM && min(a.k_max, M) <= kRankMax &&
-      select_fast(a, n, M, key_off, s_sc, sm, tid, sync))
-    return;
+  if (min(a.k_max, M) <= kRankMax) {
+    if (M <= kFastMaxM ? select_fast(a, n, M, key_off, s_sc, sm, tid, sync)
+                       : select_wide(a, n, M, key_off, s_sc, sm, tid, sync))
+      return;
+  }
   float lmax = -INFINITY, lsum = 0.0f;
   for (int i = tid; i < M; i += kSelThreads) combine_ms(lmax, lsum, s_sc[i], 1.0f);
   float smax, sumexp;
