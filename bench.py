@@ -90,9 +90,15 @@ def step_cost(w: workloads.Workload, counts: np.ndarray, indices: np.ndarray, pr
     return float(nbytes), float(flops), int(uniq)
 
 
-def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: bool) -> float:
-    """HBM bytes one launch of a kernel must move (reads + writes)."""
+def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: bool,
+                 dense: bool = False) -> float:
+    """HBM bytes one launch of a kernel must move (reads + writes).  `dense`:
+    the step runs the dense-weights path (the selection writes the weights
+    alpha as a bf16 hi / lo pair [N, P], P the longest memory rounded up to
+    64, and the activation GEMM reads them with the transposed projected
+    values [B, 2H, P])."""
     d, H, N = w.d, w.params["b_f1"].shape[0], w.N
+    P = (max(int(m) for m in w.m_sizes) + 63) // 64 * 64
     es = 2 if w.dtype == "bf16" else 4
     scores = sum(int(w.row_offsets[b + 1] - w.row_offsets[b]) * int(w.m_sizes[b]) for b in range(w.B)) * 4
     if name == "query_proj":
@@ -119,7 +125,9 @@ def kernel_bytes(name: str, w: workloads.Workload, uniq_values: int, projected: 
     if name == "select_readout":
         return scores + uniq_values * d * es + N * d * (4 + es) + N * 4 + N * w.k_max * 4
     if name == "select":
-        return scores + 3 * N * w.k_max * 4
+        return scores + 3 * N * w.k_max * 4 + (N * P * 2 * es if dense else 0)
+    if name == "act_gemm":        # alpha (hi, lo), transposed projected values, G_h, biases in; activations out
+        return es * (2 * N * P + w.B * 2 * H * P + 2 * H + N * 2 * H) + 4 * N * 2 * H
     if name == "ln_query":
         return es * (2 * N * d + 4 * d)
     if name == "finalize":
@@ -519,7 +527,8 @@ def main():
 
     # ---- roofline ----
     c_np, i_np = counts.cpu().numpy(), indices.cpu().numpy()
-    projected = "select_fuse" in per_kernel
+    dense = "act_gemm" in per_kernel
+    projected = "select_fuse" in per_kernel or dense
     folded = "score_folded" in per_kernel or "score_fusion_h" in per_kernel
     # the method's algorithmic bytes (full fusion weights, value rows), and
     # what this path's step moves (projected values: the h-half weights and
@@ -533,7 +542,7 @@ def main():
     t_roof_path = max(nbytes_path / (peaks["hbm_gbs"] * 1e9), flops_path / (peaks["bf16_tflops"] * 1e12))
     kern = {name: {"ms_avg": tot / max(n, 1), "launches": n} for name, (tot, n) in per_kernel.items()}
     dom = max(kern, key=lambda k: kern[k]["ms_avg"] * kern[k]["launches"])
-    dom_bytes = kernel_bytes(dom, w, uniq, projected)
+    dom_bytes = kernel_bytes(dom, w, uniq, projected, dense)
     achieved = dom_bytes / (kern[dom]["ms_avg"] / 1000.0) / 1e9
     launches_per_step = sum(k["launches"] for k in kern.values()) / max(n_kt, 1)
     launches = int(round(launches_per_step * args.steps))
@@ -575,8 +584,8 @@ def main():
                                         "folded_keys": folded},
                           "peaks": f"{peak_src}: {peaks['hbm_gbs']} GB/s, {peaks['bf16_tflops']} TF/s"},
         "kernels": {k: {"us_avg": 1000 * v["ms_avg"], "launches": v["launches"],
-                        "algorithmic_bytes": kernel_bytes(k, w, uniq, projected),
-                        "gbs": kernel_bytes(k, w, uniq, projected) / (v["ms_avg"] / 1000.0) / 1e9}
+                        "algorithmic_bytes": kernel_bytes(k, w, uniq, projected, dense),
+                        "gbs": kernel_bytes(k, w, uniq, projected, dense) / (v["ms_avg"] / 1000.0) / 1e9}
                     for k, v in kern.items()},
         "ms_per_step_graph_replay": graph_ms,
         "ms_per_step_kernel_timing_pass": ms_hooks,

@@ -67,3 +67,24 @@ def test_kernel_bytes_of_the_folded_launches(w7b):
     # x_h in the one, h in the other
     assert bench.kernel_bytes("score_folded", w7b, 0, True) + bench.kernel_bytes("fusion_h", w7b, 0, True) \
         == merged
+
+
+def test_kernel_bytes_of_the_dense_weights_launches():
+    """Long-memory shape (4 images of 8192 entries, 512 rows, 2H = 1024):
+    the selection writes the weights as a bf16 hi / lo pair [512, 8192]
+    (16.8 MB), and the activation GEMM reads them with the transposed
+    projected values [4, 1024, 8192] (67.1 MB) and G_h, writing the
+    activations."""
+    w = workloads.WORKLOADS[5]
+    class W:                                     # the shape alone; no inputs drawn
+        d, N, B, k_max = w.d, w.N, w.B, w.k_max
+        m_sizes = [8192] * 4
+        row_offsets = [0, 128, 256, 384, 512]
+        dtype = "bf16"
+        params = {"b_f1": np.zeros(512)}
+    alpha = 512 * 8192 * 2 * 2
+    projT = 4 * 1024 * 8192 * 2
+    assert bench.kernel_bytes("select", W, 0, True, True) - bench.kernel_bytes("select", W, 0, True) == alpha
+    act = bench.kernel_bytes("act_gemm", W, 0, True, True)
+    assert act == alpha + projT + 2 * 1024 + 512 * 1024 * 2 + 512 * 1024 * 4
+    assert abs(act / 1e6 - 87.0) < 0.1         # 16.8 + 67.1 + 1.0 (act out) + 2.1 (G_h in)
