@@ -10,10 +10,17 @@
 
 namespace fovea {
 
-struct BlockSync {
+// The CTA barrier; kLarge: the caller may pass caps above kRankMax (the
+// large-cap ordering is compiled in only then, so the kernel for small caps
+// keeps its short code).
+template <bool kLargeCaps>
+struct BlockSyncT {
+  static constexpr bool kLarge = kLargeCaps;
   __device__ __forceinline__ void operator()() const { __syncthreads(); }
 };
+using BlockSync = BlockSyncT<false>;
 
+template <bool kLargeCaps>
 __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectArgs a,
                                                              const __grid_constant__ SeqTable tab) {
   extern __shared__ float s_sc[];                            // [M] scores of this row
@@ -36,7 +43,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     s_sc[i] = v;
   }
   __syncthreads();
-  select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSync{});
+  select_row(a, n, M, tab.key_off[b], s_sc, sm, tid, BlockSyncT<kLargeCaps>{});
 }
 
 cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const int32_t* orig_index,
@@ -48,16 +55,20 @@ cudaError_t launch_select(const float* scores, const SeqTable& tab, int N, const
   const size_t smem = (size_t)max(max_m, 1) * sizeof(float);
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         FOVEA_MAX_ENTRIES * (int)sizeof(float));
-    if (e != cudaSuccess) return e;
+    for (auto k : {(const void*)select_kernel<false>, (const void*)select_kernel<true>}) {
+      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           FOVEA_MAX_ENTRIES * (int)sizeof(float));
+      if (e != cudaSuccess) return e;
+    }
     configured = true;
   }
   SelectArgs a{scores, orig_index, rho, k_min, k_max, counts, indices, sel_pos, sel_w, sel_cnt,
                nullptr, nullptr, nullptr, gate,
                static_cast<__nv_bfloat16*>(alpha_hi), static_cast<__nv_bfloat16*>(alpha_lo),
                alpha_ld};
-  return launch_pdl(select_kernel, dim3(N), dim3(kSelThreads), smem, s, a, tab);
+  if (k_max > kRankMax)
+    return launch_pdl(select_kernel<true>, dim3(N), dim3(kSelThreads), smem, s, a, tab);
+  return launch_pdl(select_kernel<false>, dim3(N), dim3(kSelThreads), smem, s, a, tab);
 }
 
 // Selection and the gathers that consume it, in one kernel: one
@@ -246,6 +257,7 @@ __device__ __forceinline__ void gather_rows_smem(const T* X, long long ld, int c
 // The selection group: the first kSelThreads threads of the CTA, synchronised
 // with a named barrier when the CTA is larger.
 struct SelGroupSync {
+  static constexpr bool kLarge = false;   // the gather kernel takes caps <= kRankMax
   __device__ __forceinline__ void operator()() const {
     asm volatile("bar.sync 1, %0;" ::"n"(kSelThreads) : "memory");
   }

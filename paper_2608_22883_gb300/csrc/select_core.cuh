@@ -6,15 +6,17 @@
 // I_n = pi_n(1..K)).
 //
 // The caller stages the row's scores in shared memory (-0 mapped to +0) and
-// calls select_row.  Rows of up to 2048 entries take a fast path with few
-// group barriers (select_fast, below).  Otherwise select_stats combines the
-// threads' softmax statistics and select_finish does the rest: a 4-pass 8-bit radix
-// select finds the K_eff-th largest score key (K_eff = min(K_max, |V|))
-// without sorting the row; only the K_eff candidates are put in order, by
+// calls select_row.  A histogram of the distance to the maximum finds the
+// bin holding the K_eff-th largest score (K_eff = min(K_max, |V|)) without
+// sorting the row: in registers for rows of up to 2048 entries (select_fast),
+// in strided passes over shared memory above that (select_wide).  The entries
+// of the bins up to it are the candidates; only they are put in order, by
 // (score desc, position asc): each candidate's rank is its count of larger
-// candidates for K_eff <= 256, a bitonic network above that.  An fp32
-// inclusive scan of exp(s - s_max) over them gives the cumulative mass, and
-// the first prefix reaching rho sets K.
+// candidates for up to 256 candidates, a bucket order above that.  An fp32
+// inclusive scan of exp(s - s_max) over the first K_eff gives the cumulative
+// mass, and the first prefix reaching rho sets K.  More than 1024 candidates
+// (many equal scores) take a 4-pass 8-bit radix select of the K_eff-th key
+// instead (select_finish).
 //
 // Used by the standalone select kernel (a CTA of 256 threads, __syncthreads)
 // and by the selection + gather kernel (its first 256 threads, a named
@@ -82,13 +84,14 @@ __device__ __forceinline__ void clear_alpha(const SelectArgs& a, int n, int tid,
 
 struct SelectSmem {
   unsigned long long cand[FOVEA_MAX_K];      // (key << 32) | ~position
-  unsigned long long sorted[kRankMax];
+  unsigned long long sorted[FOVEA_MAX_K];     // ordered keys; scratch of bucket_order
   float cum[FOVEA_MAX_K];                    // inclusive scan of exp(s - s_max)
   unsigned int hist[256];
   float red_m[kSelWarps], red_s[kSelWarps], red_lo[kSelWarps];
   float warp_tot_f[kSelWarps];
   int warp_tot[kSelWarps];
   int warp_first[kSelWarps];
+  unsigned int red_u[2][kSelWarps];
   unsigned int sh_digit, sh_above;
   int sh_cnt_gt, sh_first;
   float sh_max, sh_sum;
@@ -132,6 +135,88 @@ __device__ __forceinline__ void select_stats(float lmax, float lsum, SelectSmem&
   sumexp = sm.sh_sum;
 }
 
+// Orders the C (<= FOVEA_MAX_K) distinct keys of sm.cand descending, in
+// place: a histogram of the keys' score words over kWideBins bins (the bin is
+// monotone in the key), an exclusive scan of the bins, a scatter of the keys
+// into bin order (sm.sorted), and each key's rank among the keys of its own
+// bin.  The histogram lives in sm.cum (dead until the mass scan).
+constexpr int kOrderBins = 1024;
+static_assert(kOrderBins <= FOVEA_MAX_K && kOrderBins == 4 * kSelThreads, "bins in SelectSmem::cum");
+
+template <class Sync>
+__device__ void bucket_order(SelectSmem& sm, int C, int tid, Sync sync) {
+  const int lane = tid & 31, warp = tid >> 5;
+  unsigned int* hist = reinterpret_cast<unsigned int*>(sm.cum);
+  uint32_t kmax = 0u, kmin = 0xFFFFFFFFu;
+  for (int c = tid; c < C; c += kSelThreads) {
+    const uint32_t k = (uint32_t)(sm.cand[c] >> 32);
+    kmax = max(kmax, k);
+    kmin = min(kmin, k);
+  }
+  kmax = __reduce_max_sync(0xffffffffu, kmax);
+  kmin = __reduce_min_sync(0xffffffffu, kmin);
+  for (int i = tid; i < kOrderBins; i += kSelThreads) hist[i] = 0u;
+  if (lane == 0) {
+    sm.red_u[0][warp] = kmax;
+    sm.red_u[1][warp] = kmin;
+  }
+  sync();
+#pragma unroll
+  for (int w = 0; w < kSelWarps; ++w) {
+    kmax = max(kmax, sm.red_u[0][w]);
+    kmin = min(kmin, sm.red_u[1][w]);
+  }
+  const unsigned long long span = (unsigned long long)(kmax - kmin) + 1ull;
+  auto bin_of = [&](unsigned long long key) {
+    return (int)(((unsigned long long)(kmax - (uint32_t)(key >> 32)) * kOrderBins) / span);
+  };
+  for (int c = tid; c < C; c += kSelThreads) atomicAdd(&hist[bin_of(sm.cand[c])], 1u);
+  sync();
+  // exclusive scan of the bins: thread tid owns bins 4 tid .. 4 tid + 3
+  unsigned int cnt[4], tot = 0u;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    cnt[j] = hist[4 * tid + j];
+    tot += cnt[j];
+  }
+  unsigned int incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) sm.red_u[0][warp] = incl;
+  sync();
+  unsigned int run = incl - tot;
+  for (int w = 0; w < warp; ++w) run += sm.red_u[0][w];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    hist[4 * tid + j] = run;                       // start of the bin
+    run += cnt[j];
+  }
+  sync();
+  for (int c = tid; c < C; c += kSelThreads) {
+    const unsigned long long key = sm.cand[c];
+    sm.sorted[atomicAdd(&hist[bin_of(key)], 1u)] = key;
+  }
+  sync();
+  // hist[b] is now the end of bin b, and the start of bin b + 1
+  for (int i = tid; i < C; i += kSelThreads) {
+    const unsigned long long me = sm.sorted[i];
+    const int b = bin_of(me);
+    const int beg = b ? (int)hist[b - 1] : 0, end = (int)hist[b];
+    int r = beg;
+    for (int j = beg; j < end; ++j) r += sm.sorted[j] > me;
+    sm.cand[r] = me;
+  }
+  sync();
+}
+
+template <class Sync>
+__device__ __forceinline__ void select_tail(const SelectArgs& a, int n, int key_off,
+                                            const float* s_sc, int K_eff, int C, float smax,
+                                            float sumexp, SelectSmem& sm, int tid, Sync sync);
+
 // Radix select, candidate ordering, mass scan and the outputs of draft state
 // n, whose M (>= 1) scores are staged in s_sc.  key_off is the compacted row
 // of the sequence's first memory entry.
@@ -139,9 +224,7 @@ template <class Sync>
 __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, const float* s_sc,
                               float smax, float sumexp, SelectSmem& sm, int tid, Sync sync) {
   const int lane = tid & 31, warp = tid >> 5;
-  const int k_max = a.k_max;
-  const long long out_row = (long long)n * k_max;
-  const int K_eff = min(k_max, M);
+  const int K_eff = min(a.k_max, M);
 
   // ---- radix select of the K_eff-th largest key ----------------------------
   // (every entry selected, the dense setting: no threshold to find; every
@@ -245,95 +328,91 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
   }
   sync();
 
-  // ---- order the candidates, descending ------------------------------------
-  const unsigned long long* ordered;
-  if (K_eff <= kRankMax) {
-    // keys are distinct (the position is part of the key): rank = #larger
-    for (int c = tid; c < K_eff; c += kSelThreads) {
-      const unsigned long long me = sm.cand[c];
-      int r = 0;
-      for (int j = 0; j < K_eff; ++j) r += sm.cand[j] > me;
-      sm.sorted[r] = me;
-    }
-    ordered = sm.sorted;
-  } else {
-    int P = 1;
-    while (P < K_eff) P <<= 1;
-    for (int t = K_eff + tid; t < P; t += kSelThreads) sm.cand[t] = 0ull;
-    sync();
-    for (int k = 2; k <= P; k <<= 1) {
-      for (int j = k >> 1; j > 0; j >>= 1) {
-        for (int i = tid; i < P; i += kSelThreads) {
-          const int ixj = i ^ j;
-          if (ixj > i) {
-            const unsigned long long x = sm.cand[i], y = sm.cand[ixj];
-            const bool desc = (i & k) == 0;
-            if (desc ? (x < y) : (x > y)) {
-              sm.cand[i] = y;
-              sm.cand[ixj] = x;
-            }
-          }
-        }
-        sync();
-      }
-    }
-    ordered = sm.cand;
-  }
-  sync();
+  select_tail(a, n, key_off, s_sc, K_eff, K_eff, smax, sumexp, sm, tid, sync);
+}
 
-  // ---- cumulative mass over the ordered candidates -------------------------
-  // thread tid scans the contiguous quad 4 tid .. 4 tid + 3 (4 x 256 >= FOVEA_MAX_K)
-  {
-    float e[4];
-    float run = 0.0f;
+// select_tail for K_eff > kRankMax: the C (K_eff <= C <= FOVEA_MAX_K)
+// candidates bucket-ordered, the cumulative mass over the first K_eff four
+// contiguous entries per thread, and the outputs, the original indices of a
+// thread's outputs requested together before any is written.
+template <class Sync>
+__device__ __forceinline__ void select_tail_large(const SelectArgs& a, int n, int key_off,
+                                                   const float* s_sc, int K_eff, int C, float smax,
+                                                   float sumexp, SelectSmem& sm, int tid, Sync sync) {
+  static_assert(FOVEA_MAX_K <= 4 * kSelThreads, "four ordered entries per thread");
+  const int lane = tid & 31, warp = tid >> 5;
+  const int k_max = a.k_max;
+  bucket_order(sm, C, tid, sync);           // ends with a barrier
+  const unsigned long long* ordered = sm.cand;
+  // ---- cumulative mass: thread tid holds ordered entries 4 tid .. 4 tid + 3
+  constexpr int per = 4;
+  float e[4];
+  float run = 0.0f;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int t = 4 * tid + q;
-      e[q] = t < K_eff ? expf(s_sc[0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull)] - smax)
-                       : 0.0f;
-      run += e[q];
-    }
-    float incl = run;
+  for (int q = 0; q < 4; ++q) {
+    const int t = per * tid + q;
+    e[q] = q < per && t < K_eff
+               ? expf(s_sc[0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull)] - smax)
+               : 0.0f;
+    run += e[q];
+  }
+  float incl = run;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float t = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += t;
-    }
-    if (lane == 31) sm.warp_tot_f[warp] = incl;
-    sync();
-    float before = incl - run;
-    for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
+  for (int o = 1; o < 32; o <<= 1) {
+    const float u = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += u;
+  }
+  if (lane == 31) sm.warp_tot_f[warp] = incl;
+  sync();
+  float before = incl - run;
+  for (int w = 0; w < warp; ++w) before += sm.warp_tot_f[w];
+  int my_first = K_eff;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int t = 4 * tid + q;
-      before += e[q];
-      if (t < K_eff) sm.cum[t] = before;
+  for (int q = 0; q < 4; ++q) {
+    const int t = per * tid + q;
+    before += e[q];
+    if (q < per && t < K_eff) {
+      sm.cum[t] = before;
+      if (my_first == K_eff && before / sumexp >= a.rho) my_first = t;
     }
   }
-  if (tid == 0) sm.sh_first = K_eff;       // K_eff = "not reached within the candidates"
+  my_first = __reduce_min_sync(0xffffffffu, my_first);
+  if (lane == 0) sm.warp_first[warp] = my_first;
   sync();
-  for (int t = tid; t < K_eff; t += kSelThreads)
-    if (sm.cum[t] / sumexp >= a.rho) atomicMin(&sm.sh_first, t);
-  sync();
-  const int first = sm.sh_first;
+  int first = K_eff;
+  for (int w = 0; w < kSelWarps; ++w) first = min(first, sm.warp_first[w]);
   const int K = first < K_eff ? min(K_eff, max(a.k_min, first + 1)) : K_eff;
-  const float denom = sm.cum[K - 1];       // sum over I_n of exp(s - s_max)
-
-  for (int t = tid; t < k_max; t += kSelThreads) {
-    if (t < K) {
-      const int pos = (int)(0xFFFFFFFFu - (uint32_t)(ordered[t] & 0xFFFFFFFFull));
-      const float e = expf(s_sc[pos] - smax);
-      const int row = key_off + pos;
-      if (a.sel_pos) a.sel_pos[out_row + t] = row;
-      if (a.sel_w) a.sel_w[out_row + t] = e / denom;
-      put_alpha(a, n, pos, e / denom);
+  const float denom = sm.cum[K - 1];                          // sum over I_n of exp(s - s_max)
+  const long long out_row = (long long)n * k_max;
+  int pu[4], oi[4];
+  float wu[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int u = tid + j * kSelThreads;
+    pu[j] = 0;
+    oi[j] = -1;
+    wu[j] = 0.0f;
+    if (u < K) {
+      pu[j] = (int)(0xFFFFFFFFu - (uint32_t)(ordered[u] & 0xFFFFFFFFull));
+      wu[j] = expf(s_sc[pu[j]] - smax) / denom;
+      if (a.indices) oi[j] = a.orig_index[key_off + pu[j]];
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int u = tid + j * kSelThreads;
+    if (u < K) {
+      const int row = key_off + pu[j];
+      if (a.sel_pos) a.sel_pos[out_row + u] = row;
+      if (a.sel_w) a.sel_w[out_row + u] = wu[j];
+      put_alpha(a, n, pu[j], wu[j]);
       if (a.loc_pos) {
-        a.loc_pos[t] = row;
-        a.loc_w[t] = e / denom;
+        a.loc_pos[u] = row;
+        a.loc_w[u] = wu[j];
       }
-      if (a.indices) a.indices[out_row + t] = a.orig_index[row];
-    } else if (a.indices) {
-      a.indices[out_row + t] = -1;
+      if (a.indices) a.indices[out_row + u] = oi[j];
+    } else if (u < k_max && a.indices) {
+      a.indices[out_row + u] = -1;
     }
   }
   if (tid == 0) {
@@ -343,7 +422,7 @@ __device__ void select_finish(const SelectArgs& a, int n, int M, int key_off, co
   }
 }
 
-// Ranking of the C (>= K_eff) candidates in sm.cand by (score desc,
+// K_eff <= kRankMax: ranking of the C (>= K_eff) candidates in sm.cand by (score desc,
 // position asc), which puts the top K_eff in order in sm.sorted; then the
 // cumulative mass, one ordered entry per thread (K_eff <= kRankMax), the
 // count K and the outputs of draft state n.
@@ -351,6 +430,12 @@ template <class Sync>
 __device__ __forceinline__ void select_tail(const SelectArgs& a, int n, int key_off,
                                             const float* s_sc, int K_eff, int C, float smax,
                                             float sumexp, SelectSmem& sm, int tid, Sync sync) {
+  if constexpr (Sync::kLarge) {               // otherwise the launcher keeps K_max <= kRankMax
+    if (K_eff > kRankMax) {
+      select_tail_large(a, n, key_off, s_sc, K_eff, C, smax, sumexp, sm, tid, sync);
+      return;
+    }
+  }
   const int lane = tid & 31, warp = tid >> 5;
   const int k_max = a.k_max;
   // ---- rank the candidates: rank = #larger (keys are distinct) -------------
@@ -423,7 +508,7 @@ __device__ __forceinline__ void select_tail(const SelectArgs& a, int n, int key_
   }
 }
 
-// Fast path for rows of at most kFastMaxM entries and K_eff <= kRankMax,
+// Fast path for rows of at most kFastMaxM entries (any K_eff <= FOVEA_MAX_K),
 // with six group barriers and short dependency chains between them: the
 // threads keep their scores in registers; (1) the maximum and the minimum
 // score; (2) the softmax denominator (independent exponentials, summed in a
@@ -431,9 +516,8 @@ __device__ __forceinline__ void select_tail(const SelectArgs& a, int n, int key_
 // which gives the bin b* holding the K_eff-th largest score (the bin index is
 // monotone in the score, so the top K_eff entries all lie in bins <= b*);
 // (3) the entries of bins <= b* are gathered (one shared-memory atomic per
-// warp) and (4) ranked among themselves by (score desc, position asc), which
-// puts the top K_eff in order; (5, 6) the mass scan runs one ordered entry
-// per thread.  Returns false, having written nothing, when the candidates
+// warp) and ordered among themselves by (score desc, position asc), which
+// puts the top K_eff in order; the mass scan follows (select_tail).  Returns false, having written nothing, when the candidates
 // exceed kFastMaxCand; the caller then runs the radix path.
 constexpr int kFastMaxM = 2048;                   // 8 scores per thread
 constexpr int kFastMaxCand = FOVEA_MAX_K;         // candidates ranked directly
@@ -558,8 +642,7 @@ __device__ bool select_fast(const SelectArgs& a, int n, int M, int key_off, cons
   return true;
 }
 
-// Wide path: the fast path's steps for rows of more than kFastMaxM entries
-// (K_eff <= kRankMax), the scores read from shared memory in strided passes
+// Wide path: the fast path's steps for rows of more than kFastMaxM entries, the scores read from shared memory in strided passes
 // instead of registers and the distance to the maximum binned into kWideBins
 // bins (the histogram occupies sm.cum, which the mass scan only writes after
 // it is dead): (1) maximum and minimum; (2) softmax denominator (each
@@ -670,11 +753,9 @@ __device__ bool select_wide(const SelectArgs& a, int n, int M, int key_off, cons
 template <class Sync>
 __device__ __forceinline__ void select_row(const SelectArgs& a, int n, int M, int key_off,
                                            const float* s_sc, SelectSmem& sm, int tid, Sync sync) {
-  if (min(a.k_max, M) <= kRankMax) {
-    if (M <= kFastMaxM ? select_fast(a, n, M, key_off, s_sc, sm, tid, sync)
-                       : select_wide(a, n, M, key_off, s_sc, sm, tid, sync))
-      return;
-  }
+  if (M <= kFastMaxM ? select_fast(a, n, M, key_off, s_sc, sm, tid, sync)
+                     : select_wide(a, n, M, key_off, s_sc, sm, tid, sync))
+    return;
   float lmax = -INFINITY, lsum = 0.0f;
   for (int i = tid; i < M; i += kSelThreads) combine_ms(lmax, lsum, s_sc[i], 1.0f);
   float smax, sumexp;
