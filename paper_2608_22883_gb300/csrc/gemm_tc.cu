@@ -977,10 +977,11 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
     const int sb = C::stage_bytes(kps, rbox, DF);
     for (int S = 1; S <= 8; ++S) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
-      // the weighted-sum GEMM over <= 1024 entries: its split-K reduction and
-      // activation epilogue (measured ~4 us per round) outweigh the shorter
-      // main loop, so it runs unsplit
-      if (S > 1 && EPI == kEpiAct && kb_total <= 16) break;
+      // the weighted-sum GEMM over <= 1024 entries: when its tiles already
+      // fill half the GPU, the split-K reduction and activation epilogue
+      // (measured ~4 us per round) outweigh the shorter main loop, so it
+      // runs unsplit
+      if (S > 1 && EPI == kEpiAct && kb_total <= 16 && 2 * tiles >= sms) break;
       const int nst = (su_total + S - 1) / S;
       const long long ctas = tiles * S;
       // the accumulator tile [rows][BN + 4] fp32 (and after it, for kEpiAct

@@ -91,7 +91,7 @@ struct SelectSmem {
   float warp_tot_f[kSelWarps];
   int warp_tot[kSelWarps];
   int warp_first[kSelWarps];
-  unsigned int red_u[2][kSelWarps];
+  unsigned int red_u[kSelWarps];
   unsigned int sh_digit, sh_above;
   int sh_cnt_gt, sh_first;
   float sh_max, sh_sum;
@@ -135,11 +135,18 @@ __device__ __forceinline__ void select_stats(float lmax, float lsum, SelectSmem&
   sumexp = sm.sh_sum;
 }
 
+// The score a key was made from (ord_key inverted).
+__device__ __forceinline__ float key_score(unsigned long long key) {
+  const uint32_t k = (uint32_t)(key >> 32);
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
 // Orders the C (<= FOVEA_MAX_K) distinct keys of sm.cand descending, in
-// place: a histogram of the keys' score words over kWideBins bins (the bin is
-// monotone in the key), an exclusive scan of the bins, a scatter of the keys
-// into bin order (sm.sorted), and each key's rank among the keys of its own
-// bin.  The histogram lives in sm.cum (dead until the mass scan).
+// place: a histogram of the candidates' scores over kOrderBins bins of equal
+// width between their maximum and minimum (the bin is monotone in the score),
+// an exclusive scan of the bins, a scatter of the keys into bin order
+// (sm.sorted), and each key's rank among the keys of its own bin.  The
+// histogram lives in sm.cum (dead until the mass scan).
 constexpr int kOrderBins = 1024;
 static_assert(kOrderBins <= FOVEA_MAX_K && kOrderBins == 4 * kSelThreads, "bins in SelectSmem::cum");
 
@@ -147,28 +154,33 @@ template <class Sync>
 __device__ void bucket_order(SelectSmem& sm, int C, int tid, Sync sync) {
   const int lane = tid & 31, warp = tid >> 5;
   unsigned int* hist = reinterpret_cast<unsigned int*>(sm.cum);
-  uint32_t kmax = 0u, kmin = 0xFFFFFFFFu;
+  float smax = -INFINITY, smin = INFINITY;
   for (int c = tid; c < C; c += kSelThreads) {
-    const uint32_t k = (uint32_t)(sm.cand[c] >> 32);
-    kmax = max(kmax, k);
-    kmin = min(kmin, k);
+    const float v = key_score(sm.cand[c]);
+    smax = fmaxf(smax, v);
+    smin = fminf(smin, v);
   }
-  kmax = __reduce_max_sync(0xffffffffu, kmax);
-  kmin = __reduce_min_sync(0xffffffffu, kmin);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    smax = fmaxf(smax, __shfl_xor_sync(0xffffffffu, smax, o));
+    smin = fminf(smin, __shfl_xor_sync(0xffffffffu, smin, o));
+  }
   for (int i = tid; i < kOrderBins; i += kSelThreads) hist[i] = 0u;
   if (lane == 0) {
-    sm.red_u[0][warp] = kmax;
-    sm.red_u[1][warp] = kmin;
+    sm.red_m[warp] = smax;
+    sm.red_lo[warp] = smin;
   }
   sync();
 #pragma unroll
   for (int w = 0; w < kSelWarps; ++w) {
-    kmax = max(kmax, sm.red_u[0][w]);
-    kmin = min(kmin, sm.red_u[1][w]);
+    smax = fmaxf(smax, sm.red_m[w]);
+    smin = fminf(smin, sm.red_lo[w]);
   }
-  const unsigned long long span = (unsigned long long)(kmax - kmin) + 1ull;
+  const float range = smax - smin;
+  const float inv_w = range > 0.0f ? (float)(kOrderBins - 1) / range : 0.0f;
   auto bin_of = [&](unsigned long long key) {
-    return (int)(((unsigned long long)(kmax - (uint32_t)(key >> 32)) * kOrderBins) / span);
+    const int b = (int)((smax - key_score(key)) * inv_w);
+    return b < 0 ? 0 : (b > kOrderBins - 1 ? kOrderBins - 1 : b);
   };
   for (int c = tid; c < C; c += kSelThreads) atomicAdd(&hist[bin_of(sm.cand[c])], 1u);
   sync();
@@ -185,10 +197,10 @@ __device__ void bucket_order(SelectSmem& sm, int C, int tid, Sync sync) {
     const unsigned int t = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += t;
   }
-  if (lane == 31) sm.red_u[0][warp] = incl;
+  if (lane == 31) sm.red_u[warp] = incl;
   sync();
   unsigned int run = incl - tot;
-  for (int w = 0; w < warp; ++w) run += sm.red_u[0][w];
+  for (int w = 0; w < warp; ++w) run += sm.red_u[w];
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     hist[4 * tid + j] = run;                       // start of the bin
