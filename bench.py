@@ -697,14 +697,20 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
     ws = fovea.lm_head_workspace(vocab, d, N, k_c)
     logits = torch.empty((N, vocab), dtype=torch.float32, device=h_hat.device)
     ms = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits), flush, n_steps)
+    ms_c = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, write_logits=False), flush, n_steps)
     fovea.sync_errors(ws)
-    # algorithmic bytes: W_LM once, h_hat in, the logits out and back in for
-    # the candidate selection, the candidates out
-    nbytes = vocab * d * 2 + N * d * 2 + 2 * N * vocab * 4 + N * k_c * 8
+    # algorithmic bytes: W_LM once, h_hat in, the logits out (first form
+    # only), the per-tile candidates out and back in for the merge, the
+    # K_c candidates (index, value) out
+    tiles = (vocab + 255) // 256
+    base = vocab * d * 2 + N * d * 2 + 2 * N * tiles * k_c * 8 + N * k_c * 8
+    nbytes = base + N * vocab * 4
     gbs = nbytes / (ms / 1000.0) / 1e9
     del W, logits
     return {"vocab": vocab, "d_model": d, "draft_states": N, "k_c": k_c, "us_per_call": 1000 * ms,
             "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"],
+            "candidates_only": {"us_per_call": 1000 * ms_c, "algorithmic_bytes": base,
+                                "frac_of_measured_hbm": base / (ms_c / 1000.0) / 1e9 / peaks["hbm_gbs"]},
             "steps": n_steps, "w_lm": "synthetic N(0, 1/d), bf16"}
 
 

@@ -285,7 +285,9 @@ FOVEA_API fovea_status fovea_noalloc_sync_errors(void* stream);
  * index.
  *   W_LM      [vocab, d_model] device, dtype, row-major (16-byte aligned)
  *   h_hat     [N, d_model] device, dtype (e.g. fovea_retrieve_fuse's h_out)
- *   logits    [N, vocab] device fp32, caller-owned: z (written)
+ *   logits    [N, vocab] device fp32, caller-owned: z (written), or NULL
+ *             when only the candidates are wanted (the 4 N vocab bytes of
+ *             logits are then not written)
  *   top_idx   [N, k_c] device int32: token indices (written)
  *   top_val   [N, k_c] device fp32: their logits (or NULL)
  *   workspace device memory of fovea_lm_head_workspace_size bytes (256-byte

@@ -1024,7 +1024,6 @@ FOVEA_API fovea_status fovea_lm_head_topk(const void* W_LM, int vocab, int d_mod
   if (vocab < k_c) return fail(FOVEA_ERR_INVALID_ARG, "vocab %d < k_c %d", vocab, k_c);
   NEED_PTR(W_LM, "W_LM");
   NEED_PTR(h_hat, "h_hat");
-  NEED_PTR(logits, "logits");
   if (top_idx == nullptr) return fail(FOVEA_ERR_INVALID_ARG, "top_idx is NULL");
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(FOVEA_ERR_INVALID_ARG, "workspace is NULL or not 256-byte aligned");

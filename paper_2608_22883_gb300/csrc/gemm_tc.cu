@@ -603,8 +603,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             act_store4(args, g, m0 + cc, n0 + rr, vals, addt + 4 * it, bias_s + cc,
                        min(4, n_cols - cc));
           } else if constexpr (EPI == kEpiLogits) {
-            gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc),
-                                       bias_s + cc);
+            if (args.out2 != nullptr)               // the logits, when asked for
+              gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc),
+                                         bias_s + cc);
           } else {
             gemm_epilogue4<EPI>(args, g, m0 + cc, n0 + rr, vals, min(4, n_cols - cc), bias_s + cc);
           }
@@ -703,8 +704,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else if constexpr (EPI == kEpiLogits) {
               const int it = it0 + k * kThreads;
               *reinterpret_cast<float4*>(sums + 4 * it) = acc[k];
-              gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc[k], n0 + rr[k], vals,
-                                         min(4, n_cols - cc[k]), bias_s + cc[k]);
+              if (args.out2 != nullptr)
+                gemm_epilogue4<kEpiQueryH>(args, g, m0 + cc[k], n0 + rr[k], vals,
+                                           min(4, n_cols - cc[k]), bias_s + cc[k]);
             } else {
               gemm_epilogue4<EPI>(args, g, m0 + cc[k], n0 + rr[k], vals, min(4, n_cols - cc[k]),
                                   bias_s + cc[k]);

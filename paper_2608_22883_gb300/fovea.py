@@ -340,18 +340,23 @@ def lm_head_workspace(vocab: int, d_model: int, N: int, k_c: int, stream=None) -
 
 
 def lm_head_topk(W_LM: torch.Tensor, h_hat: torch.Tensor, k_c: int, workspace: torch.Tensor,
-                 logits: Optional[torch.Tensor] = None, stream=None):
+                 logits: Optional[torch.Tensor] = None, stream=None, write_logits: bool = True):
     """fovea_lm_head_topk: z = h_hat W_LM^T [N, V] (fp32) and the k_c largest
     logits per row (token indices, values), descending, smaller index first
-    on ties.  Returns (top_idx [N, k_c] int32, top_val [N, k_c], logits)."""
+    on ties.  Returns (top_idx [N, k_c] int32, top_val [N, k_c], logits);
+    with write_logits=False the logits are not written (NULL) and None is
+    returned in their place."""
     V, d = W_LM.shape
     N = h_hat.shape[0]
     dt = BF16 if W_LM.dtype == torch.bfloat16 else FP32
-    if logits is None:
+    if not write_logits:
+        logits = None
+    elif logits is None:
         logits = torch.empty((N, V), dtype=torch.float32, device=h_hat.device)
     idx = torch.empty((N, k_c), dtype=torch.int32, device=h_hat.device)
     val = torch.empty((N, k_c), dtype=torch.float32, device=h_hat.device)
-    _check(lib().fovea_lm_head_topk(_ptr(W_LM), V, d, dt, _ptr(h_hat), N, k_c, _ptr(logits),
+    _check(lib().fovea_lm_head_topk(_ptr(W_LM), V, d, dt, _ptr(h_hat), N, k_c,
+                                    _ptr(logits) if logits is not None else None,
                                     _ptr(idx), _ptr(val), _ptr(workspace), workspace.numel(),
                                     _stream(stream)))
     return idx, val, logits

@@ -72,11 +72,12 @@ def test_lm_head_topk_matches_oracle(fovea, V, d, N, k_c, seed):
     check(fovea, V, d, N, k_c, seed)
 
 
-def test_lm_head_exact_ties_take_the_smaller_index(fovea):
+@pytest.mark.parametrize("k_c", [32, 6])   # the warp-reduction and the register paths
+def test_lm_head_exact_ties_take_the_smaller_index(fovea, k_c):
     # rows 3, V/2 and V-1 of W_LM are equal: whenever one of them is among the
     # candidates, so are the others in index order (equal logits, equal keys)
     V, d, N = 600, 128, 24
-    idx = check(fovea, V, d, N, 32, 5, ties=True)
+    idx = check(fovea, V, d, N, k_c, 5, ties=True)
     for n in range(N):
         lst = idx[n].tolist()
         pos = [lst.index(j) for j in (3, V // 2, V - 1) if j in lst]
@@ -86,3 +87,19 @@ def test_lm_head_exact_ties_take_the_smaller_index(fovea):
 def test_lm_head_vicuna_sized(fovea):
     # a 32000-token vocabulary over d = 4096, 64 draft states, K_c = 6
     check(fovea, 32000, 4096, 64, 6, 6)
+
+
+def test_lm_head_candidates_without_logits(fovea):
+    """logits = NULL: the candidates are those of the call that writes the
+    logits, bit for bit."""
+    g = np.random.default_rng(8)
+    V, d, N, k_c = 3000, 512, 40, 6
+    Wt = bf16(g.standard_normal((V, d)) / np.sqrt(d)).cuda()
+    ht = bf16(g.standard_normal((N, d))).cuda()
+    ws = fovea.lm_head_workspace(V, d, N, k_c)
+    idx1, val1, logits = fovea.lm_head_topk(Wt, ht, k_c, ws)
+    idx2, val2, none = fovea.lm_head_topk(Wt, ht, k_c, ws, write_logits=False)
+    torch.cuda.synchronize()
+    fovea.sync_errors(ws)
+    assert none is None and logits is not None
+    assert torch.equal(idx1, idx2) and torch.equal(val1, val2)
