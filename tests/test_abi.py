@@ -168,7 +168,6 @@ def call_lm_head(L, *, W=0x10000, V=1000, d=256, dtype=fovea.BF16, h=0x10000, N=
     (dict(N=-1), fovea.ERR_INVALID_ARG),
     (dict(W=None), fovea.ERR_INVALID_ARG),
     (dict(h=0x10004), fovea.ERR_INVALID_ARG),        # misaligned
-    (dict(logits=None), fovea.ERR_INVALID_ARG),
     (dict(idx=None), fovea.ERR_INVALID_ARG),
     (dict(ws=0x10010), fovea.ERR_INVALID_ARG),       # not 256-byte aligned
     (dict(ws_bytes=1024), fovea.ERR_INVALID_ARG),
