@@ -613,7 +613,7 @@ def main():
                                            min(args.steps, 300))
         if w.dtype == "bf16" and w.B == 1:
             out["supplemental"]["lm_head_topk_v32000_k6"] = lm_head_point(
-                fovea, h_out, flush, min(args.steps, 300), peaks)
+                fovea, h_out, flush, min(args.steps, 300), peaks, step=step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, rows, secs, build_s = time_oracle(w, args.cpu_seconds)
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
@@ -685,11 +685,14 @@ def supplemental(fovea, params, mem, w, h, depth, row_scale, flush, n_steps):
     return out
 
 
-def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=7):
+def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=7, step=None):
     """The draft logits and K_c candidates (fovea_lm_head_topk) on the step's
     own h_hat: a synthetic bf16 W_LM [vocab, d] ~ N(0, 1/d), drawn on the
     device from a seeded generator; one plain call per step, L2 flushed
-    before each, CUDA events on the launching stream."""
+    before each, CUDA events on the launching stream.  With `step` (the
+    draft step writing h_hat), also the step followed by the LM head on the
+    same stream in one timed region: the LM head's weight stream starts while
+    the step's last kernel runs (programmatic dependent launch)."""
     N, d = h_hat.shape
     gen = torch.Generator(device=h_hat.device)
     gen.manual_seed(seed)
@@ -698,6 +701,15 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
     logits = torch.empty((N, vocab), dtype=torch.float32, device=h_hat.device)
     ms = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits), flush, n_steps)
     ms_c = _time_calls(lambda: fovea.lm_head_topk(W, h_hat, k_c, ws, write_logits=False), flush, n_steps)
+    after = None
+    if step is not None:
+        def step_then_head():
+            step()
+            fovea.lm_head_topk(W, h_hat, k_c, ws, logits=logits)
+        ms_s = _time_calls(step, flush, n_steps)
+        ms_sh = _time_calls(step_then_head, flush, n_steps)
+        after = {"us_step": 1000 * ms_s, "us_step_then_lm_head": 1000 * ms_sh,
+                 "us_lm_head_after_step": 1000 * (ms_sh - ms_s)}
     fovea.sync_errors(ws)
     # algorithmic bytes: W_LM once, h_hat in, the logits out (first form
     # only), the per-tile candidates out and back in for the merge, the
@@ -709,6 +721,7 @@ def lm_head_point(fovea, h_hat, flush, n_steps, peaks, vocab=32000, k_c=6, seed=
     del W, logits
     return {"vocab": vocab, "d_model": d, "draft_states": N, "k_c": k_c, "us_per_call": 1000 * ms,
             "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"],
+            "after_step": after,
             "candidates_only": {"us_per_call": 1000 * ms_c, "algorithmic_bytes": base,
                                 "frac_of_measured_hbm": base / (ms_c / 1000.0) / 1e9 / peaks["hbm_gbs"]},
             "steps": n_steps, "w_lm": "synthetic N(0, 1/d), bf16"}
