@@ -63,6 +63,7 @@ constexpr int kSmemBudget = 200 * 1024;   // shared-memory stages, one CTA per S
 constexpr int kSmemBudgetPair = 100 * 1024;  // two CTAs per SM
 constexpr int kSmemExtra = 1024 /*alignment*/ + 256 /*barriers*/ + 1024 /*tile biases*/;
 constexpr int kMaxStages = 8;
+constexpr int kRasterRows = 16;          // row tiles per band of the tile order
 
 // BN features per tile; DUAL: the row stage holds two tiles (hi and lo parts
 // of the row operand), and each feature tile is multiplied by both into the
@@ -257,13 +258,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int s1 = min(args.a_split, g.m);
   const int s2 = max(s1, min(args.a_split2, g.m));
   const int t0 = (s1 + BN - 1) / BN, t1 = (s2 - s1 + BN - 1) / BN, t2 = (g.m - s2 + BN - 1) / BN;
-  const int tx = (int)blockIdx.x / S;
+  // Tile order: with one group and no split, consecutive CTAs walk
+  // kRasterRows row tiles per feature tile, so that a wave of resident CTAs
+  // shares both operands through L2 (in feature-fastest order every wave
+  // re-reads all feature tiles from HBM).
+  int bx = (int)blockIdx.x, by = (int)blockIdx.y;
+  if (S == 1 && gridDim.z == 1 && (int)gridDim.y > kRasterRows) {
+    const int FX = (int)gridDim.x;
+    const int L = bx + FX * by;
+    const int sr = L / (kRasterRows * FX);
+    const int rows_here = min(kRasterRows, (int)gridDim.y - sr * kRasterRows);
+    const int local = L - sr * kRasterRows * FX;
+    by = sr * kRasterRows + local % rows_here;
+    bx = local / rows_here;
+  }
+  const int tx = bx / S;
   if (tx >= t0 + t1 + t2) return;
   const int part = tx < t0 ? 0 : (tx < t0 + t1 ? 1 : 2);
   const int pbeg = part == 0 ? 0 : (part == 1 ? s1 : s2);
   const int m0 = pbeg + (tx - (part == 0 ? 0 : (part == 1 ? t0 : t0 + t1))) * BN;
   const int m_end = part == 0 ? s1 : (part == 1 ? s2 : g.m);
-  const int n0 = blockIdx.y * BM;
+  const int n0 = by * BM;
   if (m0 >= m_end || n0 >= g.n) return;
 
   // folded scores: the folded keys (part 0) are a hi / lo pair of bf16 values,
