@@ -979,7 +979,19 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
   const int kb_total = a.k_total / tc::BK;
   const int r_split_kb = a.b_split / tc::BK;
   const long long ftiles = feature_tiles(a, max_m, BN);
-  const long long tiles = ftiles * row_tiles;
+  const long long tiles = ftiles * row_tiles;          // the grid (every group sized to the largest)
+  // tiles with work: groups of ragged sizes leave the rest of their grid
+  // slots empty (those CTAs exit at once), so the cost counts these
+  long long active = 0;
+  for (int gi = 0; gi < a.ngroups; ++gi)
+    active += (long long)feature_tiles(a, a.groups[gi].m, BN) *
+              ((a.groups[gi].n + tc::BM - 1) / tc::BM);
+  if (active <= 0 || active > tiles) active = tiles;
+  // the same at the narrowest feature tile: the parallelism the GEMM has
+  long long active64 = 0;
+  for (int gi = 0; gi < a.ngroups; ++gi)
+    active64 += (long long)feature_tiles(a, a.groups[gi].m, 64) *
+                ((a.groups[gi].n + tc::BM - 1) / tc::BM);
   const int rows = max_n < tc::BM ? max_n : tc::BM;
   // rows of a row tile: >= 64 so that the MMA's 128-row read stays inside its stage
   const int rbox = std::max(64, std::min(tc::BM, (max_n + 7) / 8 * 8));
@@ -994,13 +1006,13 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
     const int sb = C::stage_bytes(kps, rbox, DF);
     for (int S = 1; S <= 8; ++S) {
       if (S > 1 && (EPI == kEpiStoreKeys || S > su_total)) break;
-      // the weighted-sum GEMM over <= 1024 entries: when its tiles already
-      // fill half the GPU, the split-K reduction and activation epilogue
-      // (measured ~4 us per round) outweigh the shorter main loop, so it
-      // runs unsplit
-      if (S > 1 && EPI == kEpiAct && kb_total <= 16 && 2 * tiles >= sms) break;
+      // the weighted-sum GEMM over <= 1024 entries: when its narrowest tiles
+      // already fill half the GPU, the split-K reduction and activation
+      // epilogue (measured ~4 us per round) outweigh the shorter main loop,
+      // so it runs unsplit
+      if (S > 1 && EPI == kEpiAct && kb_total <= 16 && 2 * active64 >= sms) break;
       const int nst = (su_total + S - 1) / S;
-      const long long ctas = tiles * S;
+      const long long ctas = active * S;
       // the accumulator tile [rows][BN + 4] fp32 (and after it, for kEpiAct
       // the added term, for split kEpiLogits the reduced logits, [rows][BN])
       const int staging = EPI == kEpiStoreKeys ? rows * (BN * 2 + 16)
@@ -1023,7 +1035,7 @@ static void plan_for(const GemmArgs& a, int max_m, int max_n, long long row_tile
         const double t = plan_cost_us(streaming, sb / 1024.0, stage_f,
                                       stage_mma_us, stages, nst, std::min(ctas, cap), (int)per_sm,
                                       waves, S);
-        if (t < best_t - 1e-6 || (t < best_t + 1e-6 && ctas < best.tiles * best.splits)) {
+        if (t < best_t - 1e-6 || (t < best_t + 1e-6 && tiles * S < best.tiles * best.splits)) {
           best_t = t;
           best = GemmPlan{BN, S, stages, 0, tiles, rbox, region, kps};
         }
