@@ -1,4 +1,4 @@
-// Row helpers shared by the row kernels and the persistent step kernel:
+// Row helpers shared by the row kernels (LN, readout, finalize):
 // 16-byte vector loads of a row segment, the double-float warp sum, and the
 // single rounding of a double-float value to the stored type.
 #pragma once
