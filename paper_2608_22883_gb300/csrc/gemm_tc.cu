@@ -48,6 +48,9 @@
 // previous kernel, so the weight stream starts while the predecessor drains.
 #include <atomic>
 #include <cstring>
+#include <cstdio>
+#include <string>
+#include <unordered_map>
 
 #include "gemm_epilogue.cuh"
 #include "tc_ptx.cuh"
@@ -802,6 +805,40 @@ static bool make_map3(CUtensorMap* m, const TmaOperand& op, int box_rows, int kp
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Encoded maps of this thread, by their parameters: a tensor map is a pure
+// function of (base, shape, row stride, box), so a draft step that runs with
+// the same buffers reuses its maps instead of encoding ~10 per call.
+struct MapKey {
+  const void* base;
+  long long rows, cols, ld;
+  int box_rows, kps;
+  bool operator==(const MapKey& o) const {
+    return base == o.base && rows == o.rows && cols == o.cols && ld == o.ld &&
+           box_rows == o.box_rows && kps == o.kps;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& k) const {
+    size_t h = std::hash<const void*>()(k.base);
+    for (long long v : {k.rows, k.cols, k.ld, (long long)k.box_rows, (long long)k.kps})
+      h = h * 1000003u ^ std::hash<long long>()(v);
+    return h;
+  }
+};
+static bool cached_map3(CUtensorMap* m, const TmaOperand& op, int box_rows, int kps) {
+  static thread_local std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  const MapKey key{op.base, op.rows, op.cols, op.ld, box_rows, kps};
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *m = it->second;
+    return true;
+  }
+  if (!make_map3(m, op, box_rows, kps)) return false;
+  if (cache.size() >= 512) cache.clear();          // bounded: many distinct buffers
+  cache.emplace(key, *m);
+  return true;
+}
+
 bool encode_bf16_map(CUtensorMap* m, const void* base, long long rows, long long cols,
                      long long ld, int box_rows) {
   return make_map(m, TmaOperand{base, rows, cols, ld}, box_rows);
@@ -1055,7 +1092,7 @@ static GemmPlan plan_epi(const GemmArgs& a, int max_m, int max_n) {
   return best;
 }
 
-GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
+static GemmPlan plan_gemm_tc_uncached(int epi, const GemmArgs& a, int max_m, int max_n) {
   switch (epi) {
     case kEpiStore: return plan_epi<kEpiStore>(a, max_m, max_n);
     case kEpiScores: return plan_epi<kEpiScores>(a, max_m, max_n);
@@ -1068,6 +1105,28 @@ GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
     case kEpiLogits: return plan_epi<kEpiLogits>(a, max_m, max_n);
     default: return plan_epi<kEpiBiasF32>(a, max_m, max_n);
   }
+}
+
+// Plans of this thread, by the arguments the planner reads (a draft step
+// plans the same few GEMMs on every call).
+GemmPlan plan_gemm_tc(int epi, const GemmArgs& a, int max_m, int max_n) {
+  static thread_local std::unordered_map<std::string, GemmPlan> cache;
+  std::string key;
+  key.reserve(64 + 16 * a.ngroups);
+  char buf[160];
+  snprintf(buf, sizeof buf, "%d|%d|%d|%d|%d|%d|%d|%d|%d|", epi, max_m, max_n, a.k_total, a.b_split,
+           a.a_split, a.a_split2, a.f_lo_kb, a.ngroups);
+  key += buf;
+  for (int g = 0; g < a.ngroups; ++g) {
+    snprintf(buf, sizeof buf, "%d,%d;", a.groups[g].m, a.groups[g].n);
+    key += buf;
+  }
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  const GemmPlan p = plan_gemm_tc_uncached(epi, a, max_m, max_n);
+  if (cache.size() >= 256) cache.clear();
+  cache.emplace(key, p);
+  return p;
 }
 
 int lm_head_slots(int vocab, int d_model, int N) {
@@ -1106,9 +1165,9 @@ cudaError_t launch_gemm_tc(int epi, const GemmArgs& args, const TmaOperand& A0, 
   const TmaOperand& a1 = A1.base ? A1 : A0;
   const TmaOperand& a2 = A2.base ? A2 : a1;
   const TmaOperand& b1 = B1.base ? B1 : B0;
-  if (!make_map3(&maps[0], A0, plan.bn, plan.kps) || !make_map3(&maps[1], a1, plan.bn, plan.kps) ||
-      !make_map3(&maps[2], a2, plan.bn, plan.kps) || !make_map3(&maps[3], B0, plan.rbox, plan.kps) ||
-      !make_map3(&maps[4], b1, plan.rbox, plan.kps))
+  if (!cached_map3(&maps[0], A0, plan.bn, plan.kps) || !cached_map3(&maps[1], a1, plan.bn, plan.kps) ||
+      !cached_map3(&maps[2], a2, plan.bn, plan.kps) || !cached_map3(&maps[3], B0, plan.rbox, plan.kps) ||
+      !cached_map3(&maps[4], b1, plan.rbox, plan.kps))
     return cudaErrorInvalidValue;
   const int tiles_x = feature_tiles(a, max_m, plan.bn);
   switch (epi) {
