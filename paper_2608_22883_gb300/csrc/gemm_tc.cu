@@ -151,10 +151,161 @@ __device__ __forceinline__ uint32_t logit_order_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// Compare-exchange: a keeps the larger key, b the smaller.
+__device__ __forceinline__ void cx_desc(uint32_t& a, uint32_t& b) {
+  const uint32_t hi = max(a, b);
+  b = min(a, b);
+  a = hi;
+}
+
+// Sorts 8 keys into descending order (odd-even merge network, 19
+// compare-exchanges).
+__device__ __forceinline__ void sort8_desc(uint32_t& x0, uint32_t& x1, uint32_t& x2, uint32_t& x3,
+                                           uint32_t& x4, uint32_t& x5, uint32_t& x6, uint32_t& x7) {
+  cx_desc(x0, x1); cx_desc(x2, x3); cx_desc(x4, x5); cx_desc(x6, x7);
+  cx_desc(x0, x2); cx_desc(x1, x3); cx_desc(x4, x6); cx_desc(x5, x7);
+  cx_desc(x1, x2); cx_desc(x5, x6);
+  cx_desc(x0, x4); cx_desc(x1, x5); cx_desc(x2, x6); cx_desc(x3, x7);
+  cx_desc(x2, x4); cx_desc(x3, x5);
+  cx_desc(x1, x2); cx_desc(x3, x4); cx_desc(x5, x6);
+}
+
+constexpr int kTopkPer = 16;                 // candidates listed per thread by the threshold pass
+constexpr int kTopkLd = 4 * kTopkPer + 1;    // a row's lists (rows of a warp on distinct banks)
+
+// kEpiLogits for cand_k <= 8, the threshold form.  Four threads per row,
+// thread q taking columns q, q + 4, ... (consecutive lanes on consecutive
+// banks).  Pass 1: each thread's two largest order keys; the k-th largest of
+// the row's eight is a lower bound T on the row's k-th largest key (they are
+// eight of the row's keys).  Pass 2: each thread lists its keys >= T, as
+// 64-bit candidate keys, in its own part of the row's list in shared memory
+// (a handful per row; eight loads in flight before any store).  Pass 3: each
+// listed key's rank is its count of larger listed keys (the keys are
+// distinct), and ranks below k are the row's candidates, in order; slots past
+// the row's columns hold 0.  Integer work per element: three min / max, one
+// compare.  Returns false, having written nothing that the caller's fallback
+// does not overwrite, when a thread lists more than kTopkPer keys (many equal
+// logits) or the scratch is too small.
+template <int BN>
+__device__ __forceinline__ bool tile_topk_threshold(const GemmArgs& a, long long row0,
+                                                    int rows_real, const float* vals, int ld,
+                                                    int col0, int ncols, int slot,
+                                                    uint8_t* scratch, int scratch_bytes) {
+  constexpr int kRows = kThreads / 4;              // rows per pass
+  constexpr int kB = 8;                            // columns per thread and batch
+  const int k = a.cand_k;
+  if (scratch_bytes < kRows * kTopkLd * 8 + 16) return false;
+  unsigned long long* list = reinterpret_cast<unsigned long long*>(scratch);
+  int* overflow = reinterpret_cast<int*>(scratch + kRows * kTopkLd * 8);
+  const int q = threadIdx.x & 3;
+  const int lr = (int)(threadIdx.x >> 2);          // the row within a pass
+  if (threadIdx.x == 0) *overflow = 0;
+  __syncthreads();
+  const uint32_t list_s = smem_u32(list);
+  for (int rbase = 0; rbase < rows_real; rbase += kRows) {
+    const int rr = rbase + lr;
+    const bool real = rr < rows_real;
+    const uint32_t row_s = smem_u32(vals) + (uint32_t)(rr * ld) * 4u;
+    // pass 1: this thread's two largest keys
+    uint32_t m1 = 0u, m2 = 0u;
+    if (real) {
+      for (int c0 = q; c0 < ncols; c0 += 4 * kB) {
+        uint32_t x[kB];
+#pragma unroll
+        for (int u = 0; u < kB; ++u) {
+          const int c = c0 + 4 * u;
+          x[u] = c < ncols ? logit_order_key(lds_f32(row_s + 4u * (uint32_t)c)) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < kB; ++u) {
+          m2 = max(m2, min(m1, x[u]));
+          m1 = max(m1, x[u]);
+        }
+      }
+    }
+    uint32_t v0 = m1, v1 = m2;
+    uint32_t v2 = __shfl_xor_sync(0xffffffffu, m1, 1);
+    uint32_t v3 = __shfl_xor_sync(0xffffffffu, m2, 1);
+    uint32_t v4 = __shfl_xor_sync(0xffffffffu, v0, 2);
+    uint32_t v5 = __shfl_xor_sync(0xffffffffu, v1, 2);
+    uint32_t v6 = __shfl_xor_sync(0xffffffffu, v2, 2);
+    uint32_t v7 = __shfl_xor_sync(0xffffffffu, v3, 2);
+    sort8_desc(v0, v1, v2, v3, v4, v5, v6, v7);
+    uint32_t T = k <= 1 ? v0 : k == 2 ? v1 : k == 3 ? v2 : k == 4 ? v3 :
+                 k == 5 ? v4 : k == 6 ? v5 : k == 7 ? v6 : v7;
+    T = max(T, 1u);                                // a zero key is never a candidate
+    // pass 2: this thread's keys >= T, in a short list of its own
+    const uint32_t lst_s = list_s + (uint32_t)(lr * kTopkLd) * 8u;
+    const uint32_t own_s = lst_s + (uint32_t)(q * kTopkPer) * 8u;
+    int mine = 0;
+    if (real) {
+      for (int c0 = q; c0 < ncols; c0 += 4 * kB) {
+        uint32_t x[kB];
+#pragma unroll
+        for (int u = 0; u < kB; ++u) {
+          const int c = c0 + 4 * u;
+          x[u] = c < ncols ? logit_order_key(lds_f32(row_s + 4u * (uint32_t)c)) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < kB; ++u) {           // branch-free: a predicated store
+          const uint32_t hit = x[u] >= T ? 1u : 0u;
+          sts_u64_if(own_s + 8u * (uint32_t)min(mine, kTopkPer - 1),
+                     ((unsigned long long)x[u] << 32) |
+                         (0xFFFFFFFFu - (uint32_t)col0 - (uint32_t)(c0 + 4 * u)),
+                     hit & (mine < kTopkPer ? 1u : 0u));
+          mine += (int)hit;
+        }
+      }
+    }
+    // the row's lists packed in thread order at the front of its list area
+    // (read into registers first: a list may move onto another's place)
+    int incl = mine;                               // prefix over the row's four threads
+    int up = __shfl_up_sync(0xffffffffu, incl, 1);
+    incl += q >= 1 ? up : 0;
+    up = __shfl_up_sync(0xffffffffu, incl, 2);
+    incl += q >= 2 ? up : 0;
+    const int before = incl - mine;
+    int total = __shfl_xor_sync(0xffffffffu, mine, 1) + mine;
+    total += __shfl_xor_sync(0xffffffffu, total, 2);
+    const int over = __shfl_xor_sync(0xffffffffu, mine > kTopkPer ? 1 : 0, 1) | (mine > kTopkPer);
+    const bool overflowed = (over | __shfl_xor_sync(0xffffffffu, over, 2)) != 0;
+    unsigned long long held[kTopkPer];
+#pragma unroll
+    for (int j = 0; j < kTopkPer; ++j)
+      held[j] = j < mine && !overflowed ? lds_u64(own_s + 8u * (uint32_t)j) : 0ull;
+    __syncwarp();
+    if (!overflowed) {
+#pragma unroll
+      for (int j = 0; j < kTopkPer; ++j)
+        if (j < mine) sts_u64(lst_s + 8u * (uint32_t)(before + j), held[j]);
+    }
+    __syncwarp();
+    // pass 3: ranks within the row's list
+    if (real) {
+      if (overflowed) {
+        *overflow = 1;
+      } else {
+        unsigned long long* dst = a.cand + (row0 + rr) * a.cand_ld + (long long)slot * k;
+        for (int j = q; j < total; j += 4) {
+          const unsigned long long key = lds_u64(lst_s + 8u * (uint32_t)j);
+          int rank = 0;
+          for (int i = 0; i < total; ++i) rank += lds_u64(lst_s + 8u * (uint32_t)i) > key ? 1 : 0;
+          if (rank < k) dst[rank] = key;
+        }
+        for (int j = total + q; j < k; j += 4) dst[j] = 0ull;
+      }
+    }
+    __syncwarp();
+  }
+  __syncthreads();
+  return *overflow == 0;
+}
+
 // kEpiLogits: per row of the tile, the cand_k largest of `ncols` logits
 // (vals [rows_real][ld] in shared memory, column c is token col0 + c) into
 // the row's candidate slot as 64-bit keys, logit order key << 32 | ~token
-// (on equal logits the smaller token is larger).  One warp per row, each lane
+// (on equal logits the smaller token is larger).  Up to 8 candidates the
+// threshold form above; otherwise (or when it gives up) one warp per row, each lane
 // holding the order keys of columns lane, lane + 32, ...; each of the k rounds
 // takes the lane maxima (the smallest column on equal keys), a warp maximum,
 // the smallest column holding it (warp minimum), and clears that key: short,
@@ -163,7 +314,10 @@ __device__ __forceinline__ uint32_t logit_order_key(float f) {
 template <int BN>
 __device__ __forceinline__ void tile_topk(const GemmArgs& a, long long row0, int rows_real,
                                           const float* vals, int ld, int col0, int ncols,
-                                          int slot) {
+                                          int slot, uint8_t* scratch, int scratch_bytes) {
+  if (a.cand_k <= 8 && tile_topk_threshold<BN>(a, row0, rows_real, vals, ld, col0, ncols, slot,
+                                               scratch, scratch_bytes))
+    return;
   constexpr int J = (BN + 31) / 32;
   constexpr int R = 4;                       // rows a warp works on together (independent chains)
   constexpr int kWarps = kThreads / 32;
@@ -295,8 +449,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int stage_bytes = C::stage_bytes(KPS, rbox, dual_f);
   const int stages = dual_f ? max(1, min(args.stages, args.region / stage_bytes)) : args.stages;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
+  // the 1024-byte aligned base, derived from smem_raw by pointer arithmetic
+  // so that the compiler keeps every access through it in the shared space
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   // stage st: row tiles at smem + st * stage_bytes, feature tiles r_bytes later
   // barriers after the ring, or after the partial-tile staging area when that
   // is larger (split K)
@@ -630,7 +785,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if constexpr (EPI == kEpiLogits)
-        tile_topk<BN>(args, (long long)g.b_row0 + n0, rows_real, part, ldp, m0, n_cols, tx);
+        tile_topk<BN>(args, (long long)g.b_row0 + n0, rows_real, part, ldp, m0, n_cols, tx,
+                      reinterpret_cast<uint8_t*>(part + rows_real * ldp),
+                      args.region - rows_real * ldp * 4);
     } else {
       // Split K: each CTA stages its fp32 partial tile row-major [rows][BN + 4]
       // over its idle ring (the pitch spreads a warp's 16-byte stores over all
@@ -739,7 +896,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if constexpr (EPI == kEpiLogits) {
         __syncthreads();
         tile_topk<BN>(args, (long long)g.b_row0 + n0, rows_real, sums, q4 * 4, m0 + qlo * 4,
-                      max(0, min(q4 * 4, n_cols - qlo * 4)), tx * S + (int)rank);
+                      max(0, min(q4 * 4, n_cols - qlo * 4)), tx * S + (int)rank,
+                      reinterpret_cast<uint8_t*>(sums + rows_real * q4 * 4),
+                      args.region - (rows_real * ldp + rows_real * q4 * 4) * 4);
       }
       cluster_wait();   // no CTA leaves while another still reads its partial tile
     }

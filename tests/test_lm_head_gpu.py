@@ -67,12 +67,15 @@ def check(fovea, V, d, N, k_c, seed, ties=False):
     (777, 320, 5, 32, 2),        # the widest candidate list
     (4099, 192, 130, 1, 3),      # argmax; rows over two row tiles
     (50, 64, 1, 6, 4),           # one row, a vocabulary smaller than a tile
+    (2000, 256, 70, 8, 9),       # the widest per-thread candidate list
+    (2000, 256, 70, 9, 10),      # the narrowest warp-round list
 ])
 def test_lm_head_topk_matches_oracle(fovea, V, d, N, k_c, seed):
     check(fovea, V, d, N, k_c, seed)
 
 
-@pytest.mark.parametrize("k_c", [32, 6])   # the warp-reduction and the register paths
+# k_c > 8: one warp per row and K_c warp rounds; k_c <= 8: per-thread lists
+@pytest.mark.parametrize("k_c", [32, 9, 8, 6])
 def test_lm_head_exact_ties_take_the_smaller_index(fovea, k_c):
     # rows 3, V/2 and V-1 of W_LM are equal: whenever one of them is among the
     # candidates, so are the others in index order (equal logits, equal keys)
@@ -82,6 +85,30 @@ def test_lm_head_exact_ties_take_the_smaller_index(fovea, k_c):
         lst = idx[n].tolist()
         pos = [lst.index(j) for j in (3, V // 2, V - 1) if j in lst]
         assert pos == sorted(pos)
+
+
+@pytest.mark.parametrize("k_c", [6, 8, 12])
+def test_lm_head_many_equal_largest_logits(fovea, k_c):
+    """Twenty equal vocabulary rows, across a 256-column tile boundary, hold
+    every row's largest logit: the candidates are the k_c smallest of those
+    token indices, in index order, all with the same logit."""
+    g = np.random.default_rng(11)
+    V, d, N = 1000, 128, 33
+    W = g.standard_normal((V, d)) / np.sqrt(d)
+    W[246:266] = 4.0 / np.sqrt(d)             # far above every other logit for h > 0
+    h = np.abs(g.standard_normal((N, d))) + 0.1
+    Wt, ht = bf16(W).cuda(), bf16(h).cuda()
+    ws = fovea.lm_head_workspace(V, d, N, k_c)
+    idx, val, logits = fovea.lm_head_topk(Wt, ht, k_c, ws)
+    torch.cuda.synchronize()
+    fovea.sync_errors(ws)
+    ref = oracle.lm_head_topk(Wt.double().cpu().numpy(), ht.double().cpu().numpy(), k_c)
+    want = np.tile(np.arange(246, 246 + k_c, dtype=np.int32), (N, 1))
+    assert np.array_equal(ref["top_idx"], want)
+    assert np.array_equal(idx.cpu().numpy(), want)
+    v = val.cpu().numpy()
+    assert np.all(v == v[:, :1])
+    assert np.array_equal(v[:, 0], logits.cpu().numpy()[:, 246])
 
 
 def test_lm_head_vicuna_sized(fovea):
