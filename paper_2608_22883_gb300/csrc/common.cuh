@@ -150,7 +150,8 @@ enum EpiKind : int {
   kEpiLogits = 9,        // the draft logits: out2 (fp32)[row * ldc2 + col] = acc, and per row
                          // the cand_k largest of the CTA's columns as 64-bit keys (logit order
                          // key << 32 | ~column) into cand[row * cand_ld + slot * cand_k + r],
-                         // slot = feature tile * splits + rank
+                         // slot = feature tile * splits + rank, r = 0, 1, ... in descending
+                         // key order (zeros last: fewer columns than cand_k)
 };
 
 struct KeyFix {       // one listed key element: memory row, feature

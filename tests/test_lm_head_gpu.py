@@ -87,15 +87,17 @@ def test_lm_head_exact_ties_take_the_smaller_index(fovea, k_c):
         assert pos == sorted(pos)
 
 
-@pytest.mark.parametrize("k_c", [6, 8, 12])
-def test_lm_head_many_equal_largest_logits(fovea, k_c):
-    """Twenty equal vocabulary rows, across a 256-column tile boundary, hold
-    every row's largest logit: the candidates are the k_c smallest of those
-    token indices, in index order, all with the same logit."""
+# 20 equal rows: a few per thread of a tile's threshold pass; 100: more than
+# a thread's list holds in the second tile, so that tile takes the warp rounds
+@pytest.mark.parametrize("k_c,block", [(6, 20), (8, 20), (12, 20), (6, 100), (8, 100)])
+def test_lm_head_many_equal_largest_logits(fovea, k_c, block):
+    """Equal vocabulary rows 246 .. 246 + block - 1, across a 256-column tile
+    boundary, hold every row's largest logit: the candidates are the k_c
+    smallest of those token indices, in index order, all with one logit."""
     g = np.random.default_rng(11)
     V, d, N = 1000, 128, 33
     W = g.standard_normal((V, d)) / np.sqrt(d)
-    W[246:266] = 4.0 / np.sqrt(d)             # far above every other logit for h > 0
+    W[246:246 + block] = 4.0 / np.sqrt(d)     # far above every other logit for h > 0
     h = np.abs(g.standard_normal((N, d))) + 0.1
     Wt, ht = bf16(W).cuda(), bf16(h).cuda()
     ws = fovea.lm_head_workspace(V, d, N, k_c)
